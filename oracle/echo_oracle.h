@@ -1,0 +1,54 @@
+/*
+ * echo_oracle.h -- TEST INFRASTRUCTURE ONLY: the CPU oracle's own declarations.
+ * Nothing in the product library includes this file.
+ */
+#ifndef ECHO_ORACLE_H
+#define ECHO_ORACLE_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum { ORACLE_OK = 0, ORACLE_E_INVALID = 1, ORACLE_E_DEADLOCK = 2, ORACLE_E_NOMEM = 3 };
+
+typedef struct {
+  int64_t n_ops;
+  int32_t n_ranks, n_streams, gpus_per_node, n_groups;
+  const uint8_t *kind, *kclass, *cc_type, *cc_algo;
+  const int32_t *group;
+  const int64_t *cc_bytes;
+  const int64_t *pred_off;
+  const int32_t *pred_idx;
+  const int64_t *q_off; /* [n_ranks*n_streams+1]; queue r*n_streams+k */
+  const int32_t *q_ops;
+  const int64_t *grp_off;
+  const int32_t *grp_rank;
+} oracle_graph;
+
+typedef struct {
+  int32_t n_scen, n_kclass, n_chunk;
+  const int64_t *dur; /* [n_ops][n_scen] */
+  const double *alpha_ns, *bw_intra, *lat_intra, *bw_inter, *lat_inter, *delta; /* [n_scen] */
+  const double *slowdown;                                                      /* [n_kclass][n_scen] */
+  const int64_t *chunk_max_bytes, *chunk_bytes; /* [n_chunk]; n_chunk = 0 -> Table 6 */
+} oracle_scen;
+
+int64_t oracle_chunk_bytes(int64_t nbytes, int n_chunk, const int64_t *max_bytes,
+                           const int64_t *chunk_bytes);
+
+/* prm = {alpha_ns, bw_intra, lat_intra, bw_inter, lat_inter, delta} */
+double oracle_cc_ns(int cc_type, int cc_algo, int64_t nbytes, int N, int M, int K, double lg,
+                    const double *prm, int n_chunk, const int64_t *max_bytes,
+                    const int64_t *chunk_bytes);
+
+/* Composes scenarios [s0, s1).  Outputs are [n_ops][n_scen] (only the columns in
+ * range are written); any output pointer may be NULL. */
+int oracle_compose(const oracle_graph *g, const oracle_scen *sc, int32_t s0, int32_t s1,
+                   int32_t refine_passes, uint64_t tie_seed, int64_t *start, int64_t *finish,
+                   int64_t *makespan, double *cc_ns, uint8_t *overlapped);
+
+#ifdef __cplusplus
+}
+#endif
+#endif
