@@ -1,0 +1,341 @@
+"""Benchmark of the batched timeline composer on GB300.
+
+Workload: the GPT-175B Megatron-shaped step (96 ranks, TP8 PP6 DP2, 16 micro-batches
+1F1B, ~1.1M ops) composed for 1024 what-if scenarios per GPU.  One step = the whole
+hot path over that batch: CC estimation for every collective x scenario, the first
+composition, the overlap test and the second (slowdown-adjusted) composition.
+
+metric: node x scenario timeline updates per second (each compose pass updates
+every op in every scenario, so one step is 2 * V * S updates), plus the achieved
+HBM bandwidth of the compose kernel against the measured GB300 copy peak.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl echo|reference]
+Under torchrun each rank composes its own 1024 scenarios (weak scaling, no
+collective on the data path); the step time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "node×scenario timeline updates/sec and achieved HBM GB/s vs GB300 peak"
+UNIT = "updates/s"
+WORKLOAD = "gpt175b"
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "compose_gpt175b.md")
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def dist_env():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), \
+        int(os.environ.get("LOCAL_RANK", "0"))
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index=None):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            cmd = ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits", "-lms", "100"]
+            if self.index is not None:
+                cmd[1:1] = ["-i", str(self.index)]
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(cmd, stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception as ex:  # pragma: no cover
+            log("clock sampling unavailable:", ex)
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:  # pragma: no cover
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons, power = [], [], set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            p = [x.strip() for x in line.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                mx.append(float(p[2]))
+                power.append(float(p[3]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, p[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm), "power_w_max": max(power) if power else None}
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    with open(os.path.join(ROOT, "paper_2412_12487_gb300", "csrc", "echo_kernels.cu"), "rb") as f:
+        h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(launch_units):
+    """DRAM bytes per compose launch from the committed ncu summary, scaled to
+    ``launch_units`` node-scenarios, if it was taken on the current kernel source."""
+    try:
+        text = open(PROFILE_SUMMARY).read()
+    except OSError:
+        return None
+    m_hash = re.search(r"kernel source sha256\[:16\]:\s*([0-9a-f]{16})", text)
+    m_bytes = re.search(r"dram bytes per node-scenario \(compose\):\s*([0-9.]+)", text)
+    if not m_hash or not m_bytes or m_hash.group(1) != kernel_source_hash():
+        return None
+    return float(m_bytes.group(1)) * launch_units
+
+
+def build_inputs(rank, pinned=True):
+    import torch
+    from paper_2412_12487_gb300 import workloads as W
+    c = W.config(WORKLOAD)
+    c = W.GPTConfig(**{**c.__dict__, "scen_seed": c.scen_seed + 7919 * rank})
+    t0 = time.time()
+    g = W.build_gpt_graph(c)
+    sc = W.scenario_params(c)
+    V, S = g.n_ops, sc.n_scen
+    dur_t = torch.empty((V, S), dtype=torch.int64, pin_memory=pinned)
+    W.durations(g, sc.peak_flop_per_ns, out=dur_t.numpy())
+    log(f"[rank {rank}] inputs: V={V} S={S} dur={V * S * 8 / 1e9:.2f} GB ({time.time() - t0:.1f}s)")
+    return c, g, sc, dur_t
+
+
+def algorithmic_bytes_per_pass(g, info, S):
+    from paper_2412_12487_gb300 import workloads as W
+    v_cd = int(((g.kind == W.KIND_COMPUTE) | (g.kind == W.KIND_MEMCPY)).sum())
+    v_comm = g.n_ops - v_cd
+    graph = 8 * (g.n_ops + 1) + 4 * g.n_edges + 4 * g.n_ops
+    return S * (16 * v_cd + 8 * v_comm) + graph + 16 * info["n_signatures"] * S
+
+
+def run_echo(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2412_12487_gb300 import Echo
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    c, g, sc, dur_t = build_inputs(rank)
+    V, S = g.n_ops, sc.n_scen
+    stream = torch.cuda.current_stream()
+    e = Echo(local, stream)
+    t0 = time.time()
+    e.load_graph(g)
+    e.load_scenarios(sc, dur=dur_t)
+    info = e.info()
+    log(f"[rank {rank}] loaded in {time.time() - t0:.1f}s: {info}")
+
+    def step():
+        e.estimate_collectives()
+        e.compose(refine_passes=1)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    clocks = Clocks(local if world == 1 else None)
+    # device-resident timing
+    e.set_profiling(True)
+    e.read_profile()
+    barrier()
+    clocks.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    barrier()
+    clk = clocks.stop()
+    prof = e.read_profile()
+    e.set_profiling(False)
+    ms = ev0.elapsed_time(ev1) / args.steps
+    # end-to-end through the public API: host (pinned) durations in, makespans out
+    mk_host = torch.empty(S, dtype=torch.int64, pin_memory=True)
+
+    def e2e_step():
+        e.load_scenarios(sc, dur=dur_t)
+        e.estimate_collectives()
+        e.compose(refine_passes=1)
+        e.read_makespan(out=mk_host.numpy())
+
+    for _ in range(2):
+        e2e_step()
+    e2e_steps = max(3, min(args.steps, 10))
+    barrier()
+    ev0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    ev1.record(stream)
+    barrier()
+    e2e_ms = ev0.elapsed_time(ev1) / e2e_steps
+
+    t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms, e2e_ms = float(t[0]), float(t[1])
+    units = 2 * V * S  # two compose passes per step
+    value = units * world / (ms / 1e3)
+    e2e_value = units * world / (e2e_ms / 1e3)
+
+    comp_launches, comp_ms = prof.get("compose", (0, 0.0))
+    launches = sum(n for n, _ in prof.values())
+    peak, peak_kind = measured_peaks()
+    b_pass = algorithmic_bytes_per_pass(g, info, S)
+    per_launch_ms = comp_ms / max(comp_launches, 1)
+    achieved = b_pass / (per_launch_ms / 1e3) / 1e9 if comp_launches else None
+    traffic = profiled_traffic(V * S)
+    out = None
+    if rank == 0:
+        cpu = cpu_baseline(g, c, args) if world == 1 else None
+        h2d = V * S * 8 + 6 * S * 8 + sc.slowdown.size * 8
+        out = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": f"{c.name} x {S} scenarios per GPU", "ops": V, "edges": g.n_edges,
+                       "levels": info["n_levels"], "scenarios_per_gpu": S, "refine_passes": 1,
+                       "sigma": info["sigma"],
+                       "updates_per_step": units,
+                       "l2": f"no flush: the {V * S * 8 / 1e9:.1f} GB duration matrix and the "
+                             f"finish matrices each exceed the 129 MB L2"},
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": S * 8,
+                    "ms_per_step": e2e_ms},
+            "gpu_launches": launches,
+            "kernels": {k: {"launches": n, "ms_per_launch": t_ / max(n, 1)} for k, (n, t_) in prof.items()},
+            "roofline": {"kernel": "compose", "bound": "hbm", "achieved": achieved, "peak": peak,
+                         "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+                         "unit": "GB/s", "frac": (achieved / peak) if achieved else None,
+                         "traffic": traffic, "alg_bytes_per_launch": b_pass},
+            "clocks": clk,
+            "cpu_baseline": cpu,
+        }
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    e.close()
+    return out
+
+
+def cpu_baseline(g, c, args, n_sample=None):
+    """The CPU oracle as it stands, single-threaded, on a bounded sample of the
+    same workload (the first scenarios of the batch)."""
+    import oracle
+    from paper_2412_12487_gb300 import workloads as W
+    n_sample = n_sample or args.cpu_sample
+    sub = W.select_scenarios(W.scenario_params(c), g, list(range(n_sample)))
+    t0 = time.time()
+    oracle.compose(g, sub, refine_passes=1, threads=1, want_cc=False, want_overlap=False)
+    dt = time.time() - t0
+    return {"value": 2 * g.n_ops * n_sample / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{n_sample} of the {c.n_scen} scenarios of {c.name} ({g.n_ops} ops), "
+                      f"CC estimate + 2 compositions + overlap, {dt:.1f} s single-threaded",
+            "seconds": dt, "host_cores_available": os.cpu_count()}
+
+
+def run_reference(args):
+    """Reference arm: the CPU oracle (a plain event-driven simulator written from
+    the paper) timed on the host cores on the same workload, one scenario per step."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return None
+    import oracle
+    from paper_2412_12487_gb300 import workloads as W
+    c = W.config(WORKLOAD)
+    g = W.build_gpt_graph(c)
+    base = W.scenario_params(c)
+    oracle.build()
+
+    def step(i):
+        sub = W.select_scenarios(base, g, [i % base.n_scen])
+        oracle.compose(g, sub, refine_passes=1, threads=1, want_cc=False, want_overlap=False)
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.time()
+    for i in range(args.steps):
+        step(args.warmup + i)
+    dt = (time.time() - t0) / args.steps
+    v = 2 * g.n_ops / dt
+    return {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": f"{c.name} x 1 scenario per step (bounded sample of the "
+                                   f"{c.n_scen}-scenario batch)", "ops": g.n_ops},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": "one scenario per step, single-threaded"},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="echo", choices=["echo", "reference"])
+    ap.add_argument("--cpu-sample", type=int, default=8)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "echo":
+        log("note: warmup raised to 3")
+        args.warmup = 3
+    if args.impl == "reference":
+        out = run_reference(args)
+    else:
+        import __graft_entry__
+        __graft_entry__.build()
+        out = run_echo(args)
+    if out is not None:
+        print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,222 @@
+/*
+ * echo.h -- C ABI of the GB300 (sm_103a) timeline composer for Echo-style
+ * distributed-training simulation (arXiv 2412.12487).
+ *
+ * One context owns one device, one CUDA stream and all device memory it uses.
+ * The calls follow the paper's statement of the problem:
+ *
+ *   echo_load_graph            per-rank execution graphs merged into one graph (Sec. 4.1-4.2)
+ *   echo_load_scenarios        what-if parameters: kernel durations, link parameters,
+ *                              slowdown factors (Sec. 3 inputs, Sec. 5.3 parameters)
+ *   echo_estimate_collectives  CC estimator: sync join + execution closed forms (Sec. 5.2-5.3)
+ *   echo_compose               timeline composer (Sec. 4.2) + validator adjustment (Sec. 3, 6)
+ *   echo_read_*                per-op start/finish, step makespan, CC estimates
+ *
+ * Conventions for every call:
+ *   - The return value is an echo_status; ECHO_OK (0) on success.  On failure the
+ *     context keeps its previous state and echo_last_error() describes the cause.
+ *   - Array arguments are caller-owned HOST memory unless stated otherwise.  They
+ *     are read (or written) during the call only; nothing keeps a pointer to them.
+ *     Pinned (page-locked) host memory makes the copies faster but is not required.
+ *   - Op ids are the caller's ids 0..n_ops-1.  The library renumbers internally
+ *     and never exposes its own numbering.
+ *   - Times are int64 nanoseconds; the first op of every timeline may start at 0.
+ *   - A context is not thread-safe.  Different contexts are independent.
+ *   - Calls must come in order: graph -> scenarios -> estimate -> compose -> read.
+ *     Loading a new graph invalidates the scenarios; loading new scenarios
+ *     invalidates the estimates and the composition.  Out of order: ECHO_E_STATE.
+ *   - Work is enqueued on the context's stream.  echo_load_*, echo_estimate_collectives
+ *     and echo_read_* synchronize with that stream before returning (they report
+ *     input errors found on the device); echo_compose only enqueues.
+ */
+#ifndef ECHO_H
+#define ECHO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ECHO_ABI_VERSION 1
+
+typedef enum {
+  ECHO_OK = 0,
+  ECHO_E_INVALID_ARG = 1, /* null pointer, bad size, negative duration, bad parameter */
+  ECHO_E_BAD_GRAPH = 2,   /* index out of range, inconsistent timelines or groups     */
+  ECHO_E_CYCLE = 3,       /* the dependencies (data + issue order) form a cycle        */
+  ECHO_E_STATE = 4,       /* call made out of order                                    */
+  ECHO_E_OOM = 5,         /* device or host allocation failed                          */
+  ECHO_E_CUDA = 6,        /* a CUDA runtime call failed                                */
+  ECHO_E_TIMEOUT = 7,     /* a bounded device-side wait gave up                        */
+  ECHO_E_OVERFLOW = 8,    /* a finish time could exceed the int64 range                */
+  ECHO_E_UNSUPPORTED = 9  /* a size beyond what this build supports                    */
+} echo_status;
+
+/* op kinds (Sec. 4.2 timelines: computation, communication, memcpy) */
+enum { ECHO_OP_COMPUTE = 0, ECHO_OP_MEMCPY = 1, ECHO_OP_COLL = 2, ECHO_OP_P2P = 3 };
+/* collective types of Sec. 5.3 (send/recv is the P2P primitive of Sec. 5.2) */
+enum { ECHO_CC_ALLREDUCE = 0, ECHO_CC_ALLGATHER = 1, ECHO_CC_REDUCESCATTER = 2, ECHO_CC_SENDRECV = 3 };
+/* all-reduce algorithm (Sec. 5.1: NCCL runs ring or tree all-reduce; AUTO = the faster) */
+enum { ECHO_ALGO_RING = 0, ECHO_ALGO_TREE = 1, ECHO_ALGO_AUTO = 2 };
+
+typedef struct echo_ctx echo_ctx;
+
+/*
+ * Multi-rank execution graph (Sec. 4.1: per-rank graphs of compute and comm ops;
+ * Sec. 4.2: inter-rank dependency and matching rules, given here as shared comm
+ * nodes and explicit data edges).
+ *
+ * Timelines: every rank r has n_streams serial timelines ("streams").  Queue
+ * q = r * n_streams + k lists, in issue order, the ops rank r runs on its stream k.
+ *   - stream 0 is the rank's compute timeline: it holds exactly the rank's
+ *     ECHO_OP_COMPUTE ops and nothing else;
+ *   - streams 1..n_streams-1 are communication / memcpy timelines;
+ *   - a COMPUTE or MEMCPY op appears in exactly one queue;
+ *   - a COLL or P2P op appears exactly once on every member rank of its group
+ *     (in any stream >= 1 of that rank) and on no other rank.
+ * An op starts when, on each of its timelines, the op issued before it has
+ * finished, and all its data predecessors have finished (Sec. 5.2: a collective
+ * starts when its last member launches; a P2P op waits for its peer).  Its finish
+ * is start + duration.
+ */
+typedef struct {
+  int64_t n_ops;           /* V >= 0                                                   */
+  int32_t n_ranks;         /* >= 1                                                      */
+  int32_t n_streams;       /* timelines per rank, 1..16                                 */
+  int32_t gpus_per_node;   /* ranks r and r' share a node iff r/gpus_per_node equal     */
+  int32_t n_groups;        /* communicator groups                                      */
+  const uint8_t *kind;     /* [V] ECHO_OP_*                                             */
+  const uint8_t *kclass;   /* [V] compute ops: kernel class = row of the slowdown table */
+  const int32_t *group;    /* [V] COLL/P2P ops: group index; ignored for other kinds    */
+  const uint8_t *cc_type;  /* [V] COLL: ALLREDUCE/ALLGATHER/REDUCESCATTER; P2P: SENDRECV */
+  const uint8_t *cc_algo;  /* [V] all-reduce ops: ECHO_ALGO_*; ignored otherwise        */
+  const int64_t *cc_bytes; /* [V] comm ops: message size in bytes (>= 0)                */
+  const int64_t *pred_off; /* [V+1] CSR of data dependencies, pred_off[0] = 0           */
+  const int32_t *pred_idx; /* [pred_off[V]] predecessor op ids                          */
+  const int64_t *q_off;    /* [n_ranks*n_streams+1] CSR of the timelines, q_off[0] = 0  */
+  const int32_t *q_ops;    /* [q_off[n_ranks*n_streams]] op ids in issue order          */
+  const int64_t *grp_off;  /* [n_groups+1] CSR of group members, grp_off[0] = 0         */
+  const int32_t *grp_rank; /* [grp_off[n_groups]] member ranks, no repeats; P2P: 1 or 2 */
+} echo_graph_desc;
+
+/*
+ * S what-if scenarios.  All arrays are host memory; dur is row-major [V][S]
+ * (scenario index innermost).  Link parameters feed the CC estimator of Sec. 5.3:
+ * bandwidths in bytes/ns (= GB/s), latencies and alpha (connection setup) in ns,
+ * delta (reduction cost) in ns per byte.  slowdown[c][s] is the factor of
+ * Sec. 2.3 for a compute op of kernel class c that overlaps communication in
+ * scenario s; it stands in for the XGBoost predictor of Sec. 6.
+ */
+typedef struct {
+  int32_t n_scen;                  /* S >= 1                                          */
+  int32_t n_kclass;                /* rows of slowdown; > every compute op's kclass   */
+  int32_t n_chunk;                 /* entries of the chunk table, 0 = Table 6 default */
+  const int64_t *dur;              /* [V][S] ns >= 0; entries of COLL/P2P ops ignored */
+  const double *alpha_ns;          /* [S] >= 0                                        */
+  const double *bw_intra;          /* [S] > 0, intra-node link                        */
+  const double *lat_intra;         /* [S] >= 0                                        */
+  const double *bw_inter;          /* [S] > 0, inter-node link                        */
+  const double *lat_inter;         /* [S] >= 0                                        */
+  const double *delta;             /* [S] >= 0                                        */
+  const double *slowdown;          /* [n_kclass][S], each in (0, 1e6]                  */
+  const int64_t *chunk_max_bytes;  /* [n_chunk] ascending: messages <= max use ...    */
+  const int64_t *chunk_bytes;      /* [n_chunk] ... this chunk size (> 0); larger
+                                      messages use the last entry                     */
+} echo_scen_desc;
+
+typedef struct {
+  /* validator passes after the first composition (Sec. 3: compose, then adjust the
+   * overlapped ops).  0 = compose only; 1 = the paper's flow (default); k > 1
+   * recomputes the overlap from pass k's times and always slows the ORIGINAL
+   * durations.  At most 8. */
+  int32_t refine_passes;
+} echo_compose_opts;
+
+/* Create a context on `device`, enqueuing on `cuda_stream` (a cudaStream_t; NULL =
+ * a new non-blocking stream owned by the context). */
+int echo_create(echo_ctx **out, int device, void *cuda_stream);
+/* Free everything the context owns.  NULL is accepted. */
+int echo_destroy(echo_ctx *ctx);
+
+/* Host-only check of a graph: the validation and topological levelling that
+ * echo_load_graph performs, without a device.  Writes the number of levels and
+ * the widest level (either pointer may be NULL). */
+int echo_check_graph(const echo_graph_desc *g, int64_t *n_levels, int64_t *max_width);
+
+/* Validate, level (ASAP depth over data + issue-order dependencies), renumber in
+ * level order and upload the graph.  Errors: ECHO_E_INVALID_ARG, ECHO_E_BAD_GRAPH,
+ * ECHO_E_CYCLE, ECHO_E_UNSUPPORTED, ECHO_E_OOM, ECHO_E_CUDA. */
+int echo_load_graph(echo_ctx *ctx, const echo_graph_desc *g);
+
+/* Copy the scenarios to the device (durations permuted into the internal order)
+ * and check them: negative durations -> ECHO_E_INVALID_ARG. */
+int echo_load_scenarios(echo_ctx *ctx, const echo_scen_desc *sc);
+
+/* CC estimator (Sec. 5.2-5.3): for every comm op and scenario, the execution time
+ * of Eqs. 2-5 (ring all-gather, ring reduce-scatter, ring/tree/auto all-reduce,
+ * send/recv) in fp64 ns; the op's duration is that value rounded to the nearest
+ * integer (ties to even).  Group shape: N members, M distinct nodes, K = the
+ * largest member count on one node, log2(M) computed on the host.  A time that
+ * could overflow the composition -> ECHO_E_OVERFLOW. */
+int echo_estimate_collectives(echo_ctx *ctx);
+
+/* Timeline composer (Sec. 4.2) over all scenarios, then `refine_passes` validator
+ * passes (Sec. 3, 2.3): a compute op whose [start, finish) interval overlaps, with
+ * positive length, the interval of a comm op its rank takes part in gets duration
+ * rint(d * slowdown[kclass][s]) and the timeline is composed again.  Only
+ * enqueues work; opts may be NULL (refine_passes = 1). */
+int echo_compose(echo_ctx *ctx, const echo_compose_opts *opts);
+
+/* Final start and finish of ops [op0, op1) (caller ids), all scenarios, into host
+ * buffers of (op1-op0)*S int64 each, row-major [op][s].  Either may be NULL. */
+int echo_read_times(echo_ctx *ctx, int64_t op0, int64_t op1, int64_t *start, int64_t *finish);
+/* Step time per scenario: the largest finish time (0 for an empty graph). [S] */
+int echo_read_makespan(echo_ctx *ctx, int64_t *makespan);
+/* CC estimates (fp64 ns) of ops [op0, op1), [op][s]; NaN for non-comm ops. */
+int echo_read_cc(echo_ctx *ctx, int64_t op0, int64_t op1, double *cc_ns);
+/* Validator decisions of the last pass for ops [op0, op1), [op][s]: 1 = slowed. */
+int echo_read_overlap(echo_ctx *ctx, int64_t op0, int64_t op1, uint8_t *overlapped);
+
+/* Standalone CC estimator queries (Sec. 5.3), one fp64 time per query. */
+typedef struct {
+  int64_t n;                /* number of queries                                    */
+  const uint8_t *cc_type;   /* [n] ECHO_CC_*                                        */
+  const uint8_t *cc_algo;   /* [n] all-reduce: ECHO_ALGO_*                          */
+  const int64_t *nbytes;    /* [n] >= 0                                             */
+  const int32_t *n_ranks;   /* [n] N >= 1                                           */
+  const int32_t *n_nodes;   /* [n] 1 <= M <= N; K = ceil(N/M) (most even layout)    */
+  const double *alpha_ns, *bw_intra, *lat_intra, *bw_inter, *lat_inter, *delta; /* [n] */
+  int32_t n_chunk;          /* chunk table as in echo_scen_desc (0 = Table 6)       */
+  const int64_t *chunk_max_bytes, *chunk_bytes;
+} echo_cc_query_desc;
+int echo_cc_query(echo_ctx *ctx, const echo_cc_query_desc *q, double *out_ns);
+
+/* Shape of the loaded graph (after echo_load_graph). */
+typedef struct {
+  int64_t n_ops, n_edges, n_levels, max_width, n_queue_entries, n_comm_ops, n_signatures;
+  int32_t n_ranks, n_streams, sigma; /* sigma: scenarios per thread block of the composer */
+} echo_graph_info;
+int echo_graph_info_get(echo_ctx *ctx, echo_graph_info *info);
+
+/* Kernel timing with CUDA events on the context's stream.  While enabled, every
+ * kernel the library launches is bracketed by two events.  echo_read_profile
+ * synchronizes, reports per kernel name the launches and total milliseconds
+ * since the last read (up to `cap` entries, count in *n) and clears the record. */
+typedef struct {
+  char name[48];
+  int64_t launches;
+  double total_ms;
+} echo_kernel_stat;
+int echo_set_profiling(echo_ctx *ctx, int enable);
+int echo_read_profile(echo_ctx *ctx, echo_kernel_stat *out, int cap, int *n);
+
+const char *echo_strerror(int status);
+/* Copies the context's last error message (NUL-terminated) into buf. */
+int echo_last_error(echo_ctx *ctx, char *buf, size_t n);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ECHO_H */

@@ -1,0 +1,983 @@
+// echo_host.cpp -- host side of the C ABI declared in include/echo.h: input
+// validation, topological levelling and renumbering, collective-signature dedup,
+// device memory, kernel launches and readback.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <new>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "echo.h"
+#include "echo_internal.h"
+
+using echo::CcSig;
+using echo::ChunkTable;
+
+namespace {
+
+// Table 6 of the paper (Sec. 8.3): chunk size per tensor size, MB read as MiB.
+const int64_t kDefaultMax[5] = {4LL << 20, 8LL << 20, 64LL << 20, 128LL << 20, INT64_MAX};
+const int64_t kDefaultChunk[5] = {18000, 36000, 72000, 144000, 288000};
+
+struct Err {
+  int code = ECHO_OK;
+  std::string msg;
+};
+
+int fail(Err &e, int code, const char *fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  e.code = code;
+  e.msg = buf;
+  return code;
+}
+
+// Everything derived from a graph on the host.
+struct GraphBuild {
+  int64_t V = 0, E = 0, QE = 0, L = 0, max_width = 0;
+  int32_t R = 0, NS = 0, gpn = 1;
+  std::vector<int32_t> int2ext, ext2int;
+  std::vector<int64_t> lvl_off;
+  std::vector<int64_t> nq_off;
+  std::vector<int32_t> nq;
+  std::vector<int64_t> dp_off;
+  std::vector<int32_t> dp;
+  std::vector<uint8_t> kcl, is_comm, local;
+  std::vector<int64_t> q_off;
+  std::vector<int32_t> q_ops_int;
+  std::vector<CcSig> sigs;
+  std::vector<int32_t> sig_count, comm_node, comm_sig, node_sig;
+  int32_t max_kclass = -1;
+};
+
+bool finite_nonneg(double x) { return std::isfinite(x) && x >= 0.0; }
+
+int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
+  if (!g) return fail(e, ECHO_E_INVALID_ARG, "graph descriptor is NULL");
+  const int64_t V = g->n_ops;
+  if (V < 0 || V >= INT32_MAX) return fail(e, ECHO_E_INVALID_ARG, "n_ops %lld out of range", (long long)V);
+  if (g->n_ranks < 1 || g->n_ranks > 65535)
+    return fail(e, ECHO_E_UNSUPPORTED, "n_ranks %d outside [1, 65535]", g->n_ranks);
+  if (g->n_streams < 1 || g->n_streams > echo::kMaxStreams)
+    return fail(e, ECHO_E_UNSUPPORTED, "n_streams %d outside [1, %d]", g->n_streams, echo::kMaxStreams);
+  if (g->gpus_per_node < 1) return fail(e, ECHO_E_INVALID_ARG, "gpus_per_node must be >= 1");
+  if (g->n_groups < 0) return fail(e, ECHO_E_INVALID_ARG, "n_groups must be >= 0");
+  const int32_t R = g->n_ranks, NS = g->n_streams;
+  const int64_t NQ = (int64_t)R * NS;
+  if (!g->pred_off || !g->q_off) return fail(e, ECHO_E_INVALID_ARG, "pred_off and q_off are required");
+  if (V > 0 && (!g->kind || !g->kclass || !g->group || !g->cc_type || !g->cc_algo || !g->cc_bytes))
+    return fail(e, ECHO_E_INVALID_ARG, "per-op arrays are required when n_ops > 0");
+  if (g->n_groups > 0 && (!g->grp_off || !g->grp_rank))
+    return fail(e, ECHO_E_INVALID_ARG, "grp_off/grp_rank are required when n_groups > 0");
+
+  // data dependencies
+  if (g->pred_off[0] != 0) return fail(e, ECHO_E_BAD_GRAPH, "pred_off[0] must be 0");
+  for (int64_t v = 0; v < V; ++v)
+    if (g->pred_off[v + 1] < g->pred_off[v]) return fail(e, ECHO_E_BAD_GRAPH, "pred_off decreases at op %lld", (long long)v);
+  const int64_t E = g->pred_off[V];
+  if (E > 0 && !g->pred_idx) return fail(e, ECHO_E_INVALID_ARG, "pred_idx is NULL");
+  if (E >= INT32_MAX) return fail(e, ECHO_E_UNSUPPORTED, "too many edges");
+  for (int64_t v = 0; v < V; ++v)
+    for (int64_t k = g->pred_off[v]; k < g->pred_off[v + 1]; ++k) {
+      int32_t u = g->pred_idx[k];
+      if (u < 0 || u >= V) return fail(e, ECHO_E_BAD_GRAPH, "op %lld: predecessor %d out of range", (long long)v, u);
+      if (u == v) return fail(e, ECHO_E_CYCLE, "op %lld depends on itself", (long long)v);
+    }
+  // groups
+  std::vector<std::vector<int32_t>> members(g->n_groups);
+  if (g->n_groups > 0) {
+    if (g->grp_off[0] != 0) return fail(e, ECHO_E_BAD_GRAPH, "grp_off[0] must be 0");
+    for (int32_t gi = 0; gi < g->n_groups; ++gi) {
+      if (g->grp_off[gi + 1] < g->grp_off[gi]) return fail(e, ECHO_E_BAD_GRAPH, "grp_off decreases at group %d", gi);
+      for (int64_t k = g->grp_off[gi]; k < g->grp_off[gi + 1]; ++k) {
+        int32_t r = g->grp_rank[k];
+        if (r < 0 || r >= R) return fail(e, ECHO_E_BAD_GRAPH, "group %d: rank %d out of range", gi, r);
+        members[gi].push_back(r);
+      }
+      std::sort(members[gi].begin(), members[gi].end());
+      if (std::adjacent_find(members[gi].begin(), members[gi].end()) != members[gi].end())
+        return fail(e, ECHO_E_BAD_GRAPH, "group %d repeats a rank", gi);
+      if (members[gi].empty()) return fail(e, ECHO_E_BAD_GRAPH, "group %d is empty", gi);
+    }
+  }
+  // ops
+  int32_t max_kc = -1;
+  for (int64_t v = 0; v < V; ++v) {
+    uint8_t k = g->kind[v];
+    if (k > ECHO_OP_P2P) return fail(e, ECHO_E_BAD_GRAPH, "op %lld: kind %d", (long long)v, k);
+    if (k == ECHO_OP_COMPUTE) {
+      if (g->kclass[v] == echo::kNotSlowable) return fail(e, ECHO_E_BAD_GRAPH, "op %lld: kclass 255 is reserved", (long long)v);
+      max_kc = std::max<int32_t>(max_kc, g->kclass[v]);
+    }
+    if (k == ECHO_OP_COLL || k == ECHO_OP_P2P) {
+      int32_t gi = g->group[v];
+      if (gi < 0 || gi >= g->n_groups) return fail(e, ECHO_E_BAD_GRAPH, "op %lld: group %d out of range", (long long)v, gi);
+      if (g->cc_bytes[v] < 0) return fail(e, ECHO_E_INVALID_ARG, "op %lld: negative message size", (long long)v);
+      uint8_t t = g->cc_type[v];
+      if (k == ECHO_OP_P2P) {
+        if (t != ECHO_CC_SENDRECV) return fail(e, ECHO_E_BAD_GRAPH, "op %lld: P2P op needs cc_type SENDRECV", (long long)v);
+        if (members[gi].size() > 2) return fail(e, ECHO_E_BAD_GRAPH, "op %lld: P2P group has more than 2 ranks", (long long)v);
+      } else {
+        if (t > ECHO_CC_REDUCESCATTER) return fail(e, ECHO_E_BAD_GRAPH, "op %lld: collective cc_type %d", (long long)v, t);
+        if (t == ECHO_CC_ALLREDUCE && g->cc_algo[v] > ECHO_ALGO_AUTO)
+          return fail(e, ECHO_E_BAD_GRAPH, "op %lld: cc_algo %d", (long long)v, g->cc_algo[v]);
+      }
+    }
+  }
+  // timelines
+  if (g->q_off[0] != 0) return fail(e, ECHO_E_BAD_GRAPH, "q_off[0] must be 0");
+  for (int64_t q = 0; q < NQ; ++q)
+    if (g->q_off[q + 1] < g->q_off[q]) return fail(e, ECHO_E_BAD_GRAPH, "q_off decreases at timeline %lld", (long long)q);
+  const int64_t QE = g->q_off[NQ];
+  if (QE > 0 && !g->q_ops) return fail(e, ECHO_E_INVALID_ARG, "q_ops is NULL");
+  if (QE >= INT32_MAX) return fail(e, ECHO_E_UNSUPPORTED, "too many timeline entries");
+  std::vector<int32_t> cnt(V, 0);
+  std::vector<int64_t> comm_keys;
+  for (int64_t q = 0; q < NQ; ++q) {
+    int32_t r = (int32_t)(q / NS), k = (int32_t)(q % NS);
+    for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i) {
+      int32_t v = g->q_ops[i];
+      if (v < 0 || v >= V) return fail(e, ECHO_E_BAD_GRAPH, "timeline (%d,%d): op %d out of range", r, k, v);
+      uint8_t kd = g->kind[v];
+      if ((k == 0) != (kd == ECHO_OP_COMPUTE))
+        return fail(e, ECHO_E_BAD_GRAPH, "op %d of kind %d on stream %d of rank %d (stream 0 holds exactly the compute ops)", v, kd, k, r);
+      cnt[v]++;
+      if (kd == ECHO_OP_COLL || kd == ECHO_OP_P2P) {
+        const auto &m = members[g->group[v]];
+        if (!std::binary_search(m.begin(), m.end(), r))
+          return fail(e, ECHO_E_BAD_GRAPH, "comm op %d on rank %d, which is not in its group", v, r);
+        comm_keys.push_back((int64_t)v * R + r);
+      }
+    }
+  }
+  std::sort(comm_keys.begin(), comm_keys.end());
+  if (std::adjacent_find(comm_keys.begin(), comm_keys.end()) != comm_keys.end())
+    return fail(e, ECHO_E_BAD_GRAPH, "a comm op is issued twice on one rank");
+  for (int64_t v = 0; v < V; ++v) {
+    uint8_t kd = g->kind[v];
+    int64_t want = (kd == ECHO_OP_COLL || kd == ECHO_OP_P2P) ? (int64_t)members[g->group[v]].size() : 1;
+    if (cnt[v] != want)
+      return fail(e, ECHO_E_BAD_GRAPH, "op %lld appears on %d timelines, expected %lld", (long long)v, cnt[v], (long long)want);
+  }
+
+  // Kahn levelling over data + issue-order dependencies; level = ASAP depth
+  std::vector<int64_t> succ_off(V + 1, 0);
+  for (int64_t k = 0; k < E; ++k) succ_off[g->pred_idx[k] + 1]++;
+  for (int64_t v = 0; v < V; ++v) succ_off[v + 1] += succ_off[v];
+  std::vector<int32_t> succ(E > 0 ? E : 1);
+  {
+    std::vector<int64_t> fill(succ_off.begin(), succ_off.end() - 1);
+    for (int64_t v = 0; v < V; ++v)
+      for (int64_t k = g->pred_off[v]; k < g->pred_off[v + 1]; ++k) succ[fill[g->pred_idx[k]]++] = (int32_t)v;
+  }
+  // next op on each timeline of an op: (op, next) pairs
+  std::vector<int64_t> nx_off(V + 1, 0);
+  std::vector<int32_t> indeg(V, 0);
+  for (int64_t v = 0; v < V; ++v) indeg[v] = (int32_t)(g->pred_off[v + 1] - g->pred_off[v]);
+  for (int64_t q = 0; q < NQ; ++q)
+    for (int64_t i = g->q_off[q]; i + 1 < g->q_off[q + 1]; ++i) {
+      nx_off[g->q_ops[i] + 1]++;
+      indeg[g->q_ops[i + 1]]++;
+    }
+  for (int64_t v = 0; v < V; ++v) nx_off[v + 1] += nx_off[v];
+  std::vector<int32_t> nx(nx_off[V] > 0 ? nx_off[V] : 1);
+  {
+    std::vector<int64_t> fill(nx_off.begin(), nx_off.end() - 1);
+    for (int64_t q = 0; q < NQ; ++q)
+      for (int64_t i = g->q_off[q]; i + 1 < g->q_off[q + 1]; ++i) nx[fill[g->q_ops[i]]++] = g->q_ops[i + 1];
+  }
+  std::vector<int32_t> level(V, 0), order;
+  order.reserve(V);
+  for (int64_t v = 0; v < V; ++v)
+    if (indeg[v] == 0) order.push_back((int32_t)v);
+  for (size_t h = 0; h < order.size(); ++h) {
+    int32_t u = order[h];
+    auto relax = [&](int32_t w) {
+      level[w] = std::max(level[w], level[u] + 1);
+      if (--indeg[w] == 0) order.push_back(w);
+    };
+    for (int64_t k = succ_off[u]; k < succ_off[u + 1]; ++k) relax(succ[k]);
+    for (int64_t k = nx_off[u]; k < nx_off[u + 1]; ++k) relax(nx[k]);
+  }
+  if ((int64_t)order.size() != V)
+    return fail(e, ECHO_E_CYCLE, "the dependencies form a cycle (%lld of %lld ops orderable)", (long long)order.size(), (long long)V);
+
+  int64_t L = 0;
+  for (int64_t v = 0; v < V; ++v) L = std::max<int64_t>(L, level[v] + 1);
+  b.V = V;
+  b.E = E;
+  b.QE = QE;
+  b.L = L;
+  b.R = R;
+  b.NS = NS;
+  b.gpn = g->gpus_per_node;
+  b.max_kclass = max_kc;
+  b.lvl_off.assign(L + 1, 0);
+  for (int64_t v = 0; v < V; ++v) b.lvl_off[level[v] + 1]++;
+  b.max_width = 0;
+  for (int64_t l = 0; l < L; ++l) b.max_width = std::max(b.max_width, b.lvl_off[l + 1]);
+  for (int64_t l = 0; l < L; ++l) b.lvl_off[l + 1] += b.lvl_off[l];
+  b.int2ext.assign(V, 0);
+  b.ext2int.assign(V, 0);
+  {
+    std::vector<int64_t> cur(b.lvl_off.begin(), b.lvl_off.end() - 1);
+    for (int64_t v = 0; v < V; ++v) {
+      int64_t i = cur[level[v]]++;
+      b.int2ext[i] = (int32_t)v;
+      b.ext2int[v] = (int32_t)i;
+    }
+  }
+  // timelines of every internal node
+  b.nq_off.assign(V + 1, 0);
+  for (int64_t i = 0; i < QE; ++i) b.nq_off[b.ext2int[g->q_ops[i]] + 1]++;
+  for (int64_t v = 0; v < V; ++v) b.nq_off[v + 1] += b.nq_off[v];
+  b.nq.assign(QE > 0 ? QE : 1, 0);
+  b.q_off.assign(g->q_off, g->q_off + NQ + 1);
+  b.q_ops_int.assign(QE > 0 ? QE : 1, 0);
+  {
+    std::vector<int64_t> fill(b.nq_off.begin(), b.nq_off.end() - 1);
+    for (int64_t q = 0; q < NQ; ++q)
+      for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i) {
+        int32_t in = b.ext2int[g->q_ops[i]];
+        b.nq[fill[in]++] = (int32_t)q;
+        b.q_ops_int[i] = in;
+      }
+  }
+  // data predecessors in internal ids
+  b.dp_off.assign(V + 1, 0);
+  b.dp.assign(E > 0 ? E : 1, 0);
+  for (int64_t i = 0; i < V; ++i) {
+    int32_t v = b.int2ext[i];
+    int64_t n = g->pred_off[v + 1] - g->pred_off[v];
+    b.dp_off[i + 1] = b.dp_off[i] + n;
+    for (int64_t k = 0; k < n; ++k) b.dp[b.dp_off[i] + k] = b.ext2int[g->pred_idx[g->pred_off[v] + k]];
+  }
+  b.kcl.assign(V, echo::kNotSlowable);
+  b.is_comm.assign(V, 0);
+  b.local.assign(V, 0);
+  b.node_sig.assign(V, -1);
+  // group shape: N members, M distinct nodes, K largest per-node count, log2(M)
+  std::vector<int32_t> gN(g->n_groups), gM(g->n_groups), gK(g->n_groups);
+  for (int32_t gi = 0; gi < g->n_groups; ++gi) {
+    std::map<int32_t, int32_t> per_node;
+    for (int32_t r : members[gi]) per_node[r / g->gpus_per_node]++;
+    int32_t K = 0;
+    for (auto &kv : per_node) K = std::max(K, kv.second);
+    gN[gi] = (int32_t)members[gi].size();
+    gM[gi] = (int32_t)per_node.size();
+    gK[gi] = K;
+  }
+  std::map<std::tuple<int32_t, int32_t, int64_t, int32_t, int32_t, int32_t>, int32_t> sig_of;
+  for (int64_t i = 0; i < V; ++i) {
+    int32_t v = b.int2ext[i];
+    uint8_t kd = g->kind[v];
+    if (kd == ECHO_OP_COMPUTE) b.kcl[i] = g->kclass[v];
+    if (kd == ECHO_OP_COMPUTE || kd == ECHO_OP_MEMCPY) b.local[i] = 1;
+    if (kd == ECHO_OP_COLL || kd == ECHO_OP_P2P) {
+      b.is_comm[i] = 1;
+      int32_t gi = g->group[v];
+      int32_t t = g->cc_type[v];
+      int32_t a = (t == ECHO_CC_ALLREDUCE) ? g->cc_algo[v] : ECHO_ALGO_RING;
+      auto key = std::make_tuple(t, a, g->cc_bytes[v], gN[gi], gM[gi], gK[gi]);
+      auto it = sig_of.find(key);
+      int32_t s;
+      if (it == sig_of.end()) {
+        s = (int32_t)b.sigs.size();
+        sig_of.emplace(key, s);
+        CcSig cs;
+        cs.nbytes = g->cc_bytes[v];
+        cs.type = t;
+        cs.algo = a;
+        cs.N = gN[gi];
+        cs.M = gM[gi];
+        cs.K = gK[gi];
+        cs.pad = 0;
+        cs.lg = std::log2((double)gM[gi]);
+        b.sigs.push_back(cs);
+        b.sig_count.push_back(0);
+      } else {
+        s = it->second;
+      }
+      b.sig_count[s]++;
+      b.comm_node.push_back((int32_t)i);
+      b.comm_sig.push_back(s);
+      b.node_sig[i] = s;
+    }
+  }
+  return ECHO_OK;
+}
+
+// ------------------------------------------------------------------------------------
+template <typename T>
+struct DevArr {
+  T *p = nullptr;
+  size_t n = 0;
+};
+
+}  // namespace
+
+struct echo_ctx {
+  int device = 0;
+  int sms = 0;
+  cudaStream_t stream = nullptr;
+  bool own_stream = false;
+  std::string err;
+  int state = 0;  // 0 empty, 1 graph, 2 scenarios, 3 estimated, 4 composed
+  GraphBuild gb;
+  std::vector<void *> graph_allocs, scen_allocs;
+  // device graph
+  int64_t *lvl_off = nullptr, *nq_off = nullptr, *dp_off = nullptr, *q_off = nullptr;
+  int32_t *nq = nullptr, *dp = nullptr, *q_ops = nullptr, *int2ext = nullptr, *ext2int = nullptr;
+  int32_t *node_sig = nullptr, *comm_node = nullptr, *comm_sig = nullptr, *sig_count = nullptr;
+  uint8_t *kcl = nullptr, *is_comm = nullptr, *local = nullptr;
+  CcSig *sigs = nullptr;
+  int32_t *status = nullptr;
+  // scenarios
+  int32_t S = 0, C = 0, sigma = 1;
+  size_t scen_vs = 0;  // V*S the scenario buffers were sized for
+  ChunkTable tbl{};
+  double *prm = nullptr, *sf = nullptr, *sums = nullptr, *comm_sum = nullptr, *cc_ns = nullptr;
+  int64_t *raw = nullptr, *dur = nullptr, *f[2] = {nullptr, nullptr}, *mk = nullptr, *cc_dur = nullptr;
+  int64_t *gfrontier = nullptr;
+  uint8_t *ov[2] = {nullptr, nullptr};
+  std::vector<double> h_sums, h_maxsf;
+  int final_f = 0, final_ov = -1;
+  // scratch for readback / queries
+  void *stage = nullptr;
+  size_t stage_bytes = 0;
+  // profiling
+  bool prof = false;
+  std::vector<std::pair<std::string, std::pair<cudaEvent_t, cudaEvent_t>>> recs;
+  std::vector<cudaEvent_t> ev_pool;
+};
+
+namespace {
+
+int set_err(echo_ctx *c, int code, const std::string &msg) {
+  if (c) c->err = msg;
+  return code;
+}
+
+int cuda_fail(echo_ctx *c, cudaError_t e, const char *what) {
+  std::string m = std::string(what) + ": " + cudaGetErrorString(e);
+  if (e == cudaErrorMemoryAllocation) return set_err(c, ECHO_E_OOM, m);
+  return set_err(c, ECHO_E_CUDA, m);
+}
+
+#define CK(call, what)                           \
+  do {                                           \
+    cudaError_t _e = (call);                     \
+    if (_e != cudaSuccess) return cuda_fail(c, _e, what); \
+  } while (0)
+
+template <typename T>
+int dalloc(echo_ctx *c, std::vector<void *> &owner, T **p, size_t n) {
+  size_t bytes = std::max<size_t>(n, 1) * sizeof(T);
+  void *q = nullptr;
+  cudaError_t e = cudaMalloc(&q, bytes);
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    return set_err(c, ECHO_E_OOM, "cudaMalloc of " + std::to_string(bytes) + " bytes failed");
+  }
+  owner.push_back(q);
+  *p = static_cast<T *>(q);
+  return ECHO_OK;
+}
+
+template <typename T>
+int upload(echo_ctx *c, std::vector<void *> &owner, T **p, const std::vector<T> &h) {
+  int rc = dalloc(c, owner, p, h.size());
+  if (rc) return rc;
+  if (!h.empty()) CK(cudaMemcpyAsync(*p, h.data(), h.size() * sizeof(T), cudaMemcpyHostToDevice, c->stream), "upload");
+  return ECHO_OK;
+}
+
+void free_all(std::vector<void *> &v) {
+  for (void *p : v) cudaFree(p);
+  v.clear();
+}
+
+int stage_reserve(echo_ctx *c, size_t bytes) {
+  if (c->stage_bytes >= bytes) return ECHO_OK;
+  if (c->stage) cudaFree(c->stage);
+  c->stage = nullptr;
+  c->stage_bytes = 0;
+  cudaError_t e = cudaMalloc(&c->stage, bytes);
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    return set_err(c, ECHO_E_OOM, "cudaMalloc of the readback buffer failed");
+  }
+  c->stage_bytes = bytes;
+  return ECHO_OK;
+}
+
+template <typename F>
+cudaError_t timed(echo_ctx *c, const char *name, F &&launch) {
+  if (!c->prof) return launch();
+  auto get = [&]() {
+    cudaEvent_t ev;
+    if (!c->ev_pool.empty()) {
+      ev = c->ev_pool.back();
+      c->ev_pool.pop_back();
+    } else {
+      cudaEventCreate(&ev);
+    }
+    return ev;
+  };
+  cudaEvent_t a = get(), b = get();
+  cudaEventRecord(a, c->stream);
+  cudaError_t e = launch();
+  cudaEventRecord(b, c->stream);
+  c->recs.push_back({name, {a, b}});
+  return e;
+}
+
+int check_ctx(echo_ctx *c) {
+  if (!c) return ECHO_E_INVALID_ARG;
+  cudaError_t e = cudaSetDevice(c->device);
+  if (e != cudaSuccess) return cuda_fail(c, e, "cudaSetDevice");
+  return ECHO_OK;
+}
+
+int pick_sigma(int32_t S, int sms) {
+  int want = (S + sms - 1) / std::max(sms, 1);
+  int s = 1;
+  while (s < want && s < 16) s <<= 1;
+  return s;
+}
+
+int sync_status(echo_ctx *c, int32_t *host_status) {
+  CK(cudaMemcpyAsync(host_status, c->status, sizeof(int32_t), cudaMemcpyDeviceToHost, c->stream), "status readback");
+  CK(cudaStreamSynchronize(c->stream), "cudaStreamSynchronize");
+  return ECHO_OK;
+}
+
+int check_params(echo_ctx *c, int64_t n, const double *alpha, const double *bwa, const double *lata,
+                 const double *bwe, const double *late, const double *delta) {
+  if (n > 0 && (!alpha || !bwa || !lata || !bwe || !late || !delta))
+    return set_err(c, ECHO_E_INVALID_ARG, "link parameter arrays are required");
+  for (int64_t s = 0; s < n; ++s) {
+    if (!finite_nonneg(alpha[s]) || !finite_nonneg(lata[s]) || !finite_nonneg(late[s]) || !finite_nonneg(delta[s]))
+      return set_err(c, ECHO_E_INVALID_ARG, "alpha, latencies and delta must be finite and >= 0 (entry " + std::to_string(s) + ")");
+    if (!(std::isfinite(bwa[s]) && bwa[s] > 0.0) || !(std::isfinite(bwe[s]) && bwe[s] > 0.0))
+      return set_err(c, ECHO_E_INVALID_ARG, "bandwidths must be finite and > 0 (entry " + std::to_string(s) + ")");
+  }
+  return ECHO_OK;
+}
+
+int make_table(echo_ctx *c, int32_t n, const int64_t *mx, const int64_t *cb, ChunkTable *t) {
+  std::memset(t, 0, sizeof *t);
+  if (n == 0) {
+    t->n = 5;
+    for (int i = 0; i < 5; ++i) {
+      t->max_bytes[i] = kDefaultMax[i];
+      t->chunk[i] = kDefaultChunk[i];
+    }
+    return ECHO_OK;
+  }
+  if (n < 0 || n > echo::kMaxChunk) return set_err(c, ECHO_E_UNSUPPORTED, "chunk table size outside [0, 16]");
+  if (!mx || !cb) return set_err(c, ECHO_E_INVALID_ARG, "chunk table arrays are NULL");
+  t->n = n;
+  for (int i = 0; i < n; ++i) {
+    if (cb[i] <= 0) return set_err(c, ECHO_E_INVALID_ARG, "chunk sizes must be > 0");
+    if (i > 0 && mx[i] < mx[i - 1]) return set_err(c, ECHO_E_INVALID_ARG, "chunk_max_bytes must be ascending");
+    t->max_bytes[i] = mx[i];
+    t->chunk[i] = cb[i];
+  }
+  return ECHO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *echo_strerror(int s) {
+  switch (s) {
+    case ECHO_OK: return "ok";
+    case ECHO_E_INVALID_ARG: return "invalid argument";
+    case ECHO_E_BAD_GRAPH: return "malformed graph";
+    case ECHO_E_CYCLE: return "dependency cycle";
+    case ECHO_E_STATE: return "call out of order";
+    case ECHO_E_OOM: return "out of memory";
+    case ECHO_E_CUDA: return "CUDA error";
+    case ECHO_E_TIMEOUT: return "device wait timed out";
+    case ECHO_E_OVERFLOW: return "time overflow";
+    case ECHO_E_UNSUPPORTED: return "unsupported size";
+    default: return "unknown status";
+  }
+}
+
+int echo_last_error(echo_ctx *c, char *buf, size_t n) {
+  if (!c || !buf || n == 0) return ECHO_E_INVALID_ARG;
+  std::snprintf(buf, n, "%s", c->err.c_str());
+  return ECHO_OK;
+}
+
+int echo_create(echo_ctx **out, int device, void *cuda_stream) {
+  if (!out) return ECHO_E_INVALID_ARG;
+  *out = nullptr;
+  int n = 0;
+  if (cudaGetDeviceCount(&n) != cudaSuccess || device < 0 || device >= n) {
+    (void)cudaGetLastError();
+    return ECHO_E_INVALID_ARG;
+  }
+  echo_ctx *c = new (std::nothrow) echo_ctx();
+  if (!c) return ECHO_E_OOM;
+  c->device = device;
+  if (cudaSetDevice(device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) {
+    delete c;
+    return ECHO_E_CUDA;
+  }
+  if (cuda_stream) {
+    c->stream = static_cast<cudaStream_t>(cuda_stream);
+  } else {
+    if (cudaStreamCreateWithFlags(&c->stream, cudaStreamNonBlocking) != cudaSuccess) {
+      delete c;
+      return ECHO_E_CUDA;
+    }
+    c->own_stream = true;
+  }
+  void *st = nullptr;
+  if (cudaMalloc(&st, sizeof(int32_t)) != cudaSuccess) {
+    if (c->own_stream) cudaStreamDestroy(c->stream);
+    delete c;
+    return ECHO_E_OOM;
+  }
+  c->status = static_cast<int32_t *>(st);
+  *out = c;
+  return ECHO_OK;
+}
+
+int echo_destroy(echo_ctx *c) {
+  if (!c) return ECHO_OK;
+  cudaSetDevice(c->device);
+  cudaStreamSynchronize(c->stream);
+  free_all(c->graph_allocs);
+  free_all(c->scen_allocs);
+  if (c->stage) cudaFree(c->stage);
+  if (c->status) cudaFree(c->status);
+  for (auto &r : c->recs) {
+    cudaEventDestroy(r.second.first);
+    cudaEventDestroy(r.second.second);
+  }
+  for (auto ev : c->ev_pool) cudaEventDestroy(ev);
+  if (c->own_stream) cudaStreamDestroy(c->stream);
+  delete c;
+  return ECHO_OK;
+}
+
+int echo_check_graph(const echo_graph_desc *g, int64_t *n_levels, int64_t *max_width) {
+  GraphBuild b;
+  Err e;
+  int rc = build_graph(g, b, e);
+  if (rc) return rc;
+  if (n_levels) *n_levels = b.L;
+  if (max_width) *max_width = b.max_width;
+  return ECHO_OK;
+}
+
+int echo_load_graph(echo_ctx *c, const echo_graph_desc *g) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  GraphBuild b;
+  Err e;
+  rc = build_graph(g, b, e);
+  if (rc) return set_err(c, rc, e.msg);
+  CK(cudaStreamSynchronize(c->stream), "cudaStreamSynchronize");
+  free_all(c->graph_allocs);
+  free_all(c->scen_allocs);
+  c->scen_vs = 0;
+  c->state = 0;
+  c->gb = std::move(b);
+  const GraphBuild &B = c->gb;
+  auto &o = c->graph_allocs;
+  if ((rc = upload(c, o, &c->lvl_off, B.lvl_off)) || (rc = upload(c, o, &c->nq_off, B.nq_off)) ||
+      (rc = upload(c, o, &c->nq, B.nq)) || (rc = upload(c, o, &c->dp_off, B.dp_off)) ||
+      (rc = upload(c, o, &c->dp, B.dp)) || (rc = upload(c, o, &c->q_off, B.q_off)) ||
+      (rc = upload(c, o, &c->q_ops, B.q_ops_int)) || (rc = upload(c, o, &c->int2ext, B.int2ext)) ||
+      (rc = upload(c, o, &c->ext2int, B.ext2int)) || (rc = upload(c, o, &c->node_sig, B.node_sig)) ||
+      (rc = upload(c, o, &c->comm_node, B.comm_node)) || (rc = upload(c, o, &c->comm_sig, B.comm_sig)) ||
+      (rc = upload(c, o, &c->sig_count, B.sig_count)) || (rc = upload(c, o, &c->kcl, B.kcl)) ||
+      (rc = upload(c, o, &c->is_comm, B.is_comm)) || (rc = upload(c, o, &c->local, B.local)) ||
+      (rc = upload(c, o, &c->sigs, B.sigs))) {
+    free_all(c->graph_allocs);
+    return rc;
+  }
+  CK(cudaStreamSynchronize(c->stream), "graph upload");
+  c->state = 1;
+  return ECHO_OK;
+}
+
+int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (c->state < 1) return set_err(c, ECHO_E_STATE, "load a graph first");
+  if (!sc) return set_err(c, ECHO_E_INVALID_ARG, "scenario descriptor is NULL");
+  const GraphBuild &B = c->gb;
+  const int64_t V = B.V;
+  const int32_t S = sc->n_scen;
+  if (S < 1) return set_err(c, ECHO_E_INVALID_ARG, "n_scen must be >= 1");
+  if (sc->n_kclass < 1 || sc->n_kclass <= B.max_kclass)
+    return set_err(c, ECHO_E_INVALID_ARG, "n_kclass must exceed every compute op's kclass");
+  if (V > 0 && !sc->dur) return set_err(c, ECHO_E_INVALID_ARG, "dur is NULL");
+  if (!sc->slowdown) return set_err(c, ECHO_E_INVALID_ARG, "slowdown is NULL");
+  if ((rc = check_params(c, S, sc->alpha_ns, sc->bw_intra, sc->lat_intra, sc->bw_inter, sc->lat_inter, sc->delta)))
+    return rc;
+  const int32_t C = sc->n_kclass;
+  std::vector<double> maxsf(S, 1.0);
+  for (int64_t k = 0; k < (int64_t)C * S; ++k) {
+    double x = sc->slowdown[k];
+    if (!(std::isfinite(x) && x > 0.0 && x <= 1e6))
+      return set_err(c, ECHO_E_INVALID_ARG, "slowdown factors must be in (0, 1e6]");
+    maxsf[k % S] = std::max(maxsf[k % S], x);
+  }
+  ChunkTable tbl;
+  if ((rc = make_table(c, sc->n_chunk, sc->chunk_max_bytes, sc->chunk_bytes, &tbl))) return rc;
+
+  CK(cudaStreamSynchronize(c->stream), "cudaStreamSynchronize");
+  c->state = 1;
+  const size_t VS = (size_t)V * S;
+  const int sigma = pick_sigma(S, c->sms);
+  const int32_t G = (int32_t)B.sigs.size();
+  if (c->scen_vs != VS || c->S != S || c->C != C || c->sigma != sigma) {
+    free_all(c->scen_allocs);
+    c->scen_vs = 0;
+    auto &o = c->scen_allocs;
+    bool in_smem = true;
+    echo::compose_smem_bytes(B.R * B.NS, sigma, &in_smem);
+    int64_t nblk = (S + sigma - 1) / sigma;
+    if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sf, (size_t)C * S)) ||
+        (rc = dalloc(c, o, &c->sums, (size_t)S)) || (rc = dalloc(c, o, &c->comm_sum, (size_t)S)) ||
+        (rc = dalloc(c, o, &c->raw, VS)) || (rc = dalloc(c, o, &c->dur, VS)) ||
+        (rc = dalloc(c, o, &c->f[0], VS)) || (rc = dalloc(c, o, &c->f[1], VS)) ||
+        (rc = dalloc(c, o, &c->ov[0], VS)) || (rc = dalloc(c, o, &c->ov[1], VS)) ||
+        (rc = dalloc(c, o, &c->mk, (size_t)S)) || (rc = dalloc(c, o, &c->cc_ns, (size_t)G * S)) ||
+        (rc = dalloc(c, o, &c->cc_dur, (size_t)G * S)) ||
+        (!in_smem && (rc = dalloc(c, o, &c->gfrontier, (size_t)nblk * B.R * B.NS * sigma)))) {
+      free_all(c->scen_allocs);
+      return rc;
+    }
+    if (in_smem) c->gfrontier = nullptr;
+    c->scen_vs = VS;
+    c->S = S;
+    c->C = C;
+    c->sigma = sigma;
+  }
+  c->tbl = tbl;
+  c->h_maxsf = maxsf;
+  // parameters
+  const double *src[6] = {sc->alpha_ns, sc->bw_intra, sc->lat_intra, sc->bw_inter, sc->lat_inter, sc->delta};
+  for (int k = 0; k < 6; ++k)
+    CK(cudaMemcpyAsync(c->prm + (size_t)k * S, src[k], S * sizeof(double), cudaMemcpyHostToDevice, c->stream), "parameter upload");
+  CK(cudaMemcpyAsync(c->sf, sc->slowdown, (size_t)C * S * sizeof(double), cudaMemcpyHostToDevice, c->stream), "slowdown upload");
+  CK(cudaMemsetAsync(c->sums, 0, S * sizeof(double), c->stream), "memset");
+  CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
+  if (V > 0) {
+    CK(cudaMemcpyAsync(c->raw, sc->dur, VS * sizeof(int64_t), cudaMemcpyHostToDevice, c->stream), "duration upload");
+    CK(timed(c, "permute_rows", [&] {
+         return echo::launch_permute_rows(c->raw, c->int2ext, c->local, V, S, c->dur, c->sums, c->status, c->stream);
+       }), "permute_rows launch");
+  }
+  c->h_sums.assign(S, 0.0);
+  CK(cudaMemcpyAsync(c->h_sums.data(), c->sums, S * sizeof(double), cudaMemcpyDeviceToHost, c->stream), "sum readback");
+  int32_t st = 0;
+  if ((rc = sync_status(c, &st))) return rc;
+  if (st == echo::kDevNegativeDuration) return set_err(c, ECHO_E_INVALID_ARG, "negative duration in dur");
+  c->state = 2;
+  return ECHO_OK;
+}
+
+int echo_estimate_collectives(echo_ctx *c) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (c->state < 2) return set_err(c, ECHO_E_STATE, "load scenarios first");
+  const GraphBuild &B = c->gb;
+  const int32_t S = c->S, G = (int32_t)B.sigs.size();
+  c->state = 2;
+  echo::ScenParams p{c->prm, c->prm + S, c->prm + 2 * (size_t)S, c->prm + 3 * (size_t)S,
+                     c->prm + 4 * (size_t)S, c->prm + 5 * (size_t)S};
+  CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
+  CK(cudaMemsetAsync(c->comm_sum, 0, S * sizeof(double), c->stream), "memset");
+  CK(timed(c, "cc_estimate", [&] {
+       return echo::launch_cc_estimate(c->sigs, G, p, S, c->tbl, c->sig_count, c->cc_ns, c->cc_dur,
+                                       c->comm_sum, c->status, c->stream);
+     }), "cc_estimate launch");
+  CK(timed(c, "cc_scatter", [&] {
+       return echo::launch_cc_scatter(c->comm_node, c->comm_sig, (int64_t)B.comm_node.size(), c->cc_dur, S,
+                                      c->dur, c->stream);
+     }), "cc_scatter launch");
+  std::vector<double> comm(S, 0.0);
+  CK(cudaMemcpyAsync(comm.data(), c->comm_sum, S * sizeof(double), cudaMemcpyDeviceToHost, c->stream), "readback");
+  int32_t st = 0;
+  if ((rc = sync_status(c, &st))) return rc;
+  if (st == echo::kDevCcOverflow) return set_err(c, ECHO_E_OVERFLOW, "a collective's estimated time is not below 2^61 ns");
+  // every finish time is at most the sum of all (slowed) durations of its scenario
+  for (int32_t s = 0; s < S; ++s) {
+    double bound = c->h_sums[s] * c->h_maxsf[s] + comm[s] + (double)B.V + 1.0;
+    if (!(bound < 2305843009213693952.0))
+      return set_err(c, ECHO_E_OVERFLOW, "scenario " + std::to_string(s) + ": total duration could overflow int64");
+  }
+  c->state = 3;
+  return ECHO_OK;
+}
+
+int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (c->state < 3) return set_err(c, ECHO_E_STATE, "estimate the collectives first");
+  int32_t refine = opts ? opts->refine_passes : 1;
+  if (refine < 0 || refine > 8) return set_err(c, ECHO_E_INVALID_ARG, "refine_passes outside [0, 8]");
+  const GraphBuild &B = c->gb;
+  echo::ComposeArgs a{};
+  a.V = B.V;
+  a.S = c->S;
+  a.L = (int32_t)B.L;
+  a.n_queues = B.R * B.NS;
+  a.lvl_off = c->lvl_off;
+  a.nq_off = c->nq_off;
+  a.nq = c->nq;
+  a.dp_off = c->dp_off;
+  a.dp = c->dp;
+  a.kcl = c->kcl;
+  a.dur = c->dur;
+  a.sf = c->sf;
+  a.makespan = c->mk;
+  a.gfrontier = c->gfrontier;
+  echo::OverlapArgs o{};
+  o.S = c->S;
+  o.n_ranks = B.R;
+  o.n_streams = B.NS;
+  o.q_off = c->q_off;
+  o.q_ops = c->q_ops;
+  o.is_comm = c->is_comm;
+  o.kcl = c->kcl;
+  o.dur = c->dur;
+  o.sf = c->sf;
+  c->state = 3;
+  a.ov = nullptr;
+  a.f = c->f[0];
+  CK(timed(c, "compose", [&] { return echo::launch_compose(a, c->sigma, c->stream); }), "compose launch");
+  for (int32_t p = 1; p <= refine; ++p) {
+    o.f = c->f[(p - 1) % 2];
+    o.ov_prev = p > 1 ? c->ov[(p - 2) % 2] : nullptr;
+    o.ov = c->ov[(p - 1) % 2];
+    CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");
+    a.ov = c->ov[(p - 1) % 2];
+    a.f = c->f[p % 2];
+    CK(timed(c, "compose", [&] { return echo::launch_compose(a, c->sigma, c->stream); }), "compose launch");
+  }
+  c->final_f = refine % 2;
+  c->final_ov = refine > 0 ? (refine - 1) % 2 : -1;
+  c->state = 4;
+  return ECHO_OK;
+}
+
+static int read_range_check(echo_ctx *c, int64_t op0, int64_t op1, int need_state) {
+  if (c->state < need_state) return set_err(c, ECHO_E_STATE, "nothing to read yet");
+  if (op0 < 0 || op1 < op0 || op1 > c->gb.V) return set_err(c, ECHO_E_INVALID_ARG, "op range out of bounds");
+  return ECHO_OK;
+}
+
+int echo_read_times(echo_ctx *c, int64_t op0, int64_t op1, int64_t *start, int64_t *finish) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if ((rc = read_range_check(c, op0, op1, 4))) return rc;
+  const int32_t S = c->S;
+  const int64_t rows_per = std::max<int64_t>(1, (int64_t)(64 << 20) / S);
+  if ((rc = stage_reserve(c, (size_t)std::min<int64_t>(rows_per, std::max<int64_t>(op1 - op0, 1)) * S * 16)))
+    return rc;
+  const uint8_t *ov = c->final_ov >= 0 ? c->ov[c->final_ov] : nullptr;
+  for (int64_t a = op0; a < op1; a += rows_per) {
+    int64_t b = std::min(op1, a + rows_per);
+    int64_t n = (b - a) * S;
+    int64_t *ds = static_cast<int64_t *>(c->stage);
+    int64_t *df = ds + n;
+    CK(timed(c, "readback", [&] {
+         return echo::launch_readback(c->ext2int, a, b, S, c->f[c->final_f], c->dur, ov, c->kcl, c->sf,
+                                      start ? ds : nullptr, finish ? df : nullptr, c->stream);
+       }), "readback launch");
+    if (start) CK(cudaMemcpyAsync(start + (a - op0) * S, ds, n * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream), "D2H");
+    if (finish) CK(cudaMemcpyAsync(finish + (a - op0) * S, df, n * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream), "D2H");
+    CK(cudaStreamSynchronize(c->stream), "readback");
+  }
+  return ECHO_OK;
+}
+
+int echo_read_makespan(echo_ctx *c, int64_t *out) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (!out) return set_err(c, ECHO_E_INVALID_ARG, "output is NULL");
+  if (c->state < 4) return set_err(c, ECHO_E_STATE, "compose first");
+  CK(cudaMemcpyAsync(out, c->mk, c->S * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream), "D2H");
+  CK(cudaStreamSynchronize(c->stream), "makespan readback");
+  return ECHO_OK;
+}
+
+int echo_read_cc(echo_ctx *c, int64_t op0, int64_t op1, double *out) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (!out) return set_err(c, ECHO_E_INVALID_ARG, "output is NULL");
+  if ((rc = read_range_check(c, op0, op1, 3))) return rc;
+  const int32_t S = c->S;
+  const int64_t rows_per = std::max<int64_t>(1, (int64_t)(64 << 20) / S);
+  if ((rc = stage_reserve(c, (size_t)std::min<int64_t>(rows_per, std::max<int64_t>(op1 - op0, 1)) * S * 16)))
+    return rc;
+  for (int64_t a = op0; a < op1; a += rows_per) {
+    int64_t b = std::min(op1, a + rows_per);
+    int64_t n = (b - a) * S;
+    double *d = static_cast<double *>(c->stage);
+    CK(timed(c, "read_cc", [&] {
+         return echo::launch_read_cc(c->ext2int, a, b, S, c->node_sig, c->cc_ns, d, c->stream);
+       }), "read_cc launch");
+    CK(cudaMemcpyAsync(out + (a - op0) * S, d, n * sizeof(double), cudaMemcpyDeviceToHost, c->stream), "D2H");
+    CK(cudaStreamSynchronize(c->stream), "read_cc");
+  }
+  return ECHO_OK;
+}
+
+int echo_read_overlap(echo_ctx *c, int64_t op0, int64_t op1, uint8_t *out) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (!out) return set_err(c, ECHO_E_INVALID_ARG, "output is NULL");
+  if ((rc = read_range_check(c, op0, op1, 4))) return rc;
+  const int32_t S = c->S;
+  const int64_t rows_per = std::max<int64_t>(1, (int64_t)(64 << 20) / S);
+  if ((rc = stage_reserve(c, (size_t)std::min<int64_t>(rows_per, std::max<int64_t>(op1 - op0, 1)) * S * 16)))
+    return rc;
+  const uint8_t *ov = c->final_ov >= 0 ? c->ov[c->final_ov] : nullptr;
+  for (int64_t a = op0; a < op1; a += rows_per) {
+    int64_t b = std::min(op1, a + rows_per);
+    int64_t n = (b - a) * S;
+    uint8_t *d = static_cast<uint8_t *>(c->stage);
+    CK(timed(c, "read_overlap", [&] {
+         return echo::launch_read_ov(c->ext2int, a, b, S, ov, d, c->stream);
+       }), "read_overlap launch");
+    CK(cudaMemcpyAsync(out + (a - op0) * S, d, n, cudaMemcpyDeviceToHost, c->stream), "D2H");
+    CK(cudaStreamSynchronize(c->stream), "read_overlap");
+  }
+  return ECHO_OK;
+}
+
+int echo_cc_query(echo_ctx *c, const echo_cc_query_desc *q, double *out_ns) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (!q || (q->n > 0 && !out_ns)) return set_err(c, ECHO_E_INVALID_ARG, "query descriptor or output is NULL");
+  const int64_t n = q->n;
+  if (n < 0) return set_err(c, ECHO_E_INVALID_ARG, "negative query count");
+  if (n == 0) return ECHO_OK;
+  if (!q->cc_type || !q->cc_algo || !q->nbytes || !q->n_ranks || !q->n_nodes)
+    return set_err(c, ECHO_E_INVALID_ARG, "query arrays are required");
+  if ((rc = check_params(c, n, q->alpha_ns, q->bw_intra, q->lat_intra, q->bw_inter, q->lat_inter, q->delta))) return rc;
+  ChunkTable tbl;
+  if ((rc = make_table(c, q->n_chunk, q->chunk_max_bytes, q->chunk_bytes, &tbl))) return rc;
+  std::vector<double> lg(n);
+  std::vector<double> lg_cache(4097, -1.0);
+  for (int64_t i = 0; i < n; ++i) {
+    if (q->cc_type[i] > ECHO_CC_SENDRECV || (q->cc_type[i] == ECHO_CC_ALLREDUCE && q->cc_algo[i] > ECHO_ALGO_AUTO))
+      return set_err(c, ECHO_E_INVALID_ARG, "query " + std::to_string(i) + ": bad type or algorithm");
+    if (q->nbytes[i] < 0 || q->n_ranks[i] < 1 || q->n_nodes[i] < 1 || q->n_nodes[i] > q->n_ranks[i])
+      return set_err(c, ECHO_E_INVALID_ARG, "query " + std::to_string(i) + ": need bytes >= 0 and 1 <= M <= N");
+    int32_t m = q->n_nodes[i];
+    if (m <= 4096) {
+      if (lg_cache[m] < 0) lg_cache[m] = std::log2((double)m);
+      lg[i] = lg_cache[m];
+    } else {
+      lg[i] = std::log2((double)m);
+    }
+  }
+  // one staging allocation holds every query array: 6 param doubles, lg, bytes, N, M, type, algo, out
+  const size_t per = 6 * 8 + 8 + 8 + 4 + 4 + 1 + 1 + 8;
+  if ((rc = stage_reserve(c, per * (size_t)n + 256))) return rc;
+  char *base = static_cast<char *>(c->stage);
+  double *dprm = reinterpret_cast<double *>(base);
+  double *dlg = dprm + 6 * n;
+  int64_t *dbytes = reinterpret_cast<int64_t *>(dlg + n);
+  double *dout = reinterpret_cast<double *>(dbytes + n);
+  int32_t *dN = reinterpret_cast<int32_t *>(dout + n);
+  int32_t *dM = dN + n;
+  uint8_t *dtype = reinterpret_cast<uint8_t *>(dM + n);
+  uint8_t *dalgo = dtype + n;
+  const double *src[6] = {q->alpha_ns, q->bw_intra, q->lat_intra, q->bw_inter, q->lat_inter, q->delta};
+  for (int k = 0; k < 6; ++k)
+    CK(cudaMemcpyAsync(dprm + (size_t)k * n, src[k], n * sizeof(double), cudaMemcpyHostToDevice, c->stream), "H2D");
+  CK(cudaMemcpyAsync(dlg, lg.data(), n * sizeof(double), cudaMemcpyHostToDevice, c->stream), "H2D");
+  CK(cudaMemcpyAsync(dbytes, q->nbytes, n * sizeof(int64_t), cudaMemcpyHostToDevice, c->stream), "H2D");
+  CK(cudaMemcpyAsync(dN, q->n_ranks, n * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream), "H2D");
+  CK(cudaMemcpyAsync(dM, q->n_nodes, n * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream), "H2D");
+  CK(cudaMemcpyAsync(dtype, q->cc_type, n, cudaMemcpyHostToDevice, c->stream), "H2D");
+  CK(cudaMemcpyAsync(dalgo, q->cc_algo, n, cudaMemcpyHostToDevice, c->stream), "H2D");
+  echo::ScenParams p{dprm, dprm + n, dprm + 2 * n, dprm + 3 * n, dprm + 4 * n, dprm + 5 * n};
+  CK(timed(c, "cc_query", [&] {
+       return echo::launch_cc_query(n, dtype, dalgo, dbytes, dN, dM, dlg, p, tbl, dout, c->stream);
+     }), "cc_query launch");
+  CK(cudaMemcpyAsync(out_ns, dout, n * sizeof(double), cudaMemcpyDeviceToHost, c->stream), "D2H");
+  CK(cudaStreamSynchronize(c->stream), "cc_query");
+  return ECHO_OK;
+}
+
+int echo_graph_info_get(echo_ctx *c, echo_graph_info *info) {
+  if (!c || !info) return ECHO_E_INVALID_ARG;
+  if (c->state < 1) return set_err(c, ECHO_E_STATE, "load a graph first");
+  const GraphBuild &B = c->gb;
+  info->n_ops = B.V;
+  info->n_edges = B.E;
+  info->n_levels = B.L;
+  info->max_width = B.max_width;
+  info->n_queue_entries = B.QE;
+  info->n_comm_ops = (int64_t)B.comm_node.size();
+  info->n_signatures = (int64_t)B.sigs.size();
+  info->n_ranks = B.R;
+  info->n_streams = B.NS;
+  info->sigma = c->sigma;
+  return ECHO_OK;
+}
+
+int echo_set_profiling(echo_ctx *c, int enable) {
+  if (!c) return ECHO_E_INVALID_ARG;
+  c->prof = enable != 0;
+  return ECHO_OK;
+}
+
+int echo_read_profile(echo_ctx *c, echo_kernel_stat *out, int cap, int *n) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (!n || (cap > 0 && !out)) return set_err(c, ECHO_E_INVALID_ARG, "output is NULL");
+  CK(cudaStreamSynchronize(c->stream), "profile sync");
+  std::vector<std::string> names;
+  std::vector<std::pair<int64_t, double>> acc;
+  for (auto &r : c->recs) {
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, r.second.first, r.second.second);
+    size_t k = std::find(names.begin(), names.end(), r.first) - names.begin();
+    if (k == names.size()) {
+      names.push_back(r.first);
+      acc.push_back({0, 0.0});
+    }
+    acc[k].first++;
+    acc[k].second += ms;
+    c->ev_pool.push_back(r.second.first);
+    c->ev_pool.push_back(r.second.second);
+  }
+  c->recs.clear();
+  int m = 0;
+  for (size_t k = 0; k < names.size() && m < cap; ++k, ++m) {
+    std::snprintf(out[m].name, sizeof out[m].name, "%s", names[k].c_str());
+    out[m].launches = acc[k].first;
+    out[m].total_ms = acc[k].second;
+  }
+  *n = m;
+  return ECHO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,234 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle.
+
+Timelines are int64 ns and must match bit for bit; CC estimates are fp64 and must
+agree within 1e-9 relative (the build evaluates the same closed forms with
+explicit round-to-nearest operations, so in practice they are identical).
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2412_12487_gb300 import Echo, EchoError
+from paper_2412_12487_gb300 import workloads as W
+from tests import smallgraphs as SG
+
+pytestmark = pytest.mark.gpu
+CC_RTOL = 1e-9
+THREADS = max(1, min(16, os.cpu_count() or 1))
+
+
+def run_gpu(g, sc, refine=1, ctx=None):
+    e = ctx or Echo(0)
+    try:
+        e.load_graph(g)
+        e.load_scenarios(sc)
+        e.estimate_collectives()
+        e.compose(refine_passes=refine)
+        st, fn = e.read_times()
+        return dict(start=st, finish=fn, makespan=e.read_makespan(), cc=e.read_cc(),
+                    ov=e.read_overlap(), info=e.info())
+    finally:
+        if ctx is None:
+            e.close()
+
+
+def assert_same(got, want, g, refine=1):
+    assert np.array_equal(got["finish"], want.finish)
+    assert np.array_equal(got["start"], want.start)
+    assert np.array_equal(got["makespan"], want.makespan)
+    comm = (g.kind == W.KIND_COLL) | (g.kind == W.KIND_P2P)
+    assert np.isnan(got["cc"][~comm]).all()
+    np.testing.assert_allclose(got["cc"][comm], want.cc_ns[comm], rtol=CC_RTOL, atol=0)
+    if refine > 0:
+        assert np.array_equal(got["ov"], want.overlapped)
+
+
+def test_tiny_gpt_bit_exact():
+    c = W.config("tiny")
+    g = W.build_gpt_graph(c)
+    for S, refine in [(1, 1), (4, 0), (4, 1), (5, 2)]:
+        sc = W.make_scenarios(g, c, n_scen=S) if S == 1 else W.make_scenarios(
+            g, W.GPTConfig(**{**c.__dict__, "fixed_scenario": False}), n_scen=S)
+        assert_same(run_gpu(g, sc, refine), oracle.compose(g, sc, refine_passes=refine), g, refine)
+
+
+@pytest.mark.parametrize("S", [1, 3, 33, 130])
+def test_random_graphs_bit_exact(S):
+    rng = np.random.default_rng(77 + S)
+    e = Echo(0)
+    try:
+        for case in range(60):
+            g = SG.random_graph(rng, int(rng.integers(1, 60)), max_ranks=5, max_streams=5, p_edge=0.08)
+            sc = SG.random_scenarios(rng, g, S, max_dur=50)
+            for refine in (0, 1, 3):
+                got = run_gpu(g, sc, refine, ctx=e)
+                assert_same(got, oracle.compose(g, sc, refine_passes=refine), g, refine)
+    finally:
+        e.close()
+
+
+def test_gpt13b_all_ops_all_scenarios_bit_exact():
+    c = W.config("gpt1.3b")
+    g = W.build_gpt_graph(c)
+    sc = W.make_scenarios(g, c)
+    assert sc.n_scen == 256
+    got = run_gpu(g, sc)
+    want = oracle.compose(g, sc, threads=THREADS)
+    assert_same(got, want, g)
+    assert got["ov"].any() and (got["makespan"] > 0).all()
+
+
+def test_degenerate_inputs():
+    # empty graph
+    g = SG.graph_from_lists(2, 3, [], {}, [])
+    sc = W.Scenarios(dur=np.zeros((0, 3), np.int64), alpha_ns=np.zeros(3), bw_intra=np.ones(3),
+                     lat_intra=np.zeros(3), bw_inter=np.ones(3), lat_inter=np.zeros(3),
+                     delta=np.zeros(3), slowdown=np.ones((1, 3)), peak_flop_per_ns=np.ones(3))
+    got = run_gpu(g, sc)
+    assert (got["makespan"] == 0).all() and got["finish"].shape == (0, 3)
+    # one op, zero duration; a chain of zero durations; compute-only single stream
+    ops = [{"kind": W.KIND_COMPUTE} for _ in range(5)]
+    g = SG.graph_from_lists(1, 1, ops, {(0, 0): list(range(5))}, [])
+    sc = W.Scenarios(dur=np.zeros((5, 2), np.int64), alpha_ns=np.zeros(2), bw_intra=np.ones(2),
+                     lat_intra=np.zeros(2), bw_inter=np.ones(2), lat_inter=np.zeros(2),
+                     delta=np.zeros(2), slowdown=np.ones((1, 2)), peak_flop_per_ns=np.ones(2))
+    got = run_gpu(g, sc)
+    assert (got["finish"] == 0).all() and (got["makespan"] == 0).all()
+    sc.dur[:, 1] = [3, 0, 5, 0, 7]
+    got = run_gpu(g, sc)
+    assert got["finish"][:, 1].tolist() == [3, 3, 8, 8, 15]
+
+
+def test_high_fan_in_collective_and_global_frontier():
+    # 1024 ranks join one all-reduce: 1024 timeline reads and 1024 data preds for
+    # one node; 4096 ranks x 16 streams puts the frontier in global memory.
+    for R, NS in [(1024, 2), (4096, 16)]:
+        ops, queues = [], {}
+        for r in range(R):
+            ops.append({"kind": W.KIND_COMPUTE, "kclass": r % 3})
+            queues[(r, 0)] = [r]
+        ops.append({"kind": W.KIND_COLL, "group": 0, "cc_type": W.CC_ALLREDUCE,
+                    "cc_algo": W.ALGO_AUTO, "cc_bytes": 1 << 26, "preds": list(range(R))})
+        for r in range(R):
+            queues[(r, 1 + r % (NS - 1))] = [R]
+            ops.append({"kind": W.KIND_COMPUTE, "kclass": 0, "preds": [R]})
+            queues[(r, 0)].append(R + 1 + r)
+        g = SG.graph_from_lists(R, NS, ops, queues, [list(range(R))], gpus_per_node=8)
+        rng = np.random.default_rng(R)
+        sc = SG.random_scenarios(rng, g, 17, max_dur=10_000)
+        sc.bw_intra[:] = 300.0
+        sc.bw_inter[:] = 40.0
+        got = run_gpu(g, sc)
+        assert_same(got, oracle.compose(g, sc), g)
+
+
+def test_many_scenarios_several_waves():
+    c = W.config("tiny")
+    g = W.build_gpt_graph(c)
+    cr = W.GPTConfig(**{**c.__dict__, "fixed_scenario": False})
+    sc = W.make_scenarios(g, cr, n_scen=3001)
+    got = run_gpu(g, sc)
+    want = oracle.compose(g, sc, threads=THREADS)
+    assert_same(got, want, g)
+    assert got["info"]["sigma"] == 16
+
+
+def test_cc_queries_match_oracle():
+    q = W.make_cc_queries(1_000_000)
+    with Echo(0) as e:
+        got = e.cc_query(q)
+    lib = oracle._load()
+    import ctypes as C
+    prm = np.stack([q.alpha_ns, q.bw_intra, q.lat_intra, q.bw_inter, q.lat_inter, q.delta], 1)
+    prm = np.ascontiguousarray(prm)
+    want = np.empty(q.n)
+    K = -(-q.n_ranks // q.n_nodes)
+    lg = np.log2(q.n_nodes.astype(np.float64))
+    base = prm.ctypes.data
+    for i in range(q.n):
+        want[i] = lib.oracle_cc_ns(int(q.cc_type[i]), int(q.cc_algo[i]), int(q.nbytes[i]),
+                                   int(q.n_ranks[i]), int(q.n_nodes[i]), int(K[i]), float(lg[i]),
+                                   C.c_void_p(base + 48 * i), 0, None, None)
+    np.testing.assert_allclose(got, want, rtol=CC_RTOL, atol=0)
+    assert (got > 0).all()
+
+
+def test_call_order_and_input_errors():
+    c = W.config("tiny")
+    g = W.build_gpt_graph(c)
+    sc = W.make_scenarios(g, c)
+    with Echo(0) as e:
+        with pytest.raises(EchoError) as ei:
+            e.estimate_collectives()
+        assert ei.value.code == 4
+        e.load_graph(g)
+        with pytest.raises(EchoError) as ei:
+            e.compose()
+        assert ei.value.code == 4
+        bad = W.Scenarios(**{**sc.__dict__, "dur": sc.dur.copy()})
+        bad.dur[int(np.nonzero(g.kind == W.KIND_COMPUTE)[0][3]), 0] = -5
+        with pytest.raises(EchoError) as ei:
+            e.load_scenarios(bad)
+        assert ei.value.code == 1
+        bad = W.Scenarios(**{**sc.__dict__, "bw_inter": np.zeros(1)})
+        with pytest.raises(EchoError) as ei:
+            e.load_scenarios(bad)
+        assert ei.value.code == 1
+        huge = W.Scenarios(**{**sc.__dict__, "dur": sc.dur * 0 + (1 << 55)})
+        e.load_scenarios(huge)
+        with pytest.raises(EchoError) as ei:
+            e.estimate_collectives()
+        assert ei.value.code == 8
+        e.load_scenarios(sc)
+        e.estimate_collectives()
+        e.compose()
+        with pytest.raises(EchoError) as ei:
+            e.read_times(0, g.n_ops + 1)
+        assert ei.value.code == 1
+        a = e.read_makespan().copy()
+        e.compose()
+        assert np.array_equal(a, e.read_makespan())
+
+
+def _sampled_parity(name, cols, refine=1):
+    c = W.config(name)
+    g = W.build_gpt_graph(c)
+    sc = W.make_scenarios(g, c)
+    with Echo(0) as e:
+        e.load_graph(g)
+        e.load_scenarios(sc)
+        del sc.dur
+        e.estimate_collectives()
+        e.compose(refine_passes=refine)
+        mk = e.read_makespan()
+        V, S = g.n_ops, e.n_scen
+        fin = np.empty((V, len(cols)), np.int64)
+        st = np.empty((V, len(cols)), np.int64)
+        mk_check = np.zeros(S, np.int64)
+        step = max(1, (1 << 28) // (16 * S))
+        for a in range(0, V, step):
+            b = min(V, a + step)
+            s_, f_ = e.read_times(a, b)
+            fin[a:b] = f_[:, cols]
+            st[a:b] = s_[:, cols]
+            assert (s_ >= 0).all() and (f_ >= s_).all()
+            mk_check = np.maximum(mk_check, f_.max(0))
+        assert np.array_equal(mk, mk_check)
+    sub = W.select_scenarios(W.scenario_params(c), g, cols)
+    want = oracle.compose(g, sub, refine_passes=refine, threads=min(THREADS, len(cols)), want_cc=False,
+                          want_overlap=False)
+    assert np.array_equal(fin, want.finish)
+    assert np.array_equal(st, want.start)
+    assert np.array_equal(mk[cols], want.makespan)
+
+
+@pytest.mark.slow
+def test_gpt175b_full_size_sampled_scenarios():
+    _sampled_parity("gpt175b", [0, 1, 509, 1023])
+
+
+@pytest.mark.slow
+def test_gpt175b_1024_ranks_full_size_sampled_scenarios():
+    _sampled_parity("gpt175b-1024", [0, 63])
