@@ -861,7 +861,7 @@ int echo_read_overlap(echo_ctx *c, int64_t op0, int64_t op1, uint8_t *out) {
     int64_t n = (b - a) * S;
     uint8_t *d = static_cast<uint8_t *>(c->stage);
     CK(timed(c, "read_overlap", [&] {
-         return echo::launch_read_ov(c->ext2int, a, b, S, ov, d, c->stream);
+         return echo::launch_read_ov(c->ext2int, a, b, S, ov, c->kcl, d, c->stream);
        }), "read_overlap launch");
     CK(cudaMemcpyAsync(out + (a - op0) * S, d, n, cudaMemcpyDeviceToHost, c->stream), "D2H");
     CK(cudaStreamSynchronize(c->stream), "read_overlap");

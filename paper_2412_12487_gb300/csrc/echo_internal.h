@@ -81,7 +81,7 @@ cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, in
 cudaError_t launch_read_cc(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S,
                            const int32_t *node_sig, const double *cc_ns, double *out, cudaStream_t st);
 cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S,
-                           const uint8_t *ov, uint8_t *out, cudaStream_t st);
+                           const uint8_t *ov, const uint8_t *kcl, uint8_t *out, cudaStream_t st);
 size_t compose_smem_bytes(int32_t n_queues, int sigma, bool *frontier_in_smem);
 
 }  // namespace echo

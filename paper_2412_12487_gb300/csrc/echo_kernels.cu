@@ -300,13 +300,15 @@ __global__ void read_cc_kernel(const int32_t *__restrict__ ext2int, int64_t op0,
 }
 
 __global__ void read_ov_kernel(const int32_t *__restrict__ ext2int, int64_t op0, int64_t op1, int32_t S,
-                               const uint8_t *__restrict__ ov, uint8_t *__restrict__ out) {
+                               const uint8_t *__restrict__ ov, const uint8_t *__restrict__ kcl,
+                               uint8_t *__restrict__ out) {
   int64_t total = (op1 - op0) * S;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
        idx += (int64_t)gridDim.x * blockDim.x) {
     int64_t o = idx / S;
     int32_t s = (int32_t)(idx - o * S);
-    out[idx] = ov ? ov[(int64_t)ext2int[op0 + o] * S + s] : 0;
+    int64_t i = ext2int[op0 + o];
+    out[idx] = (ov && kcl[i] != kNotSlowable) ? ov[i * S + s] : 0;  // only compute ops are tested
   }
 }
 
@@ -420,10 +422,10 @@ cudaError_t launch_read_cc(const int32_t *ext2int, int64_t op0, int64_t op1, int
 }
 
 cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, const uint8_t *ov,
-                           uint8_t *out, cudaStream_t st) {
+                           const uint8_t *kcl, uint8_t *out, cudaStream_t st) {
   int64_t n = (op1 - op0) * S;
   if (n <= 0) return cudaSuccess;
-  read_ov_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, ov, out);
+  read_ov_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, ov, kcl, out);
   return cudaGetLastError();
 }
 
