@@ -193,6 +193,26 @@ typedef struct {
 } echo_cc_query_desc;
 int echo_cc_query(echo_ctx *ctx, const echo_cc_query_desc *q, double *out_ns);
 
+/* Allocation-free variant of echo_cc_query.  The paper has no counterpart: this
+ * entry point exists for callers that cannot call cudaMalloc, such as a process
+ * whose device memory belongs to a framework's memory pool or one that runs under
+ * a fixed device-memory budget.  It needs no context and allocates nothing.
+ *   - The per-query arrays of *q and out_ns are DEVICE memory owned by the caller
+ *     (out_ns: n doubles); the chunk table fields of *q are host memory.
+ *   - Work runs on `cuda_stream` (a cudaStream_t; NULL = the default stream) of the
+ *     current device, and the call waits for that stream before returning.
+ *   - Besides the caller's arrays it uses one static device array of about 520 KB
+ *     (a status word and log2(m) for m = 1..65536), which every GPU that loads the
+ *     library holds until the process exits.  The first call on a device fills
+ *     that table with a synchronous copy, so make the first call on each device
+ *     before any stream capture.
+ *   - Every call shares the array and clears its status word: calls that overlap
+ *     on the GPU race.
+ *   - A query whose node count M exceeds 65536 gets NaN and the call returns
+ *     ECHO_E_UNSUPPORTED; a malformed query (the checks of echo_cc_query) gets NaN
+ *     and the call returns ECHO_E_INVALID_ARG; other queries are still estimated. */
+int echo_cc_query_noalloc(const echo_cc_query_desc *q, double *out_ns, void *cuda_stream);
+
 /* Shape of the loaded graph (after echo_load_graph). */
 typedef struct {
   int64_t n_ops, n_edges, n_levels, max_width, n_queue_entries, n_comm_ops, n_signatures;

@@ -5,7 +5,12 @@
 
 #include <cmath>
 #include <cstdint>
+#include <cstring>
+#include <functional>
+#include <mutex>
+#include <vector>
 
+#include "echo.h"
 #include "echo_internal.h"
 
 namespace echo {
@@ -430,3 +435,143 @@ cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int
 }
 
 }  // namespace echo
+
+// ---------------------------------------------------------------------------------
+// Allocation-free CC queries.
+//
+// Some callers cannot call cudaMalloc: a process whose device memory is owned by a
+// framework's memory pool (a stray allocation would fail or fragment that pool), or
+// one that runs under a fixed per-process memory budget.  echo_cc_query_noalloc
+// serves them: the caller passes device arrays in and out, and the only other
+// device memory the kernel touches is the file-scope array below, which every GPU
+// that loads this library holds until the process exits.
+//
+// Layout of the array: bytes [0, 4) hold a status word, cleared at the start of
+// every call; from byte 256 on, log2(m) for m = 0..kNoallocMaxNodes, computed on
+// the host with the same libm log2 the allocating path uses, so both paths give
+// identical estimates.  Node counts above kNoallocMaxNodes are rejected.
+// ---------------------------------------------------------------------------------
+namespace echo {
+namespace {
+constexpr int32_t kNoallocMaxNodes = 65536;
+constexpr size_t kNoallocLgOffset = 256;
+constexpr size_t kNoallocScratchBytes = kNoallocLgOffset + sizeof(double) * (kNoallocMaxNodes + 1);
+constexpr int kNoallocMaxDevices = 64;
+enum : int32_t { kNoallocOk = 0, kNoallocTooManyNodes = 1, kNoallocBadQuery = 2 };
+}  // namespace
+}  // namespace echo
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[echo::kNoallocScratchBytes];
+
+namespace echo {
+namespace {
+
+struct NoallocDevice {
+  std::once_flag once;
+  unsigned char *ptr = nullptr;  // device address of g_noalloc_scratch on this device
+  cudaError_t err = cudaSuccess;
+};
+NoallocDevice g_noalloc_devices[kNoallocMaxDevices];
+
+// Once per device, with that device current: look up the array's device address
+// (host code cannot use the symbol itself) and fill the log2 table.
+void noalloc_setup(NoallocDevice &d) {
+  void *p = nullptr;
+  d.err = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (d.err != cudaSuccess) return;
+  std::vector<double> lg(kNoallocMaxNodes + 1, 0.0);
+  for (int32_t m = 1; m <= kNoallocMaxNodes; ++m) lg[m] = std::log2((double)m);
+  unsigned char *base = static_cast<unsigned char *>(p);
+  d.err = cudaMemcpy(base + kNoallocLgOffset, lg.data(), lg.size() * sizeof(double), cudaMemcpyHostToDevice);
+  if (d.err != cudaSuccess) return;
+  d.ptr = base;
+}
+
+__device__ __forceinline__ bool nonneg_finite(double x) { return isfinite(x) && x >= 0.0; }
+
+// Same estimate as cc_query_kernel; log2(M) comes from the table in the static
+// array and each query is checked on the device, since its fields live there.
+__global__ void cc_query_noalloc_kernel(int64_t n, const uint8_t *__restrict__ type,
+                                        const uint8_t *__restrict__ algo, const int64_t *__restrict__ nbytes,
+                                        const int32_t *__restrict__ N, const int32_t *__restrict__ M,
+                                        ScenParams p, ChunkTable tbl, unsigned char *scratch,
+                                        double *__restrict__ out) {
+  int32_t *status = reinterpret_cast<int32_t *>(scratch);
+  const double *lg = reinterpret_cast<const double *>(scratch + kNoallocLgOffset);
+  const double nan = __longlong_as_double(0x7ff8000000000000LL);
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int t = type[i], a = algo[i];
+    const int n_r = N[i], m = M[i];
+    const int64_t nb = nbytes[i];
+    const bool ok = t <= kSR && (t != kAR || a <= 2) && nb >= 0 && n_r >= 1 && m >= 1 && m <= n_r &&
+                    nonneg_finite(p.alpha[i]) && nonneg_finite(p.lata[i]) && nonneg_finite(p.late[i]) &&
+                    nonneg_finite(p.delta[i]) && isfinite(p.bwa[i]) && p.bwa[i] > 0.0 &&
+                    isfinite(p.bwe[i]) && p.bwe[i] > 0.0;
+    if (!ok) {
+      out[i] = nan;
+      set_status(status, kNoallocBadQuery);
+      continue;
+    }
+    if (m > kNoallocMaxNodes) {
+      out[i] = nan;
+      set_status(status, kNoallocTooManyNodes);
+      continue;
+    }
+    const int K = (n_r + m - 1) / m;
+    out[i] = cc_ns_of(t, a, nb, n_r, m, K, lg[m], p.alpha[i], p.bwa[i], p.lata[i], p.bwe[i], p.late[i],
+                      p.delta[i], tbl);
+  }
+}
+
+}  // namespace
+}  // namespace echo
+
+extern "C" int echo_cc_query_noalloc(const echo_cc_query_desc *q, double *out_ns, void *cuda_stream) {
+  using namespace echo;
+  if (!q || q->n < 0) return ECHO_E_INVALID_ARG;
+  if (q->n == 0) return ECHO_OK;
+  if (!out_ns || !q->cc_type || !q->cc_algo || !q->nbytes || !q->n_ranks || !q->n_nodes || !q->alpha_ns ||
+      !q->bw_intra || !q->lat_intra || !q->bw_inter || !q->lat_inter || !q->delta)
+    return ECHO_E_INVALID_ARG;
+  // the chunk table is a few host values passed by value to the kernel
+  ChunkTable tbl;
+  std::memset(&tbl, 0, sizeof tbl);
+  if (q->n_chunk == 0) {
+    const int64_t mx[5] = {4LL << 20, 8LL << 20, 64LL << 20, 128LL << 20, INT64_MAX};
+    const int64_t cb[5] = {18000, 36000, 72000, 144000, 288000};
+    tbl.n = 5;
+    for (int i = 0; i < 5; ++i) {
+      tbl.max_bytes[i] = mx[i];
+      tbl.chunk[i] = cb[i];
+    }
+  } else {
+    if (q->n_chunk < 0 || q->n_chunk > kMaxChunk) return ECHO_E_UNSUPPORTED;
+    if (!q->chunk_max_bytes || !q->chunk_bytes) return ECHO_E_INVALID_ARG;
+    tbl.n = q->n_chunk;
+    for (int i = 0; i < q->n_chunk; ++i) {
+      if (q->chunk_bytes[i] <= 0 || (i > 0 && q->chunk_max_bytes[i] < q->chunk_max_bytes[i - 1]))
+        return ECHO_E_INVALID_ARG;
+      tbl.max_bytes[i] = q->chunk_max_bytes[i];
+      tbl.chunk[i] = q->chunk_bytes[i];
+    }
+  }
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoallocMaxDevices) return ECHO_E_CUDA;
+  NoallocDevice &d = g_noalloc_devices[dev];
+  std::call_once(d.once, noalloc_setup, std::ref(d));
+  if (d.err != cudaSuccess || !d.ptr) return ECHO_E_CUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  if (cudaMemsetAsync(d.ptr, 0, sizeof(int32_t), st) != cudaSuccess) return ECHO_E_CUDA;
+  ScenParams p{q->alpha_ns, q->bw_intra, q->lat_intra, q->bw_inter, q->lat_inter, q->delta};
+  cc_query_noalloc_kernel<<<grid_for(q->n, 256), 256, 0, st>>>(q->n, q->cc_type, q->cc_algo, q->nbytes,
+                                                                q->n_ranks, q->n_nodes, p, tbl, d.ptr, out_ns);
+  if (cudaGetLastError() != cudaSuccess) return ECHO_E_CUDA;
+  int32_t status = 0;
+  if (cudaMemcpyAsync(&status, d.ptr, sizeof(int32_t), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return ECHO_E_CUDA;
+  if (status == kNoallocTooManyNodes) return ECHO_E_UNSUPPORTED;
+  if (status == kNoallocBadQuery) return ECHO_E_INVALID_ARG;
+  return ECHO_OK;
+}

@@ -22,7 +22,8 @@ STATUS_NAMES = {0: "ECHO_OK", 1: "ECHO_E_INVALID_ARG", 2: "ECHO_E_BAD_GRAPH", 3:
 # every function the header declares (checked by the tests)
 EXPORTS = ["echo_create", "echo_destroy", "echo_check_graph", "echo_load_graph", "echo_load_scenarios",
            "echo_estimate_collectives", "echo_compose", "echo_read_times", "echo_read_makespan",
-           "echo_read_cc", "echo_read_overlap", "echo_cc_query", "echo_graph_info_get",
+           "echo_read_cc", "echo_read_overlap", "echo_cc_query", "echo_cc_query_noalloc",
+           "echo_graph_info_get",
            "echo_set_profiling", "echo_read_profile", "echo_strerror", "echo_last_error"]
 
 
@@ -103,6 +104,7 @@ def load_library(path: Optional[str] = None):
         "echo_read_cc": ([vp, i64, i64, vp], C.c_int),
         "echo_read_overlap": ([vp, i64, i64, vp], C.c_int),
         "echo_cc_query": ([vp, C.POINTER(CCQueryDesc), vp], C.c_int),
+        "echo_cc_query_noalloc": ([C.POINTER(CCQueryDesc), vp, vp], C.c_int),
         "echo_graph_info_get": ([vp, C.POINTER(GraphInfo)], C.c_int),
         "echo_set_profiling": ([vp, C.c_int], C.c_int),
         "echo_read_profile": ([vp, C.POINTER(KernelStat), C.c_int, C.POINTER(C.c_int)], C.c_int),
