@@ -128,11 +128,12 @@ def profiled_traffic(launch_units):
     return float(m_bytes.group(1)) * launch_units
 
 
-def build_inputs(rank, pinned=True):
+def build_inputs(rank, n_scen=None, pinned=True):
     import torch
     from paper_2412_12487_gb300 import workloads as W
     c = W.config(WORKLOAD)
-    c = W.GPTConfig(**{**c.__dict__, "scen_seed": c.scen_seed + 7919 * rank})
+    c = W.GPTConfig(**{**c.__dict__, "scen_seed": c.scen_seed + 7919 * rank,
+                       "n_scen": n_scen or c.n_scen})
     t0 = time.time()
     g = W.build_gpt_graph(c)
     sc = W.scenario_params(c)
@@ -160,7 +161,7 @@ def run_echo(args):
     torch.cuda.set_device(local)
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    c, g, sc, dur_t = build_inputs(rank)
+    c, g, sc, dur_t = build_inputs(rank, args.scenarios)
     V, S = g.n_ops, sc.n_scen
     stream = torch.cuda.current_stream()
     e = Echo(local, stream)
@@ -236,7 +237,7 @@ def run_echo(args):
     traffic = profiled_traffic(V * S)
     out = None
     if rank == 0:
-        cpu = cpu_baseline(g, c, args) if world == 1 else None
+        cpu = cpu_baseline(g, c, args) if world == 1 and args.cpu_sample > 0 else None
         h2d = V * S * 8 + 6 * S * 8 + sc.slowdown.size * 8
         out = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -322,7 +323,11 @@ def main():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="echo", choices=["echo", "reference"])
-    ap.add_argument("--cpu-sample", type=int, default=8)
+    ap.add_argument("--cpu-sample", type=int, default=8,
+                    help="scenarios of the CPU-oracle baseline sample (0 = skip)")
+    ap.add_argument("--scenarios", type=int, default=None,
+                    help="scenarios per GPU (default: the workload's 1024); smaller values "
+                         "make small cases for profiling")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "echo":
         log("note: warmup raised to 3")

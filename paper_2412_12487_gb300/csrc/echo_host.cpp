@@ -7,6 +7,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <new>
@@ -47,7 +48,10 @@ struct GraphBuild {
   int64_t V = 0, E = 0, QE = 0, L = 0, max_width = 0;
   int32_t R = 0, NS = 0, gpn = 1;
   std::vector<int32_t> int2ext, ext2int;
-  std::vector<int64_t> lvl_off;
+  int64_t Ls = 0, n_seg = 0;           // segment levels, segments
+  std::vector<int64_t> seg_lvl_off;    // [Ls+1] segments of each segment level
+  std::vector<int64_t> seg_node_off;   // [n_seg+1] nodes of each segment (internal ids)
+  std::vector<int32_t> seg_int;        // [V] segment of each internal node
   std::vector<int64_t> nq_off;
   std::vector<int32_t> nq;
   std::vector<int64_t> dp_off;
@@ -57,7 +61,11 @@ struct GraphBuild {
   std::vector<int32_t> q_ops_int;
   std::vector<CcSig> sigs;
   std::vector<int32_t> sig_count, comm_node, comm_sig, node_sig;
+  std::vector<int32_t> non_compute;   // internal ids of comm and memcpy ops
+  std::vector<int64_t> ov_chunks;     // (rank, first position) of compute-timeline chunks
+  std::vector<int64_t> blk_words;     // record block size of each segment level (words, padded)
   int32_t max_kclass = -1;
+  bool stageable = true;              // every head/tail has < 2^16 timelines and predecessors
 };
 
 bool finite_nonneg(double x) { return std::isfinite(x) && x >= 0.0; }
@@ -222,20 +230,103 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
   b.NS = NS;
   b.gpn = g->gpus_per_node;
   b.max_kclass = max_kc;
-  b.lvl_off.assign(L + 1, 0);
-  for (int64_t v = 0; v < V; ++v) b.lvl_off[level[v] + 1]++;
   b.max_width = 0;
-  for (int64_t l = 0; l < L; ++l) b.max_width = std::max(b.max_width, b.lvl_off[l + 1]);
-  for (int64_t l = 0; l < L; ++l) b.lvl_off[l + 1] += b.lvl_off[l];
+  {
+    std::vector<int64_t> w(L, 0);
+    for (int64_t v = 0; v < V; ++v) w[level[v]]++;
+    for (int64_t l = 0; l < L; ++l) b.max_width = std::max(b.max_width, w[l]);
+  }
+  // Chain contraction.  v continues the segment of its predecessor u when u is v's
+  // only distinct input and v is u's only distinct consumer.  Along a segment the
+  // finish times are running sums of the durations, so only a segment's head reads
+  // other ops (timeline frontiers, data predecessors) and only its tail is read by
+  // other ops or advances a timeline.
+  std::vector<int64_t> mp_off(V + 1, 0);
+  std::vector<int32_t> mp;  // distinct predecessors over data and issue-order edges
+  {
+    std::vector<int64_t> cnt(V + 1, 0);
+    for (int64_t v = 0; v < V; ++v) cnt[v + 1] = g->pred_off[v + 1] - g->pred_off[v];
+    for (int64_t q = 0; q < NQ; ++q)
+      for (int64_t i = g->q_off[q] + 1; i < g->q_off[q + 1]; ++i) cnt[g->q_ops[i] + 1]++;
+    for (int64_t v = 0; v < V; ++v) cnt[v + 1] += cnt[v];
+    std::vector<int32_t> tmp(cnt[V] > 0 ? cnt[V] : 1);
+    std::vector<int64_t> fill(cnt.begin(), cnt.end() - 1);
+    for (int64_t v = 0; v < V; ++v)
+      for (int64_t k = g->pred_off[v]; k < g->pred_off[v + 1]; ++k) tmp[fill[v]++] = g->pred_idx[k];
+    for (int64_t q = 0; q < NQ; ++q)
+      for (int64_t i = g->q_off[q] + 1; i < g->q_off[q + 1]; ++i) tmp[fill[g->q_ops[i]]++] = g->q_ops[i - 1];
+    mp.reserve(cnt[V]);
+    for (int64_t v = 0; v < V; ++v) {
+      std::sort(tmp.begin() + cnt[v], tmp.begin() + cnt[v + 1]);
+      int32_t prev = -1;
+      for (int64_t k = cnt[v]; k < cnt[v + 1]; ++k)
+        if (tmp[k] != prev) {
+          mp.push_back(tmp[k]);
+          prev = tmp[k];
+        }
+      mp_off[v + 1] = (int64_t)mp.size();
+    }
+  }
+  std::vector<int32_t> out_cnt(V, 0);
+  for (int32_t u : mp) out_cnt[u]++;
+  std::vector<int32_t> seg_of(V, -1), nxt(V, -1);
+  std::vector<int32_t> seg_len, seg_head, seg_tail;  // by creation order
+  for (int32_t v : order) {  // topological order
+    if (mp_off[v + 1] - mp_off[v] == 1) {
+      const int32_t u = mp[mp_off[v]];
+      const int32_t su = seg_of[u];
+      if (out_cnt[u] == 1 && seg_tail[su] == u && seg_len[su] < echo::kMaxSegment) {
+        seg_of[v] = su;
+        seg_len[su]++;
+        seg_tail[su] = v;
+        nxt[u] = v;
+        continue;
+      }
+    }
+    seg_of[v] = (int32_t)seg_len.size();
+    seg_len.push_back(1);
+    seg_head.push_back(v);
+    seg_tail.push_back(v);
+  }
+  const int64_t NSg = (int64_t)seg_len.size();
+  // segment levels: ASAP depth of the contracted graph (only heads have inputs)
+  std::vector<int32_t> seg_lvl(NSg, 0);
+  for (int32_t v : order) {
+    const int32_t sv = seg_of[v];
+    if (seg_head[sv] != v) continue;
+    int32_t lv = 0;
+    for (int64_t k = mp_off[v]; k < mp_off[v + 1]; ++k) lv = std::max(lv, seg_lvl[seg_of[mp[k]]] + 1);
+    seg_lvl[sv] = lv;
+  }
+  int64_t Ls = 0;
+  for (int64_t t = 0; t < NSg; ++t) Ls = std::max<int64_t>(Ls, seg_lvl[t] + 1);
+  b.Ls = Ls;
+  b.n_seg = NSg;
+  b.seg_lvl_off.assign(Ls + 1, 0);
+  for (int64_t t = 0; t < NSg; ++t) b.seg_lvl_off[seg_lvl[t] + 1]++;
+  for (int64_t l = 0; l < Ls; ++l) b.seg_lvl_off[l + 1] += b.seg_lvl_off[l];
+  std::vector<int32_t> seg_order(NSg);  // internal segment id -> creation id
+  {
+    std::vector<int64_t> cur(b.seg_lvl_off.begin(), b.seg_lvl_off.end() - 1);
+    for (int64_t t = 0; t < NSg; ++t) seg_order[cur[seg_lvl[t]]++] = (int32_t)t;
+  }
+  // internal numbering: segment levels in order, each segment's chain contiguous
+  b.seg_node_off.assign(NSg + 1, 0);
+  b.seg_int.assign(V, 0);
   b.int2ext.assign(V, 0);
   b.ext2int.assign(V, 0);
   {
-    std::vector<int64_t> cur(b.lvl_off.begin(), b.lvl_off.end() - 1);
-    for (int64_t v = 0; v < V; ++v) {
-      int64_t i = cur[level[v]]++;
-      b.int2ext[i] = (int32_t)v;
-      b.ext2int[v] = (int32_t)i;
+    int64_t i = 0;
+    for (int64_t t = 0; t < NSg; ++t) {
+      b.seg_node_off[t] = i;
+      for (int32_t v = seg_head[seg_order[t]]; v >= 0; v = nxt[v]) {
+        b.int2ext[i] = v;
+        b.ext2int[v] = (int32_t)i;
+        b.seg_int[i] = (int32_t)t;
+        ++i;
+      }
     }
+    b.seg_node_off[NSg] = i;
   }
   // timelines of every internal node
   b.nq_off.assign(V + 1, 0);
@@ -313,8 +404,109 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
       b.comm_sig.push_back(s);
       b.node_sig[i] = s;
     }
+    if (kd != ECHO_OP_COMPUTE) b.non_compute.push_back((int32_t)i);
+  }
+  for (int32_t r = 0; r < R; ++r) {
+    const int64_t a = g->q_off[(int64_t)r * NS], z = g->q_off[(int64_t)r * NS + 1];
+    for (int64_t p = a; p < z; p += echo::kOverlapChunk) {
+      b.ov_chunks.push_back(r);
+      b.ov_chunks.push_back(p);
+    }
+  }
+  b.blk_words.assign(Ls, 0);
+  for (int64_t l = 0; l < Ls; ++l) {
+    int64_t w = 0;
+    for (int64_t t = b.seg_lvl_off[l]; t < b.seg_lvl_off[l + 1]; ++t) {
+      const int64_t h = b.seg_node_off[t], z = b.seg_node_off[t + 1] - 1;
+      const int64_t nqf = b.nq_off[h + 1] - b.nq_off[h], ndp = b.dp_off[h + 1] - b.dp_off[h];
+      const int64_t nql = b.nq_off[z + 1] - b.nq_off[z];
+      if (nqf > 0xFFFF || ndp > 0xFFFF || nql > 0xFFFF) b.stageable = false;
+      w += 4 + nqf + ndp + nql;
+    }
+    b.blk_words[l] = (w + 3) & ~(int64_t)3;
   }
   return ECHO_OK;
+}
+
+// Ring sizes of the staged compose kernels for scenario blocks of `sigma`.  The
+// duration and record rings must hold two consecutive segment levels (the one
+// being composed and the one before it, which slower threads may still read);
+// whatever more they hold is prefetch look-ahead.  Preference: a larger duration
+// ring, then a larger value ring (more predecessors served from shared memory).
+echo::StagedPlan plan_staged(const GraphBuild &b, int sigma, size_t smem_cap) {
+  echo::StagedPlan best;
+  if (!b.stageable || b.Ls == 0) return best;
+  const int32_t NQ = b.R * b.NS;
+  auto pow2 = [](int64_t x) {
+    int k = 0;
+    while (((int64_t)1 << k) < x) ++k;
+    return k;
+  };
+  int64_t rows2 = 0, words2 = 0, segmax = 0, prow = 0, pword = 0;
+  for (int64_t l = 0; l < b.Ls; ++l) {
+    const int64_t r = b.seg_node_off[b.seg_lvl_off[l + 1]] - b.seg_node_off[b.seg_lvl_off[l]];
+    rows2 = std::max(rows2, r + prow);
+    words2 = std::max(words2, b.blk_words[l] + pword);
+    segmax = std::max(segmax, b.seg_lvl_off[l + 1] - b.seg_lvl_off[l]);
+    prow = r;
+    pword = b.blk_words[l];
+  }
+  const int dmin = std::max(pow2(rows2), 4), rmin = std::max(pow2(words2), 4);
+  const int vwant = std::min(std::max(pow2(4 * segmax), 6), 12);
+  for (int d = dmin + 2; d >= dmin; --d)
+    for (int v = vwant; v >= 6; --v)
+      for (int r = rmin + 1; r >= rmin; --r) {
+        const size_t need = echo::staged_layout(NQ, sigma, v, d, r).total;
+        if (need <= smem_cap && d < 31 && r < 31) {
+          best.ok = true;
+          best.dring_log2 = d;
+          best.vring_log2 = v;
+          best.rring_log2 = r;
+          best.smem = need;
+          return best;
+        }
+      }
+  return best;
+}
+
+// Record blocks of every segment level for a value ring of 2^vlog2 segments, and
+// the per-level metadata (word offset of the block, first node, first segment).
+void build_records(const GraphBuild &b, int vlog2, std::vector<uint32_t> &recs, std::vector<uint32_t> &meta) {
+  const int64_t R = (int64_t)1 << vlog2;
+  recs.clear();
+  meta.assign(4 * (b.Ls + 1), 0);
+  for (int64_t l = 0; l < b.Ls; ++l) {
+    const int64_t s0 = b.seg_lvl_off[l], s1 = b.seg_lvl_off[l + 1];
+    const int64_t i0 = b.seg_node_off[s0];
+    const size_t base = recs.size();
+    meta[4 * l] = (uint32_t)base;
+    meta[4 * l + 1] = (uint32_t)i0;
+    meta[4 * l + 2] = (uint32_t)s0;
+    recs.resize(base + 4 * (s1 - s0), 0);
+    for (int64_t t = s0; t < s1; ++t) {
+      const int64_t h = b.seg_node_off[t], z = b.seg_node_off[t + 1] - 1;
+      const int64_t nqf = b.nq_off[h + 1] - b.nq_off[h], ndp = b.dp_off[h + 1] - b.dp_off[h];
+      const int64_t nql = b.nq_off[z + 1] - b.nq_off[z];
+      const size_t hd = base + 4 * (t - s0);
+      recs[hd] = (uint32_t)(recs.size() - base);
+      recs[hd + 1] = (uint32_t)(nqf | (ndp << 16));
+      recs[hd + 2] = (uint32_t)(h - i0);
+      recs[hd + 3] = (uint32_t)((z - h + 1) | (nql << 16));
+      for (int64_t q = b.nq_off[h]; q < b.nq_off[h + 1]; ++q) recs.push_back((uint32_t)b.nq[q]);
+      for (int64_t q = b.dp_off[h]; q < b.dp_off[h + 1]; ++q) {
+        // a predecessor of a head is the tail of its segment; its value-ring slot is
+        // rewritten by segment seg+R, which must not be in segment levels <= l
+        const int64_t u = b.dp[q], su = b.seg_int[u];
+        recs.push_back(su + R >= s1 ? (uint32_t)su : ((uint32_t)u | echo::kFarRef));
+      }
+      for (int64_t q = b.nq_off[z]; q < b.nq_off[z + 1]; ++q) recs.push_back((uint32_t)b.nq[q]);
+    }
+    while (recs.size() % 4) recs.push_back(0);
+  }
+  meta[4 * b.Ls] = (uint32_t)recs.size();
+  meta[4 * b.Ls + 1] = (uint32_t)b.V;
+  meta[4 * b.Ls + 2] = (uint32_t)b.n_seg;
+  if (recs.empty()) recs.assign(4, 0);
 }
 
 // ------------------------------------------------------------------------------------
@@ -336,7 +528,9 @@ struct echo_ctx {
   GraphBuild gb;
   std::vector<void *> graph_allocs, scen_allocs;
   // device graph
-  int64_t *lvl_off = nullptr, *nq_off = nullptr, *dp_off = nullptr, *q_off = nullptr;
+  int64_t *seg_lvl_off = nullptr, *seg_node_off = nullptr, *nq_off = nullptr, *dp_off = nullptr, *q_off = nullptr;
+  int64_t *ov_chunks = nullptr;
+  int32_t *non_compute = nullptr;
   int32_t *nq = nullptr, *dp = nullptr, *q_ops = nullptr, *int2ext = nullptr, *ext2int = nullptr;
   int32_t *node_sig = nullptr, *comm_node = nullptr, *comm_sig = nullptr, *sig_count = nullptr;
   uint8_t *kcl = nullptr, *is_comm = nullptr, *local = nullptr;
@@ -344,14 +538,24 @@ struct echo_ctx {
   int32_t *status = nullptr;
   // scenarios
   int32_t S = 0, C = 0, sigma = 1;
-  size_t scen_vs = 0;  // V*S the scenario buffers were sized for
+  size_t scen_vs = 0;  // elements of each [op][scenario] matrix (blocked layout, padded)
+  echo::MatLayout lay{0, 0};
   ChunkTable tbl{};
   double *prm = nullptr, *sf = nullptr, *sums = nullptr, *comm_sum = nullptr, *cc_ns = nullptr;
   int64_t *raw = nullptr, *dur = nullptr, *f[2] = {nullptr, nullptr}, *mk = nullptr, *cc_dur = nullptr;
   int64_t *gfrontier = nullptr;
-  uint8_t *ov[2] = {nullptr, nullptr};
+  int64_t *deff[2] = {nullptr, nullptr};  // durations of the validator's passes
+  uint8_t *ov = nullptr;
+  uint32_t *d_recs = nullptr, *d_meta = nullptr;
+  echo::StagedPlan plan;
+  uint32_t rec_words = 0;
   std::vector<double> h_sums, h_maxsf;
-  int final_f = 0, final_ov = -1;
+  int final_f = 0;
+  const int64_t *final_d = nullptr;
+  bool have_ov = false;
+  int kernel_choice = 0;            // 0 automatic, 1 direct, 2 staged, 3 pipelined (tuning and tests)
+  long long wait_limit_cycles = 0;  // bound of every device-side wait
+  int32_t skip_level = -1;          // failure injection for tests
   // scratch for readback / queries
   void *stage = nullptr;
   size_t stage_bytes = 0;
@@ -450,6 +654,10 @@ int check_ctx(echo_ctx *c) {
 }
 
 int pick_sigma(int32_t S, int sms) {
+  if (const char *e = std::getenv("ECHO_SIGMA")) {  // tuning override: 1, 2, 4, 8 or 16
+    int v = std::atoi(e);
+    if (v == 1 || v == 2 || v == 4 || v == 8 || v == 16) return v;
+  }
   int want = (S + sms - 1) / std::max(sms, 1);
   int s = 1;
   while (s < want && s < 16) s <<= 1;
@@ -555,6 +763,17 @@ int echo_create(echo_ctx **out, int device, void *cuda_stream) {
     return ECHO_E_OOM;
   }
   c->status = static_cast<int32_t *>(st);
+  if (const char *e = std::getenv("ECHO_COMPOSE_KERNEL")) {  // tuning and tests: force a compose kernel
+    const std::string k(e);
+    c->kernel_choice = k == "direct" ? 1 : k == "staged" ? 2 : k == "pipelined" ? 3 : 0;
+  }
+  // device waits give up after 2 s (tests shorten this and inject a level that never arrives)
+  int clock_khz = 0;
+  cudaDeviceGetAttribute(&clock_khz, cudaDevAttrClockRate, device);
+  double limit_ms = 2000.0;
+  if (const char *e = std::getenv("ECHO_TEST_WAIT_LIMIT_MS")) limit_ms = std::atof(e);
+  c->wait_limit_cycles = (long long)(std::max(clock_khz, 1000) * limit_ms);
+  if (const char *e = std::getenv("ECHO_TEST_SKIP_LEVEL")) c->skip_level = std::atoi(e);
   *out = c;
   return ECHO_OK;
 }
@@ -602,7 +821,9 @@ int echo_load_graph(echo_ctx *c, const echo_graph_desc *g) {
   c->gb = std::move(b);
   const GraphBuild &B = c->gb;
   auto &o = c->graph_allocs;
-  if ((rc = upload(c, o, &c->lvl_off, B.lvl_off)) || (rc = upload(c, o, &c->nq_off, B.nq_off)) ||
+  if ((rc = upload(c, o, &c->seg_lvl_off, B.seg_lvl_off)) || (rc = upload(c, o, &c->seg_node_off, B.seg_node_off)) ||
+      (rc = upload(c, o, &c->ov_chunks, B.ov_chunks)) || (rc = upload(c, o, &c->non_compute, B.non_compute)) ||
+      (rc = upload(c, o, &c->nq_off, B.nq_off)) ||
       (rc = upload(c, o, &c->nq, B.nq)) || (rc = upload(c, o, &c->dp_off, B.dp_off)) ||
       (rc = upload(c, o, &c->dp, B.dp)) || (rc = upload(c, o, &c->q_off, B.q_off)) ||
       (rc = upload(c, o, &c->q_ops, B.q_ops_int)) || (rc = upload(c, o, &c->int2ext, B.int2ext)) ||
@@ -647,8 +868,11 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
 
   CK(cudaStreamSynchronize(c->stream), "cudaStreamSynchronize");
   c->state = 1;
-  const size_t VS = (size_t)V * S;
   const int sigma = pick_sigma(S, c->sms);
+  int slog2 = 0;
+  while ((1 << slog2) < sigma) ++slog2;
+  // [op][scenario] matrices are stored in scenario blocks of sigma (the last padded)
+  const size_t VS = (size_t)V * (size_t)((S + sigma - 1) / sigma) * sigma;
   const int32_t G = (int32_t)B.sigs.size();
   if (c->scen_vs != VS || c->S != S || c->C != C || c->sigma != sigma) {
     free_all(c->scen_allocs);
@@ -659,9 +883,9 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     int64_t nblk = (S + sigma - 1) / sigma;
     if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sf, (size_t)C * S)) ||
         (rc = dalloc(c, o, &c->sums, (size_t)S)) || (rc = dalloc(c, o, &c->comm_sum, (size_t)S)) ||
-        (rc = dalloc(c, o, &c->raw, VS)) || (rc = dalloc(c, o, &c->dur, VS)) ||
+        (rc = dalloc(c, o, &c->raw, (size_t)V * S)) || (rc = dalloc(c, o, &c->dur, VS)) ||
         (rc = dalloc(c, o, &c->f[0], VS)) || (rc = dalloc(c, o, &c->f[1], VS)) ||
-        (rc = dalloc(c, o, &c->ov[0], VS)) || (rc = dalloc(c, o, &c->ov[1], VS)) ||
+        (rc = dalloc(c, o, &c->deff[0], VS)) || (rc = dalloc(c, o, &c->ov, VS)) ||
         (rc = dalloc(c, o, &c->mk, (size_t)S)) || (rc = dalloc(c, o, &c->cc_ns, (size_t)G * S)) ||
         (rc = dalloc(c, o, &c->cc_dur, (size_t)G * S)) ||
         (!in_smem && (rc = dalloc(c, o, &c->gfrontier, (size_t)nblk * B.R * B.NS * sigma)))) {
@@ -669,10 +893,44 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
       return rc;
     }
     if (in_smem) c->gfrontier = nullptr;
+    // padding lanes of the duration matrices stay zero
+    CK(cudaMemsetAsync(c->dur, 0, VS * sizeof(int64_t), c->stream), "memset");
+    CK(cudaMemsetAsync(c->deff[0], 0, VS * sizeof(int64_t), c->stream), "memset");
+    c->deff[1] = nullptr;  // second validator buffer: allocated when refine_passes > 1
+    // launch shape of the staged kernels (threads and blocks per SM may be overridden
+    // for tuning: ECHO_STAGED_THREADS, ECHO_BLOCKS_PER_SM)
+    int optin = 0, per_sm = 0;
+    cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->device);
+    cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, c->device);
+    int threads = sigma == 16 ? 1024 : sigma == 8 ? 512 : sigma == 4 ? 256 : 512;
+    int bps = 1;
+    if (const char *e = std::getenv("ECHO_STAGED_THREADS")) threads = std::atoi(e);
+    if (const char *e = std::getenv("ECHO_BLOCKS_PER_SM")) bps = std::max(1, std::atoi(e));
+    const size_t cap = std::min((size_t)std::max(optin - 1024, 0), (size_t)(per_sm / bps) - 1024);
+    c->plan = plan_staged(B, sigma, cap);
+    c->plan.threads = threads;
+    if (c->plan.ok) {
+      // the pipelined kernel moves whole rows of even width and arms each level's
+      // byte count on one mbarrier (transaction counts stay below 2^20)
+      int64_t max_bytes = 0;
+      for (int64_t l = 0; l < B.Ls; ++l) {
+        const int64_t rows = B.seg_node_off[B.seg_lvl_off[l + 1]] - B.seg_node_off[B.seg_lvl_off[l]];
+        max_bytes = std::max(max_bytes, rows * sigma * 8 + B.blk_words[l] * 4 + 32);
+      }
+      c->plan.pipelined = sigma % 2 == 0 && max_bytes < (1 << 20);
+      std::vector<uint32_t> recs, meta;
+      build_records(B, c->plan.vring_log2, recs, meta);
+      c->rec_words = meta[4 * B.Ls];
+      if ((rc = upload(c, o, &c->d_recs, recs)) || (rc = upload(c, o, &c->d_meta, meta))) {
+        free_all(c->scen_allocs);
+        return rc;
+      }
+    }
     c->scen_vs = VS;
     c->S = S;
     c->C = C;
     c->sigma = sigma;
+    c->lay = echo::MatLayout{V, slog2};
   }
   c->tbl = tbl;
   c->h_maxsf = maxsf;
@@ -684,9 +942,11 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   CK(cudaMemsetAsync(c->sums, 0, S * sizeof(double), c->stream), "memset");
   CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
   if (V > 0) {
-    CK(cudaMemcpyAsync(c->raw, sc->dur, VS * sizeof(int64_t), cudaMemcpyHostToDevice, c->stream), "duration upload");
+    CK(cudaMemcpyAsync(c->raw, sc->dur, (size_t)V * S * sizeof(int64_t), cudaMemcpyHostToDevice, c->stream),
+       "duration upload");
     CK(timed(c, "permute_rows", [&] {
-         return echo::launch_permute_rows(c->raw, c->int2ext, c->local, V, S, c->dur, c->sums, c->status, c->stream);
+         return echo::launch_permute_rows(c->raw, c->int2ext, c->local, V, S, c->lay, c->dur, c->sums, c->status,
+                                          c->stream);
        }), "permute_rows launch");
   }
   c->h_sums.assign(S, 0.0);
@@ -715,7 +975,7 @@ int echo_estimate_collectives(echo_ctx *c) {
      }), "cc_estimate launch");
   CK(timed(c, "cc_scatter", [&] {
        return echo::launch_cc_scatter(c->comm_node, c->comm_sig, (int64_t)B.comm_node.size(), c->cc_dur, S,
-                                      c->dur, c->stream);
+                                      c->lay, c->dur, c->stream);
      }), "cc_scatter launch");
   std::vector<double> comm(S, 0.0);
   CK(cudaMemcpyAsync(comm.data(), c->comm_sum, S * sizeof(double), cudaMemcpyDeviceToHost, c->stream), "readback");
@@ -739,47 +999,95 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   int32_t refine = opts ? opts->refine_passes : 1;
   if (refine < 0 || refine > 8) return set_err(c, ECHO_E_INVALID_ARG, "refine_passes outside [0, 8]");
   const GraphBuild &B = c->gb;
-  echo::ComposeArgs a{};
-  a.V = B.V;
-  a.S = c->S;
-  a.L = (int32_t)B.L;
-  a.n_queues = B.R * B.NS;
-  a.lvl_off = c->lvl_off;
-  a.nq_off = c->nq_off;
-  a.nq = c->nq;
-  a.dp_off = c->dp_off;
-  a.dp = c->dp;
-  a.kcl = c->kcl;
-  a.dur = c->dur;
-  a.sf = c->sf;
-  a.makespan = c->mk;
-  a.gfrontier = c->gfrontier;
-  echo::OverlapArgs o{};
-  o.S = c->S;
-  o.n_ranks = B.R;
-  o.n_streams = B.NS;
-  o.q_off = c->q_off;
-  o.q_ops = c->q_ops;
-  o.is_comm = c->is_comm;
-  o.kcl = c->kcl;
-  o.dur = c->dur;
-  o.sf = c->sf;
+  if (refine > 1 && !c->deff[1]) {
+    if ((rc = dalloc(c, c->scen_allocs, &c->deff[1], c->scen_vs))) return rc;
+    CK(cudaMemsetAsync(c->deff[1], 0, c->scen_vs * sizeof(int64_t), c->stream), "memset");
+  }
   c->state = 3;
-  a.ov = nullptr;
-  a.f = c->f[0];
-  CK(timed(c, "compose", [&] { return echo::launch_compose(a, c->sigma, c->stream); }), "compose launch");
+  // one composition with durations `d` into `f`
+  auto compose_pass = [&](const int64_t *d, int64_t *f) -> cudaError_t {
+    if (c->plan.ok && c->kernel_choice != 1) {
+      echo::StagedArgs a{};
+      a.S = c->S;
+      a.L = (int32_t)B.Ls;
+      a.n_queues = B.R * B.NS;
+      a.n_rows = (uint32_t)B.V;
+      a.n_words = c->rec_words;
+      a.vlog2 = c->plan.vring_log2;
+      a.dlog2 = c->plan.dring_log2;
+      a.rlog2 = c->plan.rring_log2;
+      a.meta = c->d_meta;
+      a.recs = c->d_recs;
+      a.dur = d;
+      a.f = f;
+      a.makespan = c->mk;
+      a.status = c->status;
+      a.wait_limit_cycles = c->wait_limit_cycles;
+      a.skip_level = c->skip_level;
+      const bool pipe = c->plan.pipelined && (c->kernel_choice == 0 || c->kernel_choice == 3);
+      if (pipe)
+        return timed(c, "compose", [&] { return echo::launch_compose_pipelined(a, c->sigma, c->plan, c->stream); });
+      return timed(c, "compose", [&] { return echo::launch_compose_staged(a, c->sigma, c->plan, c->stream); });
+    }
+    echo::ComposeArgs a{};
+    a.V = B.V;
+    a.lay = c->lay;
+    a.S = c->S;
+    a.L = (int32_t)B.Ls;
+    a.n_queues = B.R * B.NS;
+    a.seg_lvl_off = c->seg_lvl_off;
+    a.seg_node_off = c->seg_node_off;
+    a.nq_off = c->nq_off;
+    a.nq = c->nq;
+    a.dp_off = c->dp_off;
+    a.dp = c->dp;
+    a.dur = d;
+    a.f = f;
+    a.makespan = c->mk;
+    a.gfrontier = c->gfrontier;
+    return timed(c, "compose_direct", [&] { return echo::launch_compose(a, c->sigma, c->stream); });
+  };
+  CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
+  CK(compose_pass(c->dur, c->f[0]), "compose launch");
+  const int64_t *d_used = c->dur;
   for (int32_t p = 1; p <= refine; ++p) {
+    echo::OverlapArgs o{};
+    o.lay = c->lay;
+    o.S = c->S;
+    o.n_streams = B.NS;
+    o.n_chunks = (int64_t)B.ov_chunks.size() / 2;
+    o.chunks = c->ov_chunks;
+    o.q_off = c->q_off;
+    o.q_ops = c->q_ops;
+    o.is_comm = c->is_comm;
+    o.kcl = c->kcl;
     o.f = c->f[(p - 1) % 2];
-    o.ov_prev = p > 1 ? c->ov[(p - 2) % 2] : nullptr;
-    o.ov = c->ov[(p - 1) % 2];
+    o.d_used = d_used;
+    o.d_orig = c->dur;
+    o.sf = c->sf;
+    o.d_next = c->deff[(p - 1) % 2];
+    o.ov = c->ov;
     CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");
-    a.ov = c->ov[(p - 1) % 2];
-    a.f = c->f[p % 2];
-    CK(timed(c, "compose", [&] { return echo::launch_compose(a, c->sigma, c->stream); }), "compose launch");
+    CK(timed(c, "copy_rows", [&] {
+         return echo::launch_copy_rows(c->non_compute, (int64_t)B.non_compute.size(), c->S, c->lay, c->dur,
+                                       o.d_next, c->stream);
+       }), "copy_rows launch");
+    CK(compose_pass(o.d_next, c->f[p % 2]), "compose launch");
+    d_used = o.d_next;
   }
   c->final_f = refine % 2;
-  c->final_ov = refine > 0 ? (refine - 1) % 2 : -1;
+  c->final_d = d_used;
+  c->have_ov = refine > 0;
   c->state = 4;
+  return ECHO_OK;
+}
+
+// Device-side failures of the last composition (a bounded wait that gave up).
+static int composition_status(echo_ctx *c) {
+  int32_t st = 0;
+  int rc = sync_status(c, &st);
+  if (rc) return rc;
+  if (st == echo::kDevTimeout) return set_err(c, ECHO_E_TIMEOUT, "a device-side wait of the composer gave up");
   return ECHO_OK;
 }
 
@@ -793,18 +1101,18 @@ int echo_read_times(echo_ctx *c, int64_t op0, int64_t op1, int64_t *start, int64
   int rc = check_ctx(c);
   if (rc) return rc;
   if ((rc = read_range_check(c, op0, op1, 4))) return rc;
+  if ((rc = composition_status(c))) return rc;
   const int32_t S = c->S;
   const int64_t rows_per = std::max<int64_t>(1, (int64_t)(64 << 20) / S);
   if ((rc = stage_reserve(c, (size_t)std::min<int64_t>(rows_per, std::max<int64_t>(op1 - op0, 1)) * S * 16)))
     return rc;
-  const uint8_t *ov = c->final_ov >= 0 ? c->ov[c->final_ov] : nullptr;
   for (int64_t a = op0; a < op1; a += rows_per) {
     int64_t b = std::min(op1, a + rows_per);
     int64_t n = (b - a) * S;
     int64_t *ds = static_cast<int64_t *>(c->stage);
     int64_t *df = ds + n;
     CK(timed(c, "readback", [&] {
-         return echo::launch_readback(c->ext2int, a, b, S, c->f[c->final_f], c->dur, ov, c->kcl, c->sf,
+         return echo::launch_readback(c->ext2int, a, b, S, c->lay, c->f[c->final_f], c->final_d,
                                       start ? ds : nullptr, finish ? df : nullptr, c->stream);
        }), "readback launch");
     if (start) CK(cudaMemcpyAsync(start + (a - op0) * S, ds, n * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream), "D2H");
@@ -819,6 +1127,7 @@ int echo_read_makespan(echo_ctx *c, int64_t *out) {
   if (rc) return rc;
   if (!out) return set_err(c, ECHO_E_INVALID_ARG, "output is NULL");
   if (c->state < 4) return set_err(c, ECHO_E_STATE, "compose first");
+  if ((rc = composition_status(c))) return rc;
   CK(cudaMemcpyAsync(out, c->mk, c->S * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream), "D2H");
   CK(cudaStreamSynchronize(c->stream), "makespan readback");
   return ECHO_OK;
@@ -855,13 +1164,14 @@ int echo_read_overlap(echo_ctx *c, int64_t op0, int64_t op1, uint8_t *out) {
   const int64_t rows_per = std::max<int64_t>(1, (int64_t)(64 << 20) / S);
   if ((rc = stage_reserve(c, (size_t)std::min<int64_t>(rows_per, std::max<int64_t>(op1 - op0, 1)) * S * 16)))
     return rc;
-  const uint8_t *ov = c->final_ov >= 0 ? c->ov[c->final_ov] : nullptr;
+  if ((rc = composition_status(c))) return rc;
+  const uint8_t *ov = c->have_ov ? c->ov : nullptr;
   for (int64_t a = op0; a < op1; a += rows_per) {
     int64_t b = std::min(op1, a + rows_per);
     int64_t n = (b - a) * S;
     uint8_t *d = static_cast<uint8_t *>(c->stage);
     CK(timed(c, "read_overlap", [&] {
-         return echo::launch_read_ov(c->ext2int, a, b, S, ov, c->kcl, d, c->stream);
+         return echo::launch_read_ov(c->ext2int, a, b, S, c->lay, ov, c->kcl, d, c->stream);
        }), "read_overlap launch");
     CK(cudaMemcpyAsync(out + (a - op0) * S, d, n, cudaMemcpyDeviceToHost, c->stream), "D2H");
     CK(cudaStreamSynchronize(c->stream), "read_overlap");
@@ -937,6 +1247,8 @@ int echo_graph_info_get(echo_ctx *c, echo_graph_info *info) {
   info->n_queue_entries = B.QE;
   info->n_comm_ops = (int64_t)B.comm_node.size();
   info->n_signatures = (int64_t)B.sigs.size();
+  info->n_segments = B.n_seg;
+  info->n_segment_levels = B.Ls;
   info->n_ranks = B.R;
   info->n_streams = B.NS;
   info->sigma = c->sigma;

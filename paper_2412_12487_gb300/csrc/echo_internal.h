@@ -10,10 +10,31 @@ namespace echo {
 constexpr int kMaxStreams = 16;
 constexpr int kMaxChunk = 16;
 constexpr uint8_t kNotSlowable = 0xFF;
-constexpr int kComposeThreads = 512;
+constexpr int kComposeThreads = 512;       // direct compose kernel
+constexpr int kMetaChunk = 128;            // segment levels of metadata staged at a time
+constexpr int kMetaCap = 136;              // metadata entries per staging buffer (>= kMetaChunk + 1)
+constexpr uint32_t kFarRef = 0x80000000u;  // predecessor reference read from global memory
+constexpr int kOverlapChunk = 128;         // compute ops per overlap-test thread
+constexpr int kMaxSegment = 64;            // longest serial chain composed as one segment
+constexpr int kPipeStages = 16;            // stages (mbarrier pairs) of the pipelined compose
+constexpr int kPipeConsumerWarps = 16;     // composing warps of the pipelined compose
 
 // device status word: first error wins
-enum DeviceStatus : int32_t { kDevOk = 0, kDevNegativeDuration = 1, kDevCcOverflow = 2 };
+enum DeviceStatus : int32_t { kDevOk = 0, kDevNegativeDuration = 1, kDevCcOverflow = 2, kDevTimeout = 3 };
+
+// Device layout of every [op][scenario] matrix (durations, finish times, validator
+// outputs): scenario blocks of 2^slog2 scenarios, block b holding a contiguous
+// [V][2^slog2] array, so one thread block's rows of consecutive ops form one
+// contiguous range.  Lanes of a partial last block are padding (kept at zero in
+// the duration matrices).
+struct MatLayout {
+  int64_t V;
+  int32_t slog2;
+  __host__ __device__ int64_t at(int64_t i, int32_t s) const {
+    return (((int64_t)(s >> slog2) * V + i) << slog2) + (s & ((1 << slog2) - 1));
+  }
+  __host__ __device__ int64_t block(int32_t b) const { return ((int64_t)b * V) << slog2; }
+};
 
 struct ChunkTable {
   int32_t n;
@@ -32,32 +53,90 @@ struct ScenParams {  // device arrays [S]
   const double *alpha, *bwa, *lata, *bwe, *late, *delta;
 };
 
+// Direct compose: graph structure and durations read from global memory.  The
+// graph is composed segment level by segment level; a segment is a serial chain
+// whose nodes are numbered consecutively.
 struct ComposeArgs {
   int64_t V;
-  int32_t S, L;
+  MatLayout lay;
+  int32_t S, L;                               // L: segment levels
   int32_t n_queues;
-  const int64_t *lvl_off;                     // [L+1]
+  const int64_t *seg_lvl_off;                 // [L+1] segments of each level
+  const int64_t *seg_node_off;                // [n_seg+1] nodes of each segment
   const int64_t *nq_off; const int32_t *nq;   // timelines of each node
   const int64_t *dp_off; const int32_t *dp;   // data predecessors (internal ids)
-  const uint8_t *kcl;                         // kernel class or kNotSlowable
-  const int64_t *dur;                         // [V][S]
-  const uint8_t *ov;                          // [V][S] slow this op? (nullptr: raw durations)
-  const double *sf;                           // [C][S]
-  int64_t *f;                                 // [V][S] finish times (out)
+  const int64_t *dur;                         // durations of this pass (MatLayout)
+  int64_t *f;                                 // finish times (MatLayout, out)
   int64_t *makespan;                          // [S] (out)
   int64_t *gfrontier;                         // [grid][n_queues][sigma] when not in smem
 };
 
+// Staged and pipelined compose: per-segment-level records and duration rows are
+// copied into shared-memory rings ahead of use.  Record block of a level (32-bit
+// words): for each segment, 4 header words {offset of its entries in the block,
+// nqf | ndp << 16, first node - level's first node, length | nql << 16}; entries =
+// the head's nqf timeline ids, its ndp predecessor references (a segment id for
+// the value ring, or a node id with kFarRef set, read from global memory), the
+// tail's nql timeline ids.  Blocks are padded to 4 words.
+struct StagedArgs {
+  int32_t S, L, n_queues;        // L: segment levels
+  uint32_t n_rows, n_words;      // nodes; words of all record blocks
+  int32_t vlog2, dlog2, rlog2;   // log2 sizes: value ring (segments), duration ring (rows), record ring (words)
+  const uint32_t *meta;          // [4*(L+1)]: record word offset, first node, first segment, 0
+  const uint32_t *recs;          // record blocks
+  const int64_t *dur;            // durations (MatLayout)
+  int64_t *f;                    // finish times (MatLayout, out)
+  int64_t *makespan;             // [S] (out)
+  // pipelined kernel only
+  int32_t *status;               // device status word (kDevTimeout when a bounded wait gives up)
+  long long wait_limit_cycles;   // bound of every mbarrier wait, in SM clock cycles
+  int32_t skip_level;            // failure injection for tests: this level is never filled (-1: none)
+};
+
+// Plan of the staged kernels for one (graph, sigma); see plan_staged().
+struct StagedPlan {
+  bool ok = false;
+  bool pipelined = false;  // bulk-copy producer warp (even sigma)
+  int threads = 512;       // threads per block of the staged kernel
+  int vring_log2 = 0, dring_log2 = 0, rring_log2 = 0;  // sizes (segments, rows, words)
+  size_t smem = 0;
+};
+
+// Shared-memory layout of the staged kernels (byte offsets).  Every region starts
+// on a 16-byte boundary, as 16-byte copy destinations require.
+struct StagedLayout {
+  size_t hist, meta, fr, vr, dr, rr, total;
+};
+__host__ __device__ inline size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
+__host__ __device__ inline StagedLayout staged_layout(int32_t n_queues, int sigma, int vlog2, int dlog2,
+                                                      int rlog2) {
+  StagedLayout L;
+  L.hist = 128;                        // [0, 128): per-scenario makespans
+  L.meta = L.hist + 16 * 8;            // 16 copy-group extents
+  L.fr = L.meta + round16((size_t)2 * kMetaCap * 16);
+  L.vr = L.fr + round16((size_t)n_queues * sigma * 8);
+  L.dr = L.vr + round16(((size_t)1 << vlog2) * sigma * 8);
+  L.rr = L.dr + round16(((size_t)1 << dlog2) * sigma * 8);
+  L.total = L.rr + round16(((size_t)1 << rlog2) * 4);
+  return L;
+}
+
+// Validator: for each compute op, whether its interval overlaps a comm op of its
+// rank, and the duration to use in the next composition.
 struct OverlapArgs {
-  int32_t S, n_ranks, n_streams;
+  MatLayout lay;
+  int32_t S, n_streams;
+  int64_t n_chunks;
+  const int64_t *chunks;   // [n_chunks][2]: (rank, first compute-timeline position)
   const int64_t *q_off; const int32_t *q_ops;  // timelines in internal ids
-  const uint8_t *is_comm;                      // [V]
-  const uint8_t *kcl;                          // [V]
-  const int64_t *dur;                          // [V][S]
-  const uint8_t *ov_prev;                      // durations of the pass that produced f
-  const double *sf;
-  const int64_t *f;                            // [V][S]
-  uint8_t *ov;                                 // [V][S] (out)
+  const uint8_t *is_comm;  // [V]
+  const uint8_t *kcl;      // [V]
+  const int64_t *f;        // finish times of the last pass
+  const int64_t *d_used;   // durations of the last pass
+  const int64_t *d_orig;   // durations before any slowdown
+  const double *sf;        // [C][S]
+  int64_t *d_next;         // (out, compute rows)
+  uint8_t *ov;             // (out, compute rows)
 };
 
 // kernels.cu
@@ -65,22 +144,25 @@ cudaError_t launch_cc_estimate(const CcSig *sig, int32_t G, ScenParams p, int32_
                                const ChunkTable &tbl, const int32_t *sig_count, double *cc_ns,
                                int64_t *cc_dur, double *comm_sum, int32_t *status, cudaStream_t st);
 cudaError_t launch_cc_scatter(const int32_t *comm_node, const int32_t *comm_sig, int64_t n_comm,
-                              const int64_t *cc_dur, int32_t S, int64_t *dur, cudaStream_t st);
+                              const int64_t *cc_dur, int32_t S, MatLayout lay, int64_t *dur, cudaStream_t st);
 cudaError_t launch_cc_query(int64_t n, const uint8_t *type, const uint8_t *algo, const int64_t *nbytes,
                             const int32_t *N, const int32_t *M, const double *lg, ScenParams p,
                             const ChunkTable &tbl, double *out, cudaStream_t st);
 cudaError_t launch_permute_rows(const int64_t *raw, const int32_t *int2ext, const uint8_t *local,
-                                int64_t V, int32_t S, int64_t *dur, double *sums, int32_t *status,
+                                int64_t V, int32_t S, MatLayout lay, int64_t *dur, double *sums, int32_t *status,
                                 cudaStream_t st);
 cudaError_t launch_compose(const ComposeArgs &a, int sigma, cudaStream_t st);
+cudaError_t launch_compose_staged(const StagedArgs &a, int sigma, const StagedPlan &plan, cudaStream_t st);
+cudaError_t launch_compose_pipelined(const StagedArgs &a, int sigma, const StagedPlan &plan, cudaStream_t st);
 cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st);
-cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S,
-                            const int64_t *f, const int64_t *dur, const uint8_t *ov,
-                            const uint8_t *kcl, const double *sf, int64_t *start, int64_t *finish,
+cudaError_t launch_copy_rows(const int32_t *rows, int64_t n_rows, int32_t S, MatLayout lay, const int64_t *src,
+                             int64_t *dst, cudaStream_t st);
+cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
+                            const int64_t *f, const int64_t *d, int64_t *start, int64_t *finish,
                             cudaStream_t st);
 cudaError_t launch_read_cc(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S,
                            const int32_t *node_sig, const double *cc_ns, double *out, cudaStream_t st);
-cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S,
+cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
                            const uint8_t *ov, const uint8_t *kcl, uint8_t *out, cudaStream_t st);
 size_t compose_smem_bytes(int32_t n_queues, int sigma, bool *frontier_in_smem);
 

@@ -17,7 +17,7 @@ namespace echo {
 
 namespace {
 
-constexpr int kAR = 0, kAG = 1, kRS = 2, kSR = 3;
+constexpr int kAR = 0, kAG = 1, kSR = 3;  // reduce-scatter (2) takes the generic ring path
 constexpr int kRing = 0, kTree = 1;
 
 __device__ __forceinline__ int64_t cdiv64(int64_t a, int64_t b) { return (a + b - 1) / b; }
@@ -114,14 +114,14 @@ __global__ void cc_estimate_kernel(const CcSig *__restrict__ sig, int32_t G, Sce
 
 // every comm node takes its signature's duration row
 __global__ void cc_scatter_kernel(const int32_t *__restrict__ comm_node, const int32_t *__restrict__ comm_sig,
-                                  int64_t n_comm, const int64_t *__restrict__ cc_dur, int32_t S,
+                                  int64_t n_comm, const int64_t *__restrict__ cc_dur, int32_t S, MatLayout lay,
                                   int64_t *__restrict__ dur) {
   int64_t total = n_comm * S;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
        idx += (int64_t)gridDim.x * blockDim.x) {
     int64_t c = idx / S;
     int32_t s = (int32_t)(idx - c * S);
-    dur[(int64_t)comm_node[c] * S + s] = cc_dur[(int64_t)comm_sig[c] * S + s];
+    dur[lay.at(comm_node[c], s)] = cc_dur[(int64_t)comm_sig[c] * S + s];
   }
 }
 
@@ -139,10 +139,11 @@ __global__ void cc_query_kernel(int64_t n, const uint8_t *__restrict__ type, con
 }
 
 // ---------------------------------------------------------------------------------
-// load: caller-order rows -> level order, with validation and per-scenario sums
+// load: caller-order rows -> internal order and blocked layout, with validation
+// and per-scenario sums
 // ---------------------------------------------------------------------------------
 __global__ void permute_rows_kernel(const int64_t *__restrict__ raw, const int32_t *__restrict__ int2ext,
-                                    const uint8_t *__restrict__ local, int64_t V, int32_t S,
+                                    const uint8_t *__restrict__ local, int64_t V, int32_t S, MatLayout lay,
                                     int64_t *__restrict__ dur, double *__restrict__ sums, int32_t *status) {
   int32_t s = blockIdx.x * blockDim.x + threadIdx.x;
   if (s >= S) return;
@@ -156,23 +157,30 @@ __global__ void permute_rows_kernel(const int64_t *__restrict__ raw, const int32
       neg |= d < 0;
       acc += (double)d;
     }
-    dur[i * S + s] = d;
+    dur[lay.at(i, s)] = d;
   }
   if (neg) set_status(status, kDevNegativeDuration);
   atomicAdd(&sums[s], acc);
 }
 
 // ---------------------------------------------------------------------------------
-// B2: compose pass.  One thread block owns SIGMA scenarios and walks every level
-// of the level-ordered graph; scenarios never interact, so only block barriers
-// are needed.  f(v) = max(0, finish of the op issued before v on each of its
-// timelines, finish of each data predecessor) + d(v).  The first term comes from
-// a per-(timeline, scenario) frontier that holds the finish of the last op placed
-// on that timeline (Sec. 4.2); the per-scenario makespan is fused in.
+// B2: compose pass.  One thread block owns a block of SIGMA scenarios and walks
+// the graph segment level by segment level; scenarios never interact, so only
+// block-level synchronization is needed.  A segment is a serial chain of ops
+// (each op's only input is the previous one, which feeds nothing else), so along
+// it every op starts when the previous ends: finish = running sum.  The head of a
+// segment starts at max(0, finish of the op issued before it on each of its
+// timelines, finish of each data predecessor) (Sec. 4.2, 5.2); the first term
+// comes from a per-(timeline, scenario) frontier holding the finish of the last
+// op placed on that timeline, which the segment's tail advances.  The
+// per-scenario makespan is fused in.
+//
+// compose_direct_kernel reads the graph and the durations from global memory and
+// fits any graph; the staged and pipelined kernels are the fast paths.
 // ---------------------------------------------------------------------------------
 template <int SIGMA, bool SMEM_FRONTIER>
 __global__ void __launch_bounds__(kComposeThreads)
-compose_kernel(ComposeArgs a) {
+compose_direct_kernel(ComposeArgs a) {
   extern __shared__ __align__(16) int64_t smem[];
   const int32_t S = a.S;
   const int32_t s0 = blockIdx.x * SIGMA;
@@ -192,22 +200,18 @@ compose_kernel(ComposeArgs a) {
   int64_t *f = a.f;
   int64_t mk = 0;
   for (int32_t l = 0; l < a.L; ++l) {
-    const int64_t i0 = a.lvl_off[l], i1 = a.lvl_off[l + 1];
+    const int64_t t0 = a.seg_lvl_off[l], t1 = a.seg_lvl_off[l + 1];
     if (active) {
-      for (int64_t i = i0 + sub; i < i1; i += stride) {
-        int64_t m = 0;
-        const int64_t q0 = a.nq_off[i], q1 = a.nq_off[i + 1];
-        for (int64_t k = q0; k < q1; ++k) m = max(m, fr[(int64_t)a.nq[k] * SIGMA + j]);
-        for (int64_t k = a.dp_off[i]; k < a.dp_off[i + 1]; ++k)
-          m = max(m, f[(int64_t)a.dp[k] * S + s]);
-        int64_t d = dur[i * S + s];
-        if (a.ov) {
-          const uint8_t c = a.kcl[i];
-          if (c != kNotSlowable && a.ov[i * S + s]) d = slowed(d, a.sf[(int64_t)c * S + s]);
+      for (int64_t t = t0 + sub; t < t1; t += stride) {
+        const int64_t h = a.seg_node_off[t], z = a.seg_node_off[t + 1] - 1;
+        int64_t fv = 0;  // the head starts after its timelines and data predecessors
+        for (int64_t k = a.nq_off[h]; k < a.nq_off[h + 1]; ++k) fv = max(fv, fr[(int64_t)a.nq[k] * SIGMA + j]);
+        for (int64_t k = a.dp_off[h]; k < a.dp_off[h + 1]; ++k) fv = max(fv, f[a.lay.at(a.dp[k], s)]);
+        for (int64_t i = h; i <= z; ++i) {  // along the chain every op starts when the previous ends
+          fv += dur[a.lay.at(i, s)];
+          f[a.lay.at(i, s)] = fv;
         }
-        const int64_t fv = m + d;
-        f[i * S + s] = fv;
-        for (int64_t k = q0; k < q1; ++k) fr[(int64_t)a.nq[k] * SIGMA + j] = fv;
+        for (int64_t k = a.nq_off[z]; k < a.nq_off[z + 1]; ++k) fr[(int64_t)a.nq[k] * SIGMA + j] = fv;
         mk = max(mk, fv);
       }
     }
@@ -219,44 +223,474 @@ compose_kernel(ComposeArgs a) {
     a.makespan[s0 + threadIdx.x] = mk_s[threadIdx.x];
 }
 
+// -- asynchronous global->shared copies (cp.async; completion by wait_group) ----------
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+  unsigned d = (unsigned)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async8(void *dst, const void *src) {
+  unsigned d = (unsigned)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(d), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_dyn(int n) {
+  switch (n) {
+    case 0: cp_async_wait<0>(); break;
+    case 1: cp_async_wait<1>(); break;
+    case 2: cp_async_wait<2>(); break;
+    case 3: cp_async_wait<3>(); break;
+    case 4: cp_async_wait<4>(); break;
+    case 5: cp_async_wait<5>(); break;
+    case 6: cp_async_wait<6>(); break;
+    case 7: cp_async_wait<7>(); break;
+    case 8: cp_async_wait<8>(); break;
+    case 9: cp_async_wait<9>(); break;
+    case 10: cp_async_wait<10>(); break;
+    case 11: cp_async_wait<11>(); break;
+    case 12: cp_async_wait<12>(); break;
+    case 13: cp_async_wait<13>(); break;
+    default: cp_async_wait<14>(); break;
+  }
+}
+
+// A thread moves LANES consecutive int64 values of a row (a 16-byte vector when
+// LANES == 2; rows are 16-byte aligned whenever SIGMA is even).  The s_* forms
+// address shared memory explicitly (32-bit shared addresses).
+__device__ __forceinline__ uint32_t saddr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+template <int LANES>
+__device__ __forceinline__ void s_load(uint32_t a, int64_t (&v)[LANES]) {
+  if constexpr (LANES == 2)
+    asm volatile("ld.shared.v2.s64 {%0, %1}, [%2];\n" : "=l"(v[0]), "=l"(v[1]) : "r"(a));
+  else
+    asm volatile("ld.shared.s64 %0, [%1];\n" : "=l"(v[0]) : "r"(a));
+}
+template <int LANES>
+__device__ __forceinline__ void s_store(uint32_t a, const int64_t (&v)[LANES]) {
+  if constexpr (LANES == 2)
+    asm volatile("st.shared.v2.s64 [%0], {%1, %2};\n" ::"r"(a), "l"(v[0]), "l"(v[1]) : "memory");
+  else
+    asm volatile("st.shared.s64 [%0], %1;\n" ::"r"(a), "l"(v[0]) : "memory");
+}
+template <int LANES>
+__device__ __forceinline__ void s_max(int64_t (&m)[LANES], uint32_t a) {
+  int64_t v[LANES];
+  s_load<LANES>(a, v);
+#pragma unroll
+  for (int k = 0; k < LANES; ++k) m[k] = max(m[k], v[k]);
+}
+__device__ __forceinline__ uint32_t s_ld32(uint32_t a) {
+  uint32_t v;
+  asm volatile("ld.shared.u32 %0, [%1];\n" : "=r"(v) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ uint4 s_ld128(uint32_t a) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];\n" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+  return v;
+}
+template <int LANES>
+__device__ __forceinline__ void g_max(int64_t (&m)[LANES], const int64_t *p) {
+  if constexpr (LANES == 2) {
+    const longlong2 t = *reinterpret_cast<const longlong2 *>(p);
+    m[0] = max(m[0], (int64_t)t.x);
+    m[1] = max(m[1], (int64_t)t.y);
+  } else {
+    m[0] = max(m[0], *p);
+  }
+}
+template <int LANES>
+__device__ __forceinline__ void g_store(int64_t *p, const int64_t (&v)[LANES]) {
+  if constexpr (LANES == 2)
+    *reinterpret_cast<longlong2 *>(p) = make_longlong2(v[0], v[1]);
+  else
+    *p = v[0];
+}
+
+// Compose the segments of one segment level (shared by the staged and the
+// pipelined kernels).  Segment k's header and entries are in the record ring at
+// word `ro`; its rows are i0 + header.z ... in the duration ring.  Thread `sub`
+// handles segments sub, sub + step, ... for scenario lanes j0 .. j0+LANES-1.  This
+// block's finish rows are a contiguous [V][SIGMA] array (padding lanes included),
+// so every row moves as whole vectors.
+template <int SIGMA, int LANES>
+__device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t ro, uint32_t i0, uint32_t seg0,
+                                                 int32_t nseg, int sub, int step, int j0, int64_t *fr, int64_t *vr,
+                                                 const int64_t *dr, const uint32_t *rr, uint32_t vmask,
+                                                 uint32_t dmask, uint32_t rmask, int64_t (&mk)[LANES]) {
+  int64_t *fb = a.f + ((int64_t)blockIdx.x * a.n_rows) * SIGMA;
+  const uint32_t fr_a = saddr(fr) + j0 * 8, vr_a = saddr(vr) + j0 * 8, dr_a = saddr(dr) + j0 * 8;
+  const uint32_t rr_a = saddr(rr);
+  constexpr uint32_t kRowBytes = SIGMA * 8;
+  for (int32_t k = sub; k < nseg; k += step) {
+    const uint4 hd = s_ld128(rr_a + ((ro + 4 * k) & rmask) * 4);
+    const uint32_t nqf = hd.y & 0xFFFFu, ndp = hd.y >> 16;
+    const uint32_t len = hd.w & 0xFFFFu, nql = hd.w >> 16;
+    const uint32_t e = ro + hd.x;
+    const uint32_t first = i0 + hd.z;
+    int64_t fv[LANES];
+#pragma unroll
+    for (int j = 0; j < LANES; ++j) fv[j] = 0;
+    for (uint32_t q = 0; q < nqf; ++q) s_max<LANES>(fv, fr_a + s_ld32(rr_a + ((e + q) & rmask) * 4) * kRowBytes);
+    for (uint32_t q = 0; q < ndp; ++q) {
+      const uint32_t ref = s_ld32(rr_a + ((e + nqf + q) & rmask) * 4);
+      if (ref & kFarRef)
+        g_max<LANES>(fv, fb + (int64_t)(ref & ~kFarRef) * SIGMA + j0);
+      else
+        s_max<LANES>(fv, vr_a + (ref & vmask) * kRowBytes);
+    }
+    int64_t *gp = fb + (int64_t)first * SIGMA + j0;
+#pragma unroll 4
+    for (uint32_t t = 0; t < len; ++t, gp += SIGMA) {  // along the chain every op starts when the previous ends
+      int64_t d[LANES];
+      s_load<LANES>(dr_a + ((first + t) & dmask) * kRowBytes, d);
+#pragma unroll
+      for (int j = 0; j < LANES; ++j) fv[j] += d[j];
+      g_store<LANES>(gp, fv);
+    }
+#pragma unroll
+    for (int j = 0; j < LANES; ++j) mk[j] = max(mk[j], fv[j]);
+    s_store<LANES>(vr_a + ((seg0 + k) & vmask) * kRowBytes, fv);
+    for (uint32_t q = 0; q < nql; ++q)
+      s_store<LANES>(fr_a + s_ld32(rr_a + ((e + nqf + ndp + q) & rmask) * 4) * kRowBytes, fv);
+  }
+}
+
+// Staged compose (all threads copy and compose).  Shared memory holds the
+// per-scenario makespans, the extents of the last 16 copy groups, two metadata
+// buffers (kMetaChunk segment levels each), the frontier, a value ring with the
+// finish times of the tails of the most recent 2^vlog2 segments (read by near
+// predecessors), a ring of duration rows and a ring of record words.  Before
+// composing segment level l, every thread copies into the rings all rows and
+// record words that fit without touching level l-1 (which slower threads may still
+// read); it then waits only for the copy groups that hold level l.  Predecessors
+// too old for the value ring are read from global memory, where this block wrote
+// them at an earlier level.  SIGMA/LANES threads share a segment.
+template <int SIGMA, int THREADS>
+__global__ void __launch_bounds__(THREADS)
+compose_staged_kernel(StagedArgs a) {
+  constexpr int LANES = (SIGMA % 2 == 0) ? 2 : 1;
+  constexpr int TPN = SIGMA / LANES;  // threads per segment
+  extern __shared__ __align__(16) unsigned char sbuf[];
+  const int32_t S = a.S;
+  const int32_t s0 = blockIdx.x * SIGMA;
+  const int tid = threadIdx.x;
+  const StagedLayout lay = staged_layout(a.n_queues, SIGMA, a.vlog2, a.dlog2, a.rlog2);
+  const uint32_t vmask = (1u << a.vlog2) - 1, dmask = (1u << a.dlog2) - 1, rmask = (1u << a.rlog2) - 1;
+  const uint32_t RR = dmask + 1, RB = rmask + 1;
+  int64_t *mk_s = reinterpret_cast<int64_t *>(sbuf);                  // [SIGMA]
+  uint2 *hist = reinterpret_cast<uint2 *>(sbuf + lay.hist);           // [16] (rows, words) copied by group
+  uint32_t *meta_s = reinterpret_cast<uint32_t *>(sbuf + lay.meta);   // [2][kMetaCap][4]
+  int64_t *fr = reinterpret_cast<int64_t *>(sbuf + lay.fr);           // [n_queues][SIGMA]
+  int64_t *vr = reinterpret_cast<int64_t *>(sbuf + lay.vr);           // [value ring][SIGMA]
+  int64_t *dr = reinterpret_cast<int64_t *>(sbuf + lay.dr);           // [duration ring][SIGMA]
+  uint32_t *rr = reinterpret_cast<uint32_t *>(sbuf + lay.rr);         // [record ring]
+
+  for (int k = tid; k < a.n_queues * SIGMA; k += blockDim.x) fr[k] = 0;
+  if (tid < SIGMA) mk_s[tid] = 0;
+  auto load_meta = [&](int32_t chunk) {  // segment levels [chunk*kMetaChunk, +kMetaChunk] (inclusive)
+    uint32_t *dst = meta_s + (chunk & 1) * kMetaCap * 4;
+    const int32_t base = chunk * kMetaChunk;
+    for (int k = tid; k <= kMetaChunk; k += blockDim.x)
+      if (base + k <= a.L) cp_async16(&dst[4 * k], &a.meta[4 * (base + k)]);
+  };
+  // this block's rows are contiguous: element e of the block lands in ring element
+  // e mod (RR*SIGMA), and a 16-byte piece never straddles the ring's end
+  const int64_t *durb = a.dur + ((int64_t)blockIdx.x * a.n_rows) * SIGMA;
+  const uint32_t emask = RR * SIGMA - 1;
+  uint32_t rows_done = 0, words_done = 0;
+  auto issue_to = [&](uint32_t row_lim, uint32_t word_lim) {  // copy rows and words up to the limits
+    if constexpr (SIGMA % 2 == 0) {
+      const uint32_t e0 = rows_done * SIGMA, n16 = (row_lim - rows_done) * (SIGMA / 2);
+      for (uint32_t t = tid; t < n16; t += blockDim.x) {
+        const uint32_t e = e0 + 2 * t;
+        cp_async16(dr + (e & emask), durb + e);
+      }
+    } else {
+      for (uint32_t e = rows_done + tid; e < row_lim; e += blockDim.x) cp_async8(dr + (e & emask), durb + e);
+    }
+    for (uint32_t t = words_done + tid * 4; t < word_lim; t += blockDim.x * 4)
+      cp_async16(&rr[t & rmask], &a.recs[t]);
+    rows_done = row_lim;
+    words_done = word_lim;
+  };
+  // group 0: the first metadata chunk and as many rows and words as the rings hold
+  load_meta(0);
+  issue_to(min(RR, a.n_rows), min(RB, a.n_words));
+  cp_async_commit();
+  int32_t g = 0;  // index of the last committed copy group
+  if (tid == 0) hist[0] = make_uint2(rows_done, words_done);
+  cp_async_wait<0>();
+  __syncthreads();  // metadata and hist[0] visible to every thread
+
+  const int j0 = (tid % TPN) * LANES;  // first scenario lane of this thread
+  const int sub = tid / TPN;
+  constexpr int kSegsPerStep = THREADS / TPN;
+  int64_t mk[LANES];
+#pragma unroll
+  for (int k = 0; k < LANES; ++k) mk[k] = 0;
+  uint32_t prev_i0 = 0, prev_ro = 0;  // level l-1 (still readable by slower threads)
+  for (int32_t l = 0; l < a.L; ++l) {
+    const int32_t kc = l / kMetaChunk;
+    const int32_t cbase = kc * kMetaChunk;
+    const bool new_chunk = l > 0 && l == cbase;
+    if (new_chunk) load_meta(kc);  // its buffer was last used by chunk kc-2
+    issue_to(min(prev_i0 + RR, a.n_rows), min(prev_ro + RB, a.n_words));
+    cp_async_commit();
+    ++g;
+    if (tid == 0) hist[g & 15] = make_uint2(rows_done, words_done);
+    const uint32_t *mb = meta_s + (kc & 1) * kMetaCap * 4 + 4 * (l - cbase);
+    if (new_chunk) {
+      cp_async_wait<0>();
+    } else {
+      // the oldest copy group that completes level l (look back at most 14 groups;
+      // the slot of group g-16 is the one being rewritten now)
+      const uint32_t need_rows = mb[4 + 1], need_words = mb[4];
+      int32_t x = g;
+      while (x > 0 && g - x < 14) {
+        const uint2 ext = hist[(x - 1) & 15];
+        if (ext.x >= need_rows && ext.y >= need_words)
+          --x;
+        else
+          break;
+      }
+      cp_async_wait_dyn(g - x);
+    }
+    __syncthreads();
+
+    const uint32_t ro = mb[0], i0 = mb[1], seg0 = mb[2];
+    const int32_t nseg = (int32_t)(mb[4 + 2] - seg0);
+    compose_segments<SIGMA, LANES>(a, ro, i0, seg0, nseg, sub, kSegsPerStep, j0, fr, vr, dr, rr, vmask, dmask,
+                                   rmask, mk);
+    prev_i0 = i0;
+    prev_ro = ro;
+  }
+  cp_async_wait<0>();
+#pragma unroll
+  for (int j = 0; j < LANES; ++j) atomicMax((unsigned long long *)&mk_s[j0 + j], (unsigned long long)mk[j]);
+  __syncthreads();
+  if (tid < SIGMA && s0 + tid < S && a.makespan) a.makespan[s0 + tid] = mk_s[tid];
+}
+
+// -- mbarriers and 1-D bulk copies (TMA engine) ----------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+// wait for the phase of `parity` to complete; false once `limit` clock cycles pass
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, long long limit) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity))
+    if (clock64() - t0 > limit) return false;
+  return true;
+}
+// addresses 16-byte aligned, size a multiple of 16; completes `bytes` on the mbarrier
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n"
+               ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
+}
+// barrier over `threads` threads that also returns whether any of them passed `flag`
+__device__ __forceinline__ bool named_barrier_or(int id, int threads, bool flag) {
+  uint32_t any;
+  asm volatile(
+      "{\n .reg .pred pin, pout;\n setp.ne.u32 pin, %1, 0;\n bar.red.or.pred pout, %2, %3, pin;\n"
+      " selp.u32 %0, 1, 0, pout;\n}\n"
+      : "=r"(any) : "r"((uint32_t)flag), "r"(id), "r"(threads) : "memory");
+  return any != 0;
+}
+
+// Pipelined compose (even SIGMA): the last warp is a producer that copies each
+// segment level's duration rows, record block and metadata into the rings with the
+// TMA engine (at most five 1-D bulk copies per level: this block's rows of a level
+// are contiguous), as far ahead as the rings allow; kPipeConsumerWarps warps
+// compose.  Stage l % kPipeStages has a "full" mbarrier (armed with the level's
+// byte count) and an "empty" mbarrier (one arrival per consumer warp once the
+// level is composed).  Every wait is bounded: on expiry the block records
+// kDevTimeout, stops, and lets its copies in flight land first.
+template <int SIGMA>
+__global__ void __launch_bounds__((kPipeConsumerWarps + 1) * 32)
+compose_pipelined_kernel(StagedArgs a) {
+  constexpr int LANES = 2;
+  constexpr int TPN = SIGMA / LANES;  // threads per segment
+  constexpr int NB = kPipeStages;
+  constexpr int NCT = kPipeConsumerWarps * 32;
+  extern __shared__ __align__(16) unsigned char sbuf[];
+  const int32_t S = a.S;
+  const int32_t s0 = blockIdx.x * SIGMA;
+  const int tid = threadIdx.x;
+  const StagedLayout lay = staged_layout(a.n_queues, SIGMA, a.vlog2, a.dlog2, a.rlog2);
+  const uint32_t vmask = (1u << a.vlog2) - 1, dmask = (1u << a.dlog2) - 1, rmask = (1u << a.rlog2) - 1;
+  const uint32_t RR = dmask + 1, RB = rmask + 1;
+  int64_t *mk_s = reinterpret_cast<int64_t *>(sbuf);                       // [SIGMA]
+  uint64_t *full = reinterpret_cast<uint64_t *>(sbuf + lay.meta);          // [NB]
+  uint64_t *empty = full + NB;                                              // [NB]
+  uint32_t *hist = reinterpret_cast<uint32_t *>(sbuf + lay.meta + 256);    // [NB][2] producer only
+  uint32_t *metas = reinterpret_cast<uint32_t *>(sbuf + lay.meta + 384);   // [NB][8]
+  int64_t *fr = reinterpret_cast<int64_t *>(sbuf + lay.fr);
+  int64_t *vr = reinterpret_cast<int64_t *>(sbuf + lay.vr);
+  int64_t *dr = reinterpret_cast<int64_t *>(sbuf + lay.dr);
+  uint32_t *rr = reinterpret_cast<uint32_t *>(sbuf + lay.rr);
+
+  for (int k = tid; k < a.n_queues * SIGMA; k += blockDim.x) fr[k] = 0;
+  if (tid < SIGMA) mk_s[tid] = 0;
+  if (tid == 0) {
+    for (int b = 0; b < NB; ++b) {
+      mbar_init(&full[b], 1);  // the producer's arrive.expect_tx
+      mbar_init(&empty[b], kPipeConsumerWarps);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+  }
+  asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+  __syncthreads();
+
+  if (tid >= NCT) {
+    // ---------------- producer warp (one lane issues) ----------------
+    const int lane = tid - NCT;
+    if (lane == 0) {
+      const int64_t *durb = a.dur + ((int64_t)blockIdx.x * a.n_rows) * SIGMA;
+      const uint32_t emask = RR * SIGMA - 1;
+      int32_t c_known = 0;  // every level < c_known has been composed
+      int32_t issued = 0;   // levels [0, issued) have been armed
+      bool fail = false;
+      for (int32_t l = 0; l < a.L; ++l) {
+        if (l == a.skip_level) break;  // failure injection: level l never arrives
+        const uint4 m0 = *reinterpret_cast<const uint4 *>(a.meta + 4 * l);
+        const uint4 m1 = *reinterpret_cast<const uint4 *>(a.meta + 4 * (l + 1));
+        const uint32_t ro = m0.x, i0 = m0.y, ro1 = m1.x, i1 = m1.y;
+        // ring space: level l overwrites rows and words of levels below c_known only
+        while (c_known < l && (l - c_known >= NB || i1 > hist[2 * (c_known % NB)] + RR ||
+                               ro1 > hist[2 * (c_known % NB) + 1] + RB)) {
+          if (!mbar_wait(&empty[c_known % NB], (c_known / NB) & 1, a.wait_limit_cycles)) {
+            fail = true;
+            break;
+          }
+          ++c_known;
+        }
+        if (fail) break;
+        hist[2 * (l % NB)] = i0;
+        hist[2 * (l % NB) + 1] = ro;
+        uint64_t *bar = &full[l % NB];
+        const uint32_t e0 = i0 * SIGMA, ne = (i1 - i0) * SIGMA, w0 = ro & rmask, nw = ro1 - ro;
+        mbar_arrive_expect_tx(bar, ne * 8 + nw * 4 + 32);
+        const uint32_t ne1 = min(ne, emask + 1 - (e0 & emask));
+        bulk_g2s(dr + (e0 & emask), durb + e0, ne1 * 8, bar);
+        if (ne1 < ne) bulk_g2s(dr, durb + e0 + ne1, (ne - ne1) * 8, bar);
+        const uint32_t nw1 = min(nw, RB - w0);
+        bulk_g2s(rr + w0, a.recs + ro, nw1 * 4, bar);
+        if (nw1 < nw) bulk_g2s(rr, a.recs + ro + nw1, (nw - nw1) * 4, bar);
+        bulk_g2s(metas + 8 * (l % NB), a.meta + 4 * l, 32, bar);
+        issued = l + 1;
+      }
+      if (fail) atomicCAS(a.status, 0, kDevTimeout);
+      // let every copy this block started land before it exits
+      for (int32_t x = max(c_known, issued - NB); x < issued; ++x)
+        if (!mbar_wait(&full[x % NB], (x / NB) & 1, a.wait_limit_cycles)) atomicCAS(a.status, 0, kDevTimeout);
+    }
+    __syncwarp();
+  } else {
+    // ---------------- consumer warps ----------------
+    const int j0 = (tid % TPN) * LANES;
+    const int sub = tid / TPN;
+    constexpr int kSegsPerStep = NCT / TPN;
+    int64_t mk[LANES] = {0, 0};
+    for (int32_t l = 0; l < a.L; ++l) {
+      const bool ok = mbar_wait(&full[l % NB], (l / NB) & 1, a.wait_limit_cycles);
+      if (ok) {
+        const uint32_t *mb = metas + 8 * (l % NB);
+        const uint32_t ro = mb[0], i0 = mb[1], seg0 = mb[2];
+        const int32_t nseg = (int32_t)(mb[4 + 2] - seg0);
+        compose_segments<SIGMA, LANES>(a, ro, i0, seg0, nseg, sub, kSegsPerStep, j0, fr, vr, dr, rr, vmask, dmask,
+                                       rmask, mk);
+      }
+      // every consumer learns, in the same barrier, whether any of them gave up
+      if (named_barrier_or(1, NCT, !ok)) {
+        if (tid == 0) atomicCAS(a.status, 0, kDevTimeout);
+        break;
+      }
+      if ((tid & 31) == 0) mbar_arrive(&empty[l % NB]);
+    }
+#pragma unroll
+    for (int j = 0; j < LANES; ++j) atomicMax((unsigned long long *)&mk_s[j0 + j], (unsigned long long)mk[j]);
+  }
+  __syncthreads();
+  if (tid < SIGMA && s0 + tid < S && a.makespan) a.makespan[s0 + tid] = mk_s[tid];
+}
+
 // ---------------------------------------------------------------------------------
-// B3: validator overlap test.  One thread per (rank, scenario) walks the rank's
-// compute timeline in time order with one monotone cursor per comm/memcpy
-// timeline: ops on a timeline run one after the other, so their intervals are
-// sorted and the first comm op finishing after a kernel's start is the only
-// place a search has to resume from.
+// B3: validator overlap test.  One thread per (chunk of a rank's compute timeline,
+// scenario).  The rank's timelines run their ops one after the other, so their
+// intervals are sorted: a binary search finds, on each comm/memcpy timeline, the
+// first op finishing after the chunk's first kernel starts, and from there one
+// monotone cursor per timeline suffices.  A compute op that overlaps a comm op with
+// positive length gets rint(d * slowdown) for the next composition, others keep d.
 // ---------------------------------------------------------------------------------
 __global__ void overlap_kernel(OverlapArgs a) {
   const int32_t S = a.S;
+  const MatLayout L = a.lay;
   const int32_t s = blockIdx.x * blockDim.x + threadIdx.x;
-  const int32_t r = blockIdx.y;
-  if (s >= S) return;
+  const int64_t c = blockIdx.y + (int64_t)gridDim.y * blockIdx.z;
+  if (s >= S || c >= a.n_chunks) return;
   const int ns = a.n_streams;
-  const int64_t qbase = (int64_t)r * ns;
+  const int64_t r = a.chunks[2 * c];
+  const int64_t qbase = r * ns;
+  const int64_t c0 = a.chunks[2 * c + 1];
+  const int64_t c1 = min(a.q_off[qbase + 1], c0 + kOverlapChunk);
+  const int64_t *__restrict__ f = a.f;
+  const int64_t *__restrict__ du = a.d_used;
   int64_t cur[kMaxStreams];
-  for (int k = 1; k < ns; ++k) cur[k] = a.q_off[qbase + k];
-  const int64_t c0 = a.q_off[qbase], c1 = a.q_off[qbase + 1];
+  {  // cursors: first op on each timeline that finishes after the chunk's first start
+    const int64_t v = a.q_ops[c0];
+    const int64_t sv = f[L.at(v, s)] - du[L.at(v, s)];
+    for (int k = 1; k < ns; ++k) {
+      int64_t lo = a.q_off[qbase + k], hi = a.q_off[qbase + k + 1];
+      while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if (f[L.at(a.q_ops[mid], s)] > sv)
+          hi = mid;
+        else
+          lo = mid + 1;
+      }
+      cur[k] = lo;
+    }
+  }
   for (int64_t i = c0; i < c1; ++i) {
     const int64_t v = a.q_ops[i];
-    int64_t dv = a.dur[v * S + s];
-    if (a.ov_prev && a.ov_prev[v * S + s]) dv = slowed(dv, a.sf[(int64_t)a.kcl[v] * S + s]);
-    const int64_t fv = a.f[v * S + s];
-    const int64_t sv = fv - dv;
+    const int64_t fv = f[L.at(v, s)];
+    const int64_t sv = fv - du[L.at(v, s)];
+    const int64_t d0 = a.d_orig == du ? fv - sv : a.d_orig[L.at(v, s)];
     uint8_t hit = 0;
     if (sv < fv) {
       for (int k = 1; k < ns && !hit; ++k) {
         const int64_t e = a.q_off[qbase + k + 1];
-        int64_t c = cur[k];
-        while (c < e) {
-          const int64_t w = a.q_ops[c];
-          if (a.is_comm[w] && a.f[w * S + s] > sv) break;
-          ++c;
+        int64_t cc = cur[k];
+        while (cc < e) {
+          const int64_t w = a.q_ops[cc];
+          if (a.is_comm[w] && f[L.at(w, s)] > sv) break;
+          ++cc;
         }
-        cur[k] = c;
-        for (int64_t jj = c; jj < e; ++jj) {
+        cur[k] = cc;
+        for (int64_t jj = cc; jj < e; ++jj) {
           const int64_t w = a.q_ops[jj];
-          const int64_t fw = a.f[w * S + s];
-          const int64_t sw = fw - a.dur[w * S + s];
+          const int64_t fw = f[L.at(w, s)];
+          const int64_t sw = fw - du[L.at(w, s)];
           if (sw >= fv) break;
           if (a.is_comm[w] && sw < fw) {
             hit = 1;
@@ -265,28 +699,36 @@ __global__ void overlap_kernel(OverlapArgs a) {
         }
       }
     }
-    a.ov[v * S + s] = hit;
+    a.ov[L.at(v, s)] = hit;
+    a.d_next[L.at(v, s)] = hit ? slowed(d0, a.sf[(int64_t)a.kcl[v] * S + s]) : d0;
+  }
+}
+
+__global__ void copy_rows_kernel(const int32_t *__restrict__ rows, int64_t n_rows, int32_t S, MatLayout lay,
+                                 const int64_t *__restrict__ src, int64_t *__restrict__ dst) {
+  int64_t total = n_rows * S;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    int64_t k = idx / S;
+    int64_t at = lay.at(rows[k], (int32_t)(idx - k * S));
+    dst[at] = src[at];
   }
 }
 
 // ---------------------------------------------------------------------------------
-// readback: internal order -> caller order
+// readback: internal order and blocked layout -> caller order, [op][scenario]
 // ---------------------------------------------------------------------------------
 __global__ void readback_kernel(const int32_t *__restrict__ ext2int, int64_t op0, int64_t op1, int32_t S,
-                                const int64_t *__restrict__ f, const int64_t *__restrict__ dur,
-                                const uint8_t *__restrict__ ov, const uint8_t *__restrict__ kcl,
-                                const double *__restrict__ sf, int64_t *__restrict__ start,
-                                int64_t *__restrict__ finish) {
+                                MatLayout lay, const int64_t *__restrict__ f, const int64_t *__restrict__ d,
+                                int64_t *__restrict__ start, int64_t *__restrict__ finish) {
   int64_t total = (op1 - op0) * S;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
        idx += (int64_t)gridDim.x * blockDim.x) {
     int64_t o = idx / S;
     int32_t s = (int32_t)(idx - o * S);
-    int64_t i = ext2int[op0 + o];
-    int64_t fv = f[i * S + s];
-    int64_t d = dur[i * S + s];
-    if (ov && kcl[i] != kNotSlowable && ov[i * S + s]) d = slowed(d, sf[(int64_t)kcl[i] * S + s]);
-    if (start) start[idx] = fv - d;
+    int64_t at = lay.at(ext2int[op0 + o], s);
+    int64_t fv = f[at];
+    if (start) start[idx] = fv - d[at];
     if (finish) finish[idx] = fv;
   }
 }
@@ -305,7 +747,7 @@ __global__ void read_cc_kernel(const int32_t *__restrict__ ext2int, int64_t op0,
 }
 
 __global__ void read_ov_kernel(const int32_t *__restrict__ ext2int, int64_t op0, int64_t op1, int32_t S,
-                               const uint8_t *__restrict__ ov, const uint8_t *__restrict__ kcl,
+                               MatLayout lay, const uint8_t *__restrict__ ov, const uint8_t *__restrict__ kcl,
                                uint8_t *__restrict__ out) {
   int64_t total = (op1 - op0) * S;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
@@ -313,7 +755,7 @@ __global__ void read_ov_kernel(const int32_t *__restrict__ ext2int, int64_t op0,
     int64_t o = idx / S;
     int32_t s = (int32_t)(idx - o * S);
     int64_t i = ext2int[op0 + o];
-    out[idx] = (ov && kcl[i] != kNotSlowable) ? ov[i * S + s] : 0;  // only compute ops are tested
+    out[idx] = (ov && kcl[i] != kNotSlowable) ? ov[lay.at(i, s)] : 0;  // only compute ops are tested
   }
 }
 
@@ -330,14 +772,34 @@ cudaError_t launch_compose_t(const ComposeArgs &a, cudaStream_t st) {
   size_t smem = compose_smem_bytes(a.n_queues, SIGMA, &in_smem);
   dim3 grid((a.S + SIGMA - 1) / SIGMA);
   if (in_smem) {
-    auto k = compose_kernel<SIGMA, true>;
+    auto k = compose_direct_kernel<SIGMA, true>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     k<<<grid, kComposeThreads, smem, st>>>(a);
   } else {
-    auto k = compose_kernel<SIGMA, false>;
+    auto k = compose_direct_kernel<SIGMA, false>;
     k<<<grid, kComposeThreads, smem, st>>>(a);
   }
+  return cudaGetLastError();
+}
+
+template <int SIGMA, int THREADS>
+cudaError_t launch_staged_t(const StagedArgs &a, const StagedPlan &plan, cudaStream_t st) {
+  auto k = compose_staged_kernel<SIGMA, THREADS>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid((a.S + SIGMA - 1) / SIGMA);
+  k<<<grid, THREADS, plan.smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+template <int SIGMA>
+cudaError_t launch_pipelined_t(const StagedArgs &a, const StagedPlan &plan, cudaStream_t st) {
+  auto k = compose_pipelined_kernel<SIGMA>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid((a.S + SIGMA - 1) / SIGMA);
+  k<<<grid, (kPipeConsumerWarps + 1) * 32, plan.smem, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -364,9 +826,9 @@ cudaError_t launch_cc_estimate(const CcSig *sig, int32_t G, ScenParams p, int32_
 }
 
 cudaError_t launch_cc_scatter(const int32_t *comm_node, const int32_t *comm_sig, int64_t n_comm,
-                              const int64_t *cc_dur, int32_t S, int64_t *dur, cudaStream_t st) {
+                              const int64_t *cc_dur, int32_t S, MatLayout lay, int64_t *dur, cudaStream_t st) {
   if (n_comm == 0) return cudaSuccess;
-  cc_scatter_kernel<<<grid_for(n_comm * S, 256), 256, 0, st>>>(comm_node, comm_sig, n_comm, cc_dur, S, dur);
+  cc_scatter_kernel<<<grid_for(n_comm * S, 256), 256, 0, st>>>(comm_node, comm_sig, n_comm, cc_dur, S, lay, dur);
   return cudaGetLastError();
 }
 
@@ -379,13 +841,14 @@ cudaError_t launch_cc_query(int64_t n, const uint8_t *type, const uint8_t *algo,
 }
 
 cudaError_t launch_permute_rows(const int64_t *raw, const int32_t *int2ext, const uint8_t *local, int64_t V,
-                                int32_t S, int64_t *dur, double *sums, int32_t *status, cudaStream_t st) {
+                                int32_t S, MatLayout lay, int64_t *dur, double *sums, int32_t *status,
+                                cudaStream_t st) {
   if (V == 0 || S == 0) return cudaSuccess;
   int tx = S >= 128 ? 128 : ((S + 31) / 32) * 32;
   dim3 block(tx);
   int64_t gy = V < 8192 ? V : 8192;
   dim3 grid((S + tx - 1) / tx, (unsigned)gy);
-  permute_rows_kernel<<<grid, block, 0, st>>>(raw, int2ext, local, V, S, dur, sums, status);
+  permute_rows_kernel<<<grid, block, 0, st>>>(raw, int2ext, local, V, S, lay, dur, sums, status);
   return cudaGetLastError();
 }
 
@@ -401,20 +864,55 @@ cudaError_t launch_compose(const ComposeArgs &a, int sigma, cudaStream_t st) {
   }
 }
 
+cudaError_t launch_compose_staged(const StagedArgs &a, int sigma, const StagedPlan &plan, cudaStream_t st) {
+  if (a.S == 0) return cudaSuccess;
+  switch (sigma * 10000 + plan.threads) {
+    case 1 * 10000 + 256: return launch_staged_t<1, 256>(a, plan, st);
+    case 1 * 10000 + 512: return launch_staged_t<1, 512>(a, plan, st);
+    case 1 * 10000 + 1024: return launch_staged_t<1, 1024>(a, plan, st);
+    case 2 * 10000 + 256: return launch_staged_t<2, 256>(a, plan, st);
+    case 2 * 10000 + 512: return launch_staged_t<2, 512>(a, plan, st);
+    case 4 * 10000 + 256: return launch_staged_t<4, 256>(a, plan, st);
+    case 4 * 10000 + 512: return launch_staged_t<4, 512>(a, plan, st);
+    case 8 * 10000 + 512: return launch_staged_t<8, 512>(a, plan, st);
+    case 16 * 10000 + 1024: return launch_staged_t<16, 1024>(a, plan, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_compose_pipelined(const StagedArgs &a, int sigma, const StagedPlan &plan, cudaStream_t st) {
+  if (a.S == 0) return cudaSuccess;
+  switch (sigma) {
+    case 2: return launch_pipelined_t<2>(a, plan, st);
+    case 4: return launch_pipelined_t<4>(a, plan, st);
+    case 8: return launch_pipelined_t<8>(a, plan, st);
+    case 16: return launch_pipelined_t<16>(a, plan, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
-  if (a.S == 0 || a.n_ranks == 0) return cudaSuccess;
+  if (a.S == 0 || a.n_chunks == 0) return cudaSuccess;
   int tx = a.S >= 128 ? 128 : ((a.S + 31) / 32) * 32;
-  dim3 grid((a.S + tx - 1) / tx, a.n_ranks);
+  int64_t gy = a.n_chunks < 65535 ? a.n_chunks : 65535;
+  int64_t gz = (a.n_chunks + gy - 1) / gy;
+  dim3 grid((a.S + tx - 1) / tx, (unsigned)gy, (unsigned)gz);
   overlap_kernel<<<grid, tx, 0, st>>>(a);
   return cudaGetLastError();
 }
 
-cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, const int64_t *f,
-                            const int64_t *dur, const uint8_t *ov, const uint8_t *kcl, const double *sf,
-                            int64_t *start, int64_t *finish, cudaStream_t st) {
+cudaError_t launch_copy_rows(const int32_t *rows, int64_t n_rows, int32_t S, MatLayout lay, const int64_t *src,
+                             int64_t *dst, cudaStream_t st) {
+  if (n_rows == 0 || S == 0) return cudaSuccess;
+  copy_rows_kernel<<<grid_for(n_rows * S, 256), 256, 0, st>>>(rows, n_rows, S, lay, src, dst);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
+                            const int64_t *f, const int64_t *d, int64_t *start, int64_t *finish, cudaStream_t st) {
   int64_t n = (op1 - op0) * S;
   if (n <= 0) return cudaSuccess;
-  readback_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, f, dur, ov, kcl, sf, start, finish);
+  readback_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, lay, f, d, start, finish);
   return cudaGetLastError();
 }
 
@@ -426,11 +924,11 @@ cudaError_t launch_read_cc(const int32_t *ext2int, int64_t op0, int64_t op1, int
   return cudaGetLastError();
 }
 
-cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, const uint8_t *ov,
-                           const uint8_t *kcl, uint8_t *out, cudaStream_t st) {
+cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
+                           const uint8_t *ov, const uint8_t *kcl, uint8_t *out, cudaStream_t st) {
   int64_t n = (op1 - op0) * S;
   if (n <= 0) return cudaSuccess;
-  read_ov_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, ov, kcl, out);
+  read_ov_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, lay, ov, kcl, out);
   return cudaGetLastError();
 }
 

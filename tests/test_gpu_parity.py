@@ -232,3 +232,56 @@ def test_gpt175b_full_size_sampled_scenarios():
 @pytest.mark.slow
 def test_gpt175b_1024_ranks_full_size_sampled_scenarios():
     _sampled_parity("gpt175b-1024", [0, 63])
+
+
+@pytest.mark.parametrize("sigma", ["1", "2", "4", "8", "16"])
+@pytest.mark.parametrize("kernel", ["direct", "staged", "pipelined"])
+def test_every_compose_variant_bit_exact(sigma, kernel, monkeypatch):
+    # the three compose kernels (global-memory, cp.async-staged, bulk-copy pipelined;
+    # the pipelined one needs an even block width) at every scenario-block width,
+    # with full and partial scenario blocks
+    monkeypatch.setenv("ECHO_SIGMA", sigma)
+    monkeypatch.setenv("ECHO_COMPOSE_KERNEL", kernel)
+    c = W.config("gpt1.3b")
+    g = W.build_gpt_graph(c)
+    for S in (32, 37):
+        sc = W.make_scenarios(g, c, n_scen=S)
+        for refine in (0, 1, 2):
+            got = run_gpu(g, sc, refine)
+            assert_same(got, oracle.compose(g, sc, refine_passes=refine, threads=THREADS), g, refine)
+    rng = np.random.default_rng(int(sigma) * 7 + len(kernel))
+    e = Echo(0)
+    try:
+        for _ in range(15):
+            g = SG.random_graph(rng, int(rng.integers(1, 80)), max_ranks=6, max_streams=4, p_edge=0.05)
+            sc = SG.random_scenarios(rng, g, int(rng.choice([16, 32, 48, 64, 37])), max_dur=30)
+            got = run_gpu(g, sc, 1, ctx=e)
+            assert_same(got, oracle.compose(g, sc, refine_passes=1), g, 1)
+    finally:
+        e.close()
+
+
+def test_bounded_wait_reports_timeout(monkeypatch):
+    # failure detection without a GPU fault: the producer of the pipelined kernel
+    # never fills one segment level, every consumer's bounded wait gives up after
+    # 20 ms, the block records the timeout and exits, and the host reports it
+    c = W.config("gpt1.3b")
+    g = W.build_gpt_graph(c)
+    sc = W.make_scenarios(g, c, n_scen=64)
+    monkeypatch.setenv("ECHO_SIGMA", "2")
+    monkeypatch.setenv("ECHO_COMPOSE_KERNEL", "pipelined")
+    monkeypatch.setenv("ECHO_TEST_SKIP_LEVEL", "5")
+    monkeypatch.setenv("ECHO_TEST_WAIT_LIMIT_MS", "20")
+    with Echo(0) as e:
+        e.load_graph(g)
+        e.load_scenarios(sc)
+        e.estimate_collectives()
+        e.compose(refine_passes=0)
+        with pytest.raises(EchoError) as ei:
+            e.read_makespan()
+        assert ei.value.code == 7  # ECHO_E_TIMEOUT
+    # the device is still usable: a context without the injected fault is exact
+    monkeypatch.delenv("ECHO_TEST_SKIP_LEVEL")
+    monkeypatch.delenv("ECHO_TEST_WAIT_LIMIT_MS")
+    got = run_gpu(g, sc, 1)
+    assert_same(got, oracle.compose(g, sc, refine_passes=1, threads=THREADS), g, 1)
