@@ -10,8 +10,9 @@ every op in every scenario, so one step is 2 * V * S updates), plus the achieved
 HBM bandwidth of the compose kernel against the measured GB300 copy peak.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl echo|reference]
-Under torchrun each rank composes its own 1024 scenarios (weak scaling, no
-collective on the data path); the step time is the max over ranks.
+Under torchrun each rank composes its own slice of 1024 scenarios of one batch of
+1024 * N (weak scaling, no collective on the data path); the step time is the
+max over ranks.
 """
 from __future__ import annotations
 
@@ -128,15 +129,17 @@ def profiled_traffic(launch_units):
     return float(m_bytes.group(1)) * launch_units
 
 
-def build_inputs(rank, n_scen=None, pinned=True):
+def build_inputs(rank, world, n_scen=None, pinned=True):
+    """The graph and this rank's slice of a batch of n_scen * world scenarios."""
     import torch
+    from paper_2412_12487_gb300 import sharding as SH
     from paper_2412_12487_gb300 import workloads as W
     c = W.config(WORKLOAD)
-    c = W.GPTConfig(**{**c.__dict__, "scen_seed": c.scen_seed + 7919 * rank,
-                       "n_scen": n_scen or c.n_scen})
+    c = W.GPTConfig(**{**c.__dict__, "n_scen": n_scen or c.n_scen})
     t0 = time.time()
     g = W.build_gpt_graph(c)
-    sc = W.scenario_params(c)
+    s0, s1 = SH.shard_bounds(c.n_scen * world, world, rank)
+    sc = SH.slice_scenarios(W.scenario_params(c, c.n_scen * world), s0, s1)
     V, S = g.n_ops, sc.n_scen
     dur_t = torch.empty((V, S), dtype=torch.int64, pin_memory=pinned)
     W.durations(g, sc.peak_flop_per_ns, out=dur_t.numpy())
@@ -156,14 +159,17 @@ def run_echo(args):
     import torch
     import torch.distributed as dist
     from paper_2412_12487_gb300 import Echo
+    from paper_2412_12487_gb300 import sharding as SH
 
     rank, world, local = dist_env()
     torch.cuda.set_device(local)
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    c, g, sc, dur_t = build_inputs(rank, args.scenarios)
+    c, g, sc, dur_t = build_inputs(rank, world, args.scenarios)
     V, S = g.n_ops, sc.n_scen
-    stream = torch.cuda.current_stream()
+    # a stream of its own: the events below and every library launch share it
+    stream = torch.cuda.Stream(local)
+    torch.cuda.set_stream(stream)
     e = Echo(local, stream)
     t0 = time.time()
     e.load_graph(g)
@@ -220,10 +226,7 @@ def run_echo(args):
     barrier()
     e2e_ms = ev0.elapsed_time(ev1) / e2e_steps
 
-    t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms, e2e_ms = float(t[0]), float(t[1])
+    ms, e2e_ms = SH.max_over_ranks([ms, e2e_ms], device=torch.device("cuda", local))
     units = 2 * V * S  # two compose passes per step
     value = units * world / (ms / 1e3)
     e2e_value = units * world / (e2e_ms / 1e3)

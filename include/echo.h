@@ -135,7 +135,8 @@ typedef struct {
 } echo_compose_opts;
 
 /* Create a context on `device`, enqueuing on `cuda_stream` (a cudaStream_t; NULL =
- * a new non-blocking stream owned by the context). */
+ * a new non-blocking stream owned by the context; the legacy default stream is
+ * passed as cudaStreamLegacy).  The caller's stream must outlive the context. */
 int echo_create(echo_ctx **out, int device, void *cuda_stream);
 /* Free everything the context owns.  NULL is accepted. */
 int echo_destroy(echo_ctx *ctx);

@@ -23,7 +23,7 @@
  *     whose first-pass interval overlaps a communication op on the same rank is
  *     stretched by its factor and the timeline is composed again.
  *
- * Readings where the paper is silent or garbled (each is listed in the design doc):
+ * Readings where the paper is silent or garbled:
  *   time is int64 ns, sources start at 0; a rank has any number of serial streams
  *   (its compute timeline plus comm/memcpy timelines); overlap means
  *   a positive-length intersection of [start, finish) intervals and slows the

@@ -63,6 +63,9 @@ struct GraphBuild {
   std::vector<int32_t> sig_count, comm_node, comm_sig, node_sig;
   std::vector<int32_t> non_compute;   // internal ids of comm and memcpy ops
   std::vector<int64_t> ov_chunks;     // (rank, first position) of compute-timeline chunks
+  int32_t n_cq = 0;                   // comm timelines per rank in cq_off (max over ranks)
+  std::vector<int64_t> cq_off;        // [R*n_cq+1] comm ops of each (rank, comm timeline)
+  std::vector<int32_t> cq_ops;        // internal ids, in issue order
   std::vector<int64_t> blk_words;     // record block size of each segment level (words, padded)
   int32_t max_kclass = -1;
   bool stageable = true;              // every head/tail has < 2^16 timelines and predecessors
@@ -413,6 +416,32 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
       b.ov_chunks.push_back(p);
     }
   }
+  // the comm ops of each rank's timelines that hold any, in issue order
+  for (int32_t r = 0; r < R; ++r) {
+    int32_t n = 0;
+    for (int32_t k = 1; k < NS; ++k) {
+      const int64_t q = (int64_t)r * NS + k;
+      for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i)
+        if (b.is_comm[b.q_ops_int[i]]) {
+          ++n;
+          break;
+        }
+    }
+    b.n_cq = std::max(b.n_cq, n);
+  }
+  b.cq_off.assign((size_t)R * b.n_cq + 1, 0);
+  for (int32_t r = 0; r < R; ++r) {
+    int32_t j = 0;
+    for (int32_t k = 1; k < NS; ++k) {
+      const int64_t q = (int64_t)r * NS + k;
+      const size_t before = b.cq_ops.size();
+      for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i)
+        if (b.is_comm[b.q_ops_int[i]]) b.cq_ops.push_back(b.q_ops_int[i]);
+      if (b.cq_ops.size() > before) b.cq_off[(size_t)r * b.n_cq + ++j] = (int64_t)b.cq_ops.size();
+    }
+    for (; j < b.n_cq; ++j) b.cq_off[(size_t)r * b.n_cq + j + 1] = (int64_t)b.cq_ops.size();
+  }
+  if (b.cq_ops.empty()) b.cq_ops.push_back(0);
   b.blk_words.assign(Ls, 0);
   for (int64_t l = 0; l < Ls; ++l) {
     int64_t w = 0;
@@ -529,11 +558,12 @@ struct echo_ctx {
   std::vector<void *> graph_allocs, scen_allocs;
   // device graph
   int64_t *seg_lvl_off = nullptr, *seg_node_off = nullptr, *nq_off = nullptr, *dp_off = nullptr, *q_off = nullptr;
-  int64_t *ov_chunks = nullptr;
+  int64_t *ov_chunks = nullptr, *cq_off = nullptr;
+  int32_t *cq_ops = nullptr;
   int32_t *non_compute = nullptr;
   int32_t *nq = nullptr, *dp = nullptr, *q_ops = nullptr, *int2ext = nullptr, *ext2int = nullptr;
   int32_t *node_sig = nullptr, *comm_node = nullptr, *comm_sig = nullptr, *sig_count = nullptr;
-  uint8_t *kcl = nullptr, *is_comm = nullptr, *local = nullptr;
+  uint8_t *kcl = nullptr, *local = nullptr;
   CcSig *sigs = nullptr;
   int32_t *status = nullptr;
   // scenarios
@@ -553,6 +583,7 @@ struct echo_ctx {
   int final_f = 0;
   const int64_t *final_d = nullptr;
   bool have_ov = false;
+  echo::OverlapArgs last_ov{};  // inputs of the last validator pass (to recompute its decisions)
   int kernel_choice = 0;            // 0 automatic, 1 direct, 2 staged, 3 pipelined (tuning and tests)
   long long wait_limit_cycles = 0;  // bound of every device-side wait
   int32_t skip_level = -1;          // failure injection for tests
@@ -822,7 +853,8 @@ int echo_load_graph(echo_ctx *c, const echo_graph_desc *g) {
   const GraphBuild &B = c->gb;
   auto &o = c->graph_allocs;
   if ((rc = upload(c, o, &c->seg_lvl_off, B.seg_lvl_off)) || (rc = upload(c, o, &c->seg_node_off, B.seg_node_off)) ||
-      (rc = upload(c, o, &c->ov_chunks, B.ov_chunks)) || (rc = upload(c, o, &c->non_compute, B.non_compute)) ||
+      (rc = upload(c, o, &c->ov_chunks, B.ov_chunks)) ||
+      (rc = upload(c, o, &c->cq_off, B.cq_off)) || (rc = upload(c, o, &c->cq_ops, B.cq_ops)) || (rc = upload(c, o, &c->non_compute, B.non_compute)) ||
       (rc = upload(c, o, &c->nq_off, B.nq_off)) ||
       (rc = upload(c, o, &c->nq, B.nq)) || (rc = upload(c, o, &c->dp_off, B.dp_off)) ||
       (rc = upload(c, o, &c->dp, B.dp)) || (rc = upload(c, o, &c->q_off, B.q_off)) ||
@@ -830,7 +862,7 @@ int echo_load_graph(echo_ctx *c, const echo_graph_desc *g) {
       (rc = upload(c, o, &c->ext2int, B.ext2int)) || (rc = upload(c, o, &c->node_sig, B.node_sig)) ||
       (rc = upload(c, o, &c->comm_node, B.comm_node)) || (rc = upload(c, o, &c->comm_sig, B.comm_sig)) ||
       (rc = upload(c, o, &c->sig_count, B.sig_count)) || (rc = upload(c, o, &c->kcl, B.kcl)) ||
-      (rc = upload(c, o, &c->is_comm, B.is_comm)) || (rc = upload(c, o, &c->local, B.local)) ||
+      (rc = upload(c, o, &c->local, B.local)) ||
       (rc = upload(c, o, &c->sigs, B.sigs))) {
     free_all(c->graph_allocs);
     return rc;
@@ -1059,14 +1091,16 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     o.chunks = c->ov_chunks;
     o.q_off = c->q_off;
     o.q_ops = c->q_ops;
-    o.is_comm = c->is_comm;
+    o.n_cq = B.n_cq;
+    o.cq_off = c->cq_off;
+    o.cq_ops = c->cq_ops;
     o.kcl = c->kcl;
     o.f = c->f[(p - 1) % 2];
     o.d_used = d_used;
     o.d_orig = c->dur;
     o.sf = c->sf;
     o.d_next = c->deff[(p - 1) % 2];
-    o.ov = c->ov;
+    o.ov = nullptr;  // the decisions are recomputed on demand by echo_read_overlap
     CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");
     CK(timed(c, "copy_rows", [&] {
          return echo::launch_copy_rows(c->non_compute, (int64_t)B.non_compute.size(), c->S, c->lay, c->dur,
@@ -1074,6 +1108,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
        }), "copy_rows launch");
     CK(compose_pass(o.d_next, c->f[p % 2]), "compose launch");
     d_used = o.d_next;
+    c->last_ov = o;
   }
   c->final_f = refine % 2;
   c->final_d = d_used;
@@ -1165,7 +1200,16 @@ int echo_read_overlap(echo_ctx *c, int64_t op0, int64_t op1, uint8_t *out) {
   if ((rc = stage_reserve(c, (size_t)std::min<int64_t>(rows_per, std::max<int64_t>(op1 - op0, 1)) * S * 16)))
     return rc;
   if ((rc = composition_status(c))) return rc;
-  const uint8_t *ov = c->have_ov ? c->ov : nullptr;
+  const uint8_t *ov = nullptr;
+  if (c->have_ov) {
+    // the last pass's inputs (its finish times and durations) are still intact:
+    // run its overlap test again, keeping only the decisions
+    echo::OverlapArgs o = c->last_ov;
+    o.d_next = nullptr;
+    o.ov = c->ov;
+    CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");
+    ov = c->ov;
+  }
   for (int64_t a = op0; a < op1; a += rows_per) {
     int64_t b = std::min(op1, a + rows_per);
     int64_t n = (b - a) * S;

@@ -126,17 +126,18 @@ __host__ __device__ inline StagedLayout staged_layout(int32_t n_queues, int sigm
 struct OverlapArgs {
   MatLayout lay;
   int32_t S, n_streams;
+  int32_t n_cq;            // comm timelines per rank (lists of a rank with fewer are empty)
   int64_t n_chunks;
   const int64_t *chunks;   // [n_chunks][2]: (rank, first compute-timeline position)
-  const int64_t *q_off; const int32_t *q_ops;  // timelines in internal ids
-  const uint8_t *is_comm;  // [V]
+  const int64_t *q_off; const int32_t *q_ops;    // timelines in internal ids (compute: stream 0)
+  const int64_t *cq_off; const int32_t *cq_ops;  // [R*n_cq+1]: comm ops of each (rank, comm timeline)
   const uint8_t *kcl;      // [V]
   const int64_t *f;        // finish times of the last pass
   const int64_t *d_used;   // durations of the last pass
   const int64_t *d_orig;   // durations before any slowdown
   const double *sf;        // [C][S]
-  int64_t *d_next;         // (out, compute rows)
-  uint8_t *ov;             // (out, compute rows)
+  int64_t *d_next;         // (out, compute rows; may be null)
+  uint8_t *ov;             // (out, compute rows; may be null)
 };
 
 // kernels.cu

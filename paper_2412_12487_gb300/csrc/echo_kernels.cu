@@ -636,71 +636,114 @@ compose_pipelined_kernel(StagedArgs a) {
 
 // ---------------------------------------------------------------------------------
 // B3: validator overlap test.  One thread per (chunk of a rank's compute timeline,
-// scenario).  The rank's timelines run their ops one after the other, so their
-// intervals are sorted: a binary search finds, on each comm/memcpy timeline, the
-// first op finishing after the chunk's first kernel starts, and from there one
-// monotone cursor per timeline suffices.  A compute op that overlaps a comm op with
-// positive length gets rint(d * slowdown) for the next composition, others keep d.
+// scenario); a warp covers 32 scenarios of one chunk and shares its op list.
+// Every timeline of a rank runs its ops one after the other, so on each of the
+// rank's comm timelines the intervals are sorted and the compute ops' starts only
+// grow.  The thread keeps, per comm timeline, a cursor at the first comm op of
+// positive length that finishes after the current compute op starts, with that
+// op's interval in registers: the compute op overlaps this timeline iff that
+// interval starts before the compute op finishes (any later comm op starts after
+// the cursor op ends).  A binary search places the cursors at the chunk's first
+// op; from there they only move forward, and only then touch memory.  A compute
+// op of positive length that overlaps gets rint(d * slowdown) for the next
+// composition (d_next), others keep d; the decisions themselves are stored only
+// when `ov` is given.  The finish times and durations of 8 consecutive ops are
+// loaded together before they are tested.
 // ---------------------------------------------------------------------------------
-__global__ void overlap_kernel(OverlapArgs a) {
+constexpr int kOverlapThreads = 128;
+constexpr int kOverlapBatch = 8;  // divides 32 (the shuffled op list's width)
+template <int NCMAX>
+__global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a) {
   const int32_t S = a.S;
-  const MatLayout L = a.lay;
   const int32_t s = blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t c = blockIdx.y + (int64_t)gridDim.y * blockIdx.z;
-  if (s >= S || c >= a.n_chunks) return;
-  const int ns = a.n_streams;
+  if (c >= a.n_chunks) return;  // uniform over the block
+  const bool act = s < S;       // inactive lanes still take part in the warp shuffles
+  const int32_t sl = act ? s : 0;
+  const int lane = threadIdx.x & 31;
+  const int nc = a.n_cq;
   const int64_t r = a.chunks[2 * c];
-  const int64_t qbase = r * ns;
   const int64_t c0 = a.chunks[2 * c + 1];
-  const int64_t c1 = min(a.q_off[qbase + 1], c0 + kOverlapChunk);
-  const int64_t *__restrict__ f = a.f;
-  const int64_t *__restrict__ du = a.d_used;
-  int64_t cur[kMaxStreams];
-  {  // cursors: first op on each timeline that finishes after the chunk's first start
-    const int64_t v = a.q_ops[c0];
-    const int64_t sv = f[L.at(v, s)] - du[L.at(v, s)];
-    for (int k = 1; k < ns; ++k) {
-      int64_t lo = a.q_off[qbase + k], hi = a.q_off[qbase + k + 1];
-      while (lo < hi) {
-        const int64_t mid = (lo + hi) >> 1;
-        if (f[L.at(a.q_ops[mid], s)] > sv)
-          hi = mid;
-        else
-          lo = mid + 1;
+  const int64_t c1 = min(a.q_off[r * a.n_streams + 1], c0 + kOverlapChunk);
+  // element (i, s) of a matrix sits at base + (i << sh)
+  const int sh = a.lay.slog2;
+  const int64_t base = a.lay.at(0, sl);
+  const int64_t *__restrict__ f = a.f + base;
+  const int64_t *__restrict__ du = a.d_used + base;
+  const bool same = a.d_orig == a.d_used;
+  int32_t qreg = c0 + lane < c1 ? a.q_ops[c0 + lane] : 0;  // ops c0 .. c0+31 of the chunk
+  int64_t cur[NCMAX], end[NCMAX], sw[NCMAX], fw[NCMAX];
+  {
+    const int64_t v = __shfl_sync(0xffffffffu, qreg, 0);
+    const int64_t sv = act ? f[v << sh] - du[v << sh] : 0;
+#pragma unroll
+    for (int j = 0; j < NCMAX; ++j) {
+      cur[j] = end[j] = 0;
+      sw[j] = fw[j] = INT64_MAX;
+      if (j < nc && act) {
+        int64_t lo = a.cq_off[r * nc + j], hi = a.cq_off[r * nc + j + 1];
+        end[j] = hi;
+        while (lo < hi) {  // first comm op finishing after sv (finishes are sorted)
+          const int64_t mid = (lo + hi) >> 1;
+          if (f[(int64_t)a.cq_ops[mid] << sh] > sv)
+            hi = mid;
+          else
+            lo = mid + 1;
+        }
+        cur[j] = lo;
+        if (lo < end[j]) {
+          const int64_t w = a.cq_ops[lo];
+          fw[j] = f[w << sh];
+          sw[j] = fw[j] - du[w << sh];
+        }
       }
-      cur[k] = lo;
     }
   }
-  for (int64_t i = c0; i < c1; ++i) {
-    const int64_t v = a.q_ops[i];
-    const int64_t fv = f[L.at(v, s)];
-    const int64_t sv = fv - du[L.at(v, s)];
-    const int64_t d0 = a.d_orig == du ? fv - sv : a.d_orig[L.at(v, s)];
-    uint8_t hit = 0;
-    if (sv < fv) {
-      for (int k = 1; k < ns && !hit; ++k) {
-        const int64_t e = a.q_off[qbase + k + 1];
-        int64_t cc = cur[k];
-        while (cc < e) {
-          const int64_t w = a.q_ops[cc];
-          if (a.is_comm[w] && f[L.at(w, s)] > sv) break;
-          ++cc;
-        }
-        cur[k] = cc;
-        for (int64_t jj = cc; jj < e; ++jj) {
-          const int64_t w = a.q_ops[jj];
-          const int64_t fw = f[L.at(w, s)];
-          const int64_t sw = fw - du[L.at(w, s)];
-          if (sw >= fv) break;
-          if (a.is_comm[w] && sw < fw) {
-            hit = 1;
-            break;
+  // groups of kOverlapBatch ops: their finish times and durations are loaded together
+  for (int64_t i0 = c0; i0 < c1; i0 += kOverlapBatch) {
+    if (i0 > c0 && ((i0 - c0) & 31) == 0) qreg = i0 + lane < c1 ? a.q_ops[i0 + lane] : 0;
+    int64_t vb[kOverlapBatch], fb[kOverlapBatch], db[kOverlapBatch];
+#pragma unroll
+    for (int u = 0; u < kOverlapBatch; ++u) {
+      vb[u] = __shfl_sync(0xffffffffu, qreg, (int)((i0 - c0 + u) & 31));
+      fb[u] = db[u] = 0;
+      if (act && i0 + u < c1) {
+        fb[u] = f[vb[u] << sh];
+        db[u] = du[vb[u] << sh];
+      }
+    }
+    if (!act) continue;
+#pragma unroll
+    for (int u = 0; u < kOverlapBatch; ++u) {
+      if (i0 + u < c1) {
+        const int64_t v = vb[u], fv = fb[u], dv = db[u];
+        const int64_t sv = fv - dv;
+        bool hit = false;
+#pragma unroll
+        for (int j = 0; j < NCMAX; ++j) {
+          if (j < nc) {
+            // skip comm ops that ended by sv or have zero length
+            while (cur[j] < end[j] && (fw[j] <= sv || sw[j] >= fw[j])) {
+              if (++cur[j] < end[j]) {
+                const int64_t w = a.cq_ops[cur[j]];
+                fw[j] = f[w << sh];
+                sw[j] = fw[j] - du[w << sh];
+              } else {
+                sw[j] = fw[j] = INT64_MAX;
+              }
+            }
+            hit |= sw[j] < fv;
           }
+        }
+        hit = hit && sv < fv;
+        const int64_t at = base + (v << sh);
+        if (a.ov) a.ov[at] = hit;
+        if (a.d_next) {
+          const int64_t d0 = same ? dv : a.d_orig[at];
+          a.d_next[at] = hit ? slowed(d0, a.sf[(int64_t)a.kcl[v] * S + sl]) : d0;
         }
       }
     }
-    a.ov[L.at(v, s)] = hit;
-    a.d_next[L.at(v, s)] = hit ? slowed(d0, a.sf[(int64_t)a.kcl[v] * S + s]) : d0;
   }
 }
 
@@ -893,11 +936,23 @@ cudaError_t launch_compose_pipelined(const StagedArgs &a, int sigma, const Stage
 
 cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
   if (a.S == 0 || a.n_chunks == 0) return cudaSuccess;
-  int tx = a.S >= 128 ? 128 : ((a.S + 31) / 32) * 32;
+  if (a.n_cq < 0 || a.n_cq > kMaxStreams) return cudaErrorInvalidValue;
+  const int tx = a.S >= kOverlapThreads ? kOverlapThreads : ((a.S + 31) / 32) * 32;
   int64_t gy = a.n_chunks < 65535 ? a.n_chunks : 65535;
   int64_t gz = (a.n_chunks + gy - 1) / gy;
   dim3 grid((a.S + tx - 1) / tx, (unsigned)gy, (unsigned)gz);
-  overlap_kernel<<<grid, tx, 0, st>>>(a);
+  if (a.n_cq <= 1)
+    overlap_kernel<1><<<grid, tx, 0, st>>>(a);
+  else if (a.n_cq <= 2)
+    overlap_kernel<2><<<grid, tx, 0, st>>>(a);
+  else if (a.n_cq <= 3)
+    overlap_kernel<3><<<grid, tx, 0, st>>>(a);
+  else if (a.n_cq <= 4)
+    overlap_kernel<4><<<grid, tx, 0, st>>>(a);
+  else if (a.n_cq <= 8)
+    overlap_kernel<8><<<grid, tx, 0, st>>>(a);
+  else
+    overlap_kernel<kMaxStreams><<<grid, tx, 0, st>>>(a);
   return cudaGetLastError();
 }
 

@@ -33,6 +33,9 @@ class EchoError(RuntimeError):
         self.code = code
 
 
+CUDA_STREAM_LEGACY = 0x1  # cudaStreamLegacy
+
+
 class GraphDesc(C.Structure):
     _fields_ = [("n_ops", C.c_int64), ("n_ranks", C.c_int32), ("n_streams", C.c_int32),
                 ("gpus_per_node", C.c_int32), ("n_groups", C.c_int32),
@@ -168,7 +171,12 @@ class Echo:
         if stream is None:
             import torch
             stream = torch.cuda.current_stream(device)
-        handle = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream or 0)
+        if hasattr(stream, "cuda_stream"):
+            # torch's default stream has handle 0, the legacy default stream: pass it as
+            # cudaStreamLegacy so the library's work stays in that stream's order
+            handle = stream.cuda_stream or CUDA_STREAM_LEGACY
+        else:
+            handle = int(stream or 0)
         h = C.c_void_p()
         rc = self.lib.echo_create(C.byref(h), int(device), C.c_void_p(handle) if handle else None)
         if rc:

@@ -50,9 +50,9 @@ def graph_from_lists(n_ranks, n_streams, ops, queues, groups, gpus_per_node=8):
 
 
 def random_graph(rng: np.random.Generator, n_ops: int, max_ranks: int = 3, max_streams: int = 3,
-                 gpus_per_node: int = 2, p_edge: float = 0.25):
+                 gpus_per_node: int = 2, p_edge: float = 0.25, min_streams: int = 2):
     n_ranks = int(rng.integers(1, max_ranks + 1))
-    n_streams = int(rng.integers(2, max_streams + 1))
+    n_streams = int(rng.integers(min_streams, max_streams + 1))
     ops, groups = [], []
     queues = {}
     for v in range(n_ops):

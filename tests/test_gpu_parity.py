@@ -69,6 +69,25 @@ def test_random_graphs_bit_exact(S):
         e.close()
 
 
+@pytest.mark.parametrize("S", [33, 130])
+def test_validator_many_comm_timelines_long_compute_timelines(S):
+    """Ranks with up to 15 comm timelines and several hundred compute ops each:
+    the overlap test's cursors cross chunk and warp-shuffle boundaries, and every
+    register-cursor width (1..15 comm timelines) is exercised."""
+    rng = np.random.default_rng(900 + S)
+    e = Echo(0)
+    try:
+        for case in range(16):
+            g = SG.random_graph(rng, int(rng.integers(300, 900)), max_ranks=3, max_streams=16,
+                                min_streams=6 if case % 2 else 2, p_edge=0.004)
+            sc = SG.random_scenarios(rng, g, S, max_dur=50)
+            for refine in (1, 2):
+                got = run_gpu(g, sc, refine, ctx=e)
+                assert_same(got, oracle.compose(g, sc, refine_passes=refine), g, refine)
+    finally:
+        e.close()
+
+
 def test_gpt13b_all_ops_all_scenarios_bit_exact():
     c = W.config("gpt1.3b")
     g = W.build_gpt_graph(c)
