@@ -110,7 +110,7 @@ def measured_peaks():
 
 def kernel_source_hash():
     h = hashlib.sha256()
-    with open(os.path.join(ROOT, "paper_2412_12487_gb300", "csrc", "echo_kernels.cu"), "rb") as f:
+    with open(os.path.join(ROOT, "paper_2412_12487_gb300", "csrc", "echo_compose.cu"), "rb") as f:
         h.update(f.read())
     return h.hexdigest()[:16]
 

@@ -1,6 +1,6 @@
 """Build ``libecho.so`` in-tree with nvcc for sm_103a (GB300).
 
-The two translation units compile in parallel and link into one shared library
+The three translation units compile in parallel and link into one shared library
 exporting the C ABI of ``include/echo.h``.
 """
 from __future__ import annotations
@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libecho.so")
 BUILD_DIR = os.path.join(PKG, "_build")
-SOURCES = ["echo_kernels.cu", "echo_host.cpp"]
+SOURCES = ["echo_kernels.cu", "echo_compose.cu", "echo_host.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -67,8 +67,10 @@ struct GraphBuild {
   std::vector<int64_t> cq_off;        // [R*n_cq+1] comm ops of each (rank, comm timeline)
   std::vector<int32_t> cq_ops;        // internal ids, in issue order
   std::vector<int64_t> blk_words;     // record block size of each segment level (words, padded)
+  std::vector<int64_t> hin_off;       // [n_seg+1] inputs of each segment's head
+  std::vector<int32_t> hin;           // (internal ids, each the tail of an earlier segment)
   int32_t max_kclass = -1;
-  bool stageable = true;              // every head/tail has < 2^16 timelines and predecessors
+  bool stageable = true;              // every head has < 2^16 inputs
 };
 
 bool finite_nonneg(double x) { return std::isfinite(x) && x >= 0.0; }
@@ -312,6 +314,18 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
   {
     std::vector<int64_t> cur(b.seg_lvl_off.begin(), b.seg_lvl_off.end() - 1);
     for (int64_t t = 0; t < NSg; ++t) seg_order[cur[seg_lvl[t]]++] = (int32_t)t;
+    // within a level the heaviest segments first (inputs and tail timelines weigh
+    // twice a chain step), so that a warp's lanes hold segments of similar weight
+    std::vector<int32_t> ntl(V, 0);
+    for (int64_t i = 0; i < QE; ++i) ntl[g->q_ops[i]]++;
+    std::vector<int64_t> cost(NSg);
+    for (int64_t t = 0; t < NSg; ++t) {
+      const int32_t h = seg_head[t], z = seg_tail[t];
+      cost[t] = 2 * (ntl[h] + (g->pred_off[h + 1] - g->pred_off[h]) + ntl[z]) + seg_len[t];
+    }
+    for (int64_t l = 0; l < Ls; ++l)
+      std::stable_sort(seg_order.begin() + b.seg_lvl_off[l], seg_order.begin() + b.seg_lvl_off[l + 1],
+                       [&](int32_t x, int32_t y) { return cost[x] > cost[y]; });
   }
   // internal numbering: segment levels in order, each segment's chain contiguous
   b.seg_node_off.assign(NSg + 1, 0);
@@ -330,6 +344,23 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
       }
     }
     b.seg_node_off[NSg] = i;
+  }
+  // Inputs of every segment head: its distinct predecessors over data and issue
+  // order (each the tail of an earlier segment, as a chain only continues through
+  // an op's single consumer), less any that is itself a direct predecessor of
+  // another input: that one finishes no earlier, so the maximum is unchanged.
+  b.hin_off.assign(NSg + 1, 0);
+  b.hin.clear();
+  for (int64_t t = 0; t < NSg; ++t) {
+    const int32_t v = b.int2ext[b.seg_node_off[t]];
+    const int32_t *p0 = mp.data() + mp_off[v], *p1 = mp.data() + mp_off[v + 1];
+    for (const int32_t *pu = p0; pu < p1; ++pu) {
+      bool dominated = false;
+      for (const int32_t *pw = p0; pw < p1 && !dominated; ++pw)
+        if (pw != pu) dominated = std::binary_search(mp.data() + mp_off[*pw], mp.data() + mp_off[*pw + 1], *pu);
+      if (!dominated) b.hin.push_back(b.ext2int[*pu]);
+    }
+    b.hin_off[t + 1] = (int64_t)b.hin.size();
   }
   // timelines of every internal node
   b.nq_off.assign(V + 1, 0);
@@ -446,11 +477,9 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
   for (int64_t l = 0; l < Ls; ++l) {
     int64_t w = 0;
     for (int64_t t = b.seg_lvl_off[l]; t < b.seg_lvl_off[l + 1]; ++t) {
-      const int64_t h = b.seg_node_off[t], z = b.seg_node_off[t + 1] - 1;
-      const int64_t nqf = b.nq_off[h + 1] - b.nq_off[h], ndp = b.dp_off[h + 1] - b.dp_off[h];
-      const int64_t nql = b.nq_off[z + 1] - b.nq_off[z];
-      if (nqf > 0xFFFF || ndp > 0xFFFF || nql > 0xFFFF) b.stageable = false;
-      w += 4 + nqf + ndp + nql;
+      const int64_t nin = b.hin_off[t + 1] - b.hin_off[t];
+      if (nin > 0xFFFF) b.stageable = false;
+      w += 4 + nin;
     }
     b.blk_words[l] = (w + 3) & ~(int64_t)3;
   }
@@ -465,7 +494,6 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
 echo::StagedPlan plan_staged(const GraphBuild &b, int sigma, size_t smem_cap) {
   echo::StagedPlan best;
   if (!b.stageable || b.Ls == 0) return best;
-  const int32_t NQ = b.R * b.NS;
   auto pow2 = [](int64_t x) {
     int k = 0;
     while (((int64_t)1 << k) < x) ++k;
@@ -485,7 +513,7 @@ echo::StagedPlan plan_staged(const GraphBuild &b, int sigma, size_t smem_cap) {
   for (int d = dmin + 2; d >= dmin; --d)
     for (int v = vwant; v >= 6; --v)
       for (int r = rmin + 1; r >= rmin; --r) {
-        const size_t need = echo::staged_layout(NQ, sigma, v, d, r).total;
+        const size_t need = echo::staged_layout(sigma, v, d, r).total;
         if (need <= smem_cap && d < 31 && r < 31) {
           best.ok = true;
           best.dring_log2 = d;
@@ -498,12 +526,17 @@ echo::StagedPlan plan_staged(const GraphBuild &b, int sigma, size_t smem_cap) {
   return best;
 }
 
-// Record blocks of every segment level for a value ring of 2^vlog2 segments, and
-// the per-level metadata (word offset of the block, first node, first segment).
-void build_records(const GraphBuild &b, int vlog2, std::vector<uint32_t> &recs, std::vector<uint32_t> &meta) {
+// Record blocks of every segment level for scenario blocks of `sigma` and a value
+// ring of 2^vlog2 segments, and the per-level metadata (word offset of the block,
+// first node, first segment).  A head's inputs recent enough to be in the value
+// ring become byte offsets of their slots, the others node ids.
+void build_records(const GraphBuild &b, int sigma, int vlog2, std::vector<uint32_t> &recs,
+                   std::vector<uint32_t> &meta) {
   const int64_t R = (int64_t)1 << vlog2;
+  const uint32_t row = (uint32_t)sigma * 8;
   recs.clear();
   meta.assign(4 * (b.Ls + 1), 0);
+  std::vector<uint32_t> far;
   for (int64_t l = 0; l < b.Ls; ++l) {
     const int64_t s0 = b.seg_lvl_off[l], s1 = b.seg_lvl_off[l + 1];
     const int64_t i0 = b.seg_node_off[s0];
@@ -514,21 +547,25 @@ void build_records(const GraphBuild &b, int vlog2, std::vector<uint32_t> &recs, 
     recs.resize(base + 4 * (s1 - s0), 0);
     for (int64_t t = s0; t < s1; ++t) {
       const int64_t h = b.seg_node_off[t], z = b.seg_node_off[t + 1] - 1;
-      const int64_t nqf = b.nq_off[h + 1] - b.nq_off[h], ndp = b.dp_off[h + 1] - b.dp_off[h];
-      const int64_t nql = b.nq_off[z + 1] - b.nq_off[z];
       const size_t hd = base + 4 * (t - s0);
       recs[hd] = (uint32_t)(recs.size() - base);
-      recs[hd + 1] = (uint32_t)(nqf | (ndp << 16));
       recs[hd + 2] = (uint32_t)(h - i0);
-      recs[hd + 3] = (uint32_t)((z - h + 1) | (nql << 16));
-      for (int64_t q = b.nq_off[h]; q < b.nq_off[h + 1]; ++q) recs.push_back((uint32_t)b.nq[q]);
-      for (int64_t q = b.dp_off[h]; q < b.dp_off[h + 1]; ++q) {
-        // a predecessor of a head is the tail of its segment; its value-ring slot is
-        // rewritten by segment seg+R, which must not be in segment levels <= l
-        const int64_t u = b.dp[q], su = b.seg_int[u];
-        recs.push_back(su + R >= s1 ? (uint32_t)su : ((uint32_t)u | echo::kFarRef));
+      recs[hd + 3] = (uint32_t)(z - h + 1);
+      far.clear();
+      uint32_t nin = 0;
+      for (int64_t q = b.hin_off[t]; q < b.hin_off[t + 1]; ++q) {
+        // an input's value-ring slot is rewritten by segment seg+R, which must not
+        // be in segment levels <= l
+        const int64_t u = b.hin[q], su = b.seg_int[u];
+        if (su + R >= s1) {
+          recs.push_back((uint32_t)(su & (R - 1)) * row);
+          ++nin;
+        } else {
+          far.push_back((uint32_t)u);
+        }
       }
-      for (int64_t q = b.nq_off[z]; q < b.nq_off[z + 1]; ++q) recs.push_back((uint32_t)b.nq[q]);
+      recs.insert(recs.end(), far.begin(), far.end());
+      recs[hd + 1] = nin | ((uint32_t)far.size() << 16);
     }
     while (recs.size() % 4) recs.push_back(0);
   }
@@ -571,7 +608,9 @@ struct echo_ctx {
   size_t scen_vs = 0;  // elements of each [op][scenario] matrix (blocked layout, padded)
   echo::MatLayout lay{0, 0};
   ChunkTable tbl{};
-  double *prm = nullptr, *sf = nullptr, *sums = nullptr, *comm_sum = nullptr, *cc_ns = nullptr;
+  double *prm = nullptr, *sums = nullptr, *comm_sum = nullptr, *cc_ns = nullptr;
+  uint64_t *sfx = nullptr;  // packed slowdown factors [C][S]
+  std::vector<uint64_t> h_sfx;
   int64_t *raw = nullptr, *dur = nullptr, *f[2] = {nullptr, nullptr}, *mk = nullptr, *cc_dur = nullptr;
   int64_t *gfrontier = nullptr;
   int64_t *deff[2] = {nullptr, nullptr};  // durations of the validator's passes
@@ -913,7 +952,7 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     bool in_smem = true;
     echo::compose_smem_bytes(B.R * B.NS, sigma, &in_smem);
     int64_t nblk = (S + sigma - 1) / sigma;
-    if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sf, (size_t)C * S)) ||
+    if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sfx, (size_t)C * S)) ||
         (rc = dalloc(c, o, &c->sums, (size_t)S)) || (rc = dalloc(c, o, &c->comm_sum, (size_t)S)) ||
         (rc = dalloc(c, o, &c->raw, (size_t)V * S)) || (rc = dalloc(c, o, &c->dur, VS)) ||
         (rc = dalloc(c, o, &c->f[0], VS)) || (rc = dalloc(c, o, &c->f[1], VS)) ||
@@ -951,7 +990,7 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
       }
       c->plan.pipelined = sigma % 2 == 0 && max_bytes < (1 << 20);
       std::vector<uint32_t> recs, meta;
-      build_records(B, c->plan.vring_log2, recs, meta);
+      build_records(B, sigma, c->plan.vring_log2, recs, meta);
       c->rec_words = meta[4 * B.Ls];
       if ((rc = upload(c, o, &c->d_recs, recs)) || (rc = upload(c, o, &c->d_meta, meta))) {
         free_all(c->scen_allocs);
@@ -970,7 +1009,16 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   const double *src[6] = {sc->alpha_ns, sc->bw_intra, sc->lat_intra, sc->bw_inter, sc->lat_inter, sc->delta};
   for (int k = 0; k < 6; ++k)
     CK(cudaMemcpyAsync(c->prm + (size_t)k * S, src[k], S * sizeof(double), cudaMemcpyHostToDevice, c->stream), "parameter upload");
-  CK(cudaMemcpyAsync(c->sf, sc->slowdown, (size_t)C * S * sizeof(double), cudaMemcpyHostToDevice, c->stream), "slowdown upload");
+  // slowdown factors as (significand << 11) | biased exponent (factors are finite and > 0)
+  c->h_sfx.resize((size_t)C * S);
+  for (size_t k = 0; k < c->h_sfx.size(); ++k) {
+    uint64_t b;
+    std::memcpy(&b, &sc->slowdown[k], sizeof b);
+    const uint64_t ex = (b >> 52) & 0x7FF, fr = b & ((1ull << 52) - 1);
+    c->h_sfx[k] = ex == 0 ? (fr << 11) | 1 : ((fr | (1ull << 52)) << 11) | ex;
+  }
+  CK(cudaMemcpyAsync(c->sfx, c->h_sfx.data(), c->h_sfx.size() * sizeof(uint64_t), cudaMemcpyHostToDevice, c->stream),
+     "slowdown upload");
   CK(cudaMemsetAsync(c->sums, 0, S * sizeof(double), c->stream), "memset");
   CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
   if (V > 0) {
@@ -1042,7 +1090,6 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       echo::StagedArgs a{};
       a.S = c->S;
       a.L = (int32_t)B.Ls;
-      a.n_queues = B.R * B.NS;
       a.n_rows = (uint32_t)B.V;
       a.n_words = c->rec_words;
       a.vlog2 = c->plan.vring_log2;
@@ -1098,7 +1145,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     o.f = c->f[(p - 1) % 2];
     o.d_used = d_used;
     o.d_orig = c->dur;
-    o.sf = c->sf;
+    o.sfx = c->sfx;
     o.d_next = c->deff[(p - 1) % 2];
     o.ov = nullptr;  // the decisions are recomputed on demand by echo_read_overlap
     CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");

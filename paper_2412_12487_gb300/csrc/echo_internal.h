@@ -74,12 +74,12 @@ struct ComposeArgs {
 // Staged and pipelined compose: per-segment-level records and duration rows are
 // copied into shared-memory rings ahead of use.  Record block of a level (32-bit
 // words): for each segment, 4 header words {offset of its entries in the block,
-// nqf | ndp << 16, first node - level's first node, length | nql << 16}; entries =
-// the head's nqf timeline ids, its ndp predecessor references (a segment id for
-// the value ring, or a node id with kFarRef set, read from global memory), the
-// tail's nql timeline ids.  Blocks are padded to 4 words.
+// nin | nfar << 16, first node - level's first node, length}; entries = the
+// head's nin inputs held in the value ring (byte offsets of their slots), then its
+// nfar inputs too old for the ring (node ids, read from global memory).  Every
+// input is the tail of an earlier segment.  Blocks are padded to 4 words.
 struct StagedArgs {
-  int32_t S, L, n_queues;        // L: segment levels
+  int32_t S, L;                  // L: segment levels
   uint32_t n_rows, n_words;      // nodes; words of all record blocks
   int32_t vlog2, dlog2, rlog2;   // log2 sizes: value ring (segments), duration ring (rows), record ring (words)
   const uint32_t *meta;          // [4*(L+1)]: record word offset, first node, first segment, 0
@@ -105,16 +105,14 @@ struct StagedPlan {
 // Shared-memory layout of the staged kernels (byte offsets).  Every region starts
 // on a 16-byte boundary, as 16-byte copy destinations require.
 struct StagedLayout {
-  size_t hist, meta, fr, vr, dr, rr, total;
+  size_t hist, meta, vr, dr, rr, total;
 };
 __host__ __device__ inline size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
-__host__ __device__ inline StagedLayout staged_layout(int32_t n_queues, int sigma, int vlog2, int dlog2,
-                                                      int rlog2) {
+__host__ __device__ inline StagedLayout staged_layout(int sigma, int vlog2, int dlog2, int rlog2) {
   StagedLayout L;
   L.hist = 128;                        // [0, 128): per-scenario makespans
   L.meta = L.hist + 16 * 8;            // 16 copy-group extents
-  L.fr = L.meta + round16((size_t)2 * kMetaCap * 16);
-  L.vr = L.fr + round16((size_t)n_queues * sigma * 8);
+  L.vr = L.meta + round16((size_t)2 * kMetaCap * 16);
   L.dr = L.vr + round16(((size_t)1 << vlog2) * sigma * 8);
   L.rr = L.dr + round16(((size_t)1 << dlog2) * sigma * 8);
   L.total = L.rr + round16(((size_t)1 << rlog2) * 4);
@@ -135,7 +133,7 @@ struct OverlapArgs {
   const int64_t *f;        // finish times of the last pass
   const int64_t *d_used;   // durations of the last pass
   const int64_t *d_orig;   // durations before any slowdown
-  const double *sf;        // [C][S]
+  const uint64_t *sfx;     // [C][S] slowdown factors, packed as (53-bit significand << 11) | (exponent + 1075)
   int64_t *d_next;         // (out, compute rows; may be null)
   uint8_t *ov;             // (out, compute rows; may be null)
 };

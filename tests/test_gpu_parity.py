@@ -88,6 +88,39 @@ def test_validator_many_comm_timelines_long_compute_timelines(S):
         e.close()
 
 
+def test_slowdown_rounding_is_exact():
+    """The validator evaluates rint(d * factor) in integers: every scenario slows one
+    kernel that overlaps a collective from time 0, with edge-case durations (around
+    2^31, 2^52, 2^53, large) and factors (exact ties, 1 + 2^-52, 1/3, tiny, subnormal),
+    and the slowed duration must equal the fp64 product rounded to nearest even."""
+    ops = [{"kind": W.KIND_COMPUTE, "kclass": 0}, {"kind": W.KIND_COMPUTE, "kclass": 0},
+           {"kind": W.KIND_COLL, "group": 0, "cc_type": W.CC_ALLREDUCE, "cc_bytes": 1 << 20}]
+    g = SG.graph_from_lists(2, 2, ops, {(0, 0): [0], (1, 0): [1], (0, 1): [2], (1, 1): [2]}, [[0, 1]])
+    edge_d = [0, 1, 2, 3, 5, 7, 2**31 - 1, 2**31, 2**32 + 1, 2**52 - 1, 2**52, 2**52 + 1, 2**53 - 1, 2**53,
+              2**53 + 1, 2**53 + 3, 2**54 + 2, 2**55 + 7, 2**56 + 12345, 2**57 - 1]
+    edge_f = [1.0, 1.5, 2.5, 0.5, 0.25, 1.0000000000000002, 1.4, 1.2, 1 / 3, 0.9999999999999999, 3.0,
+              1e-300, 5e-324, 2.2250738585072014e-308, 1.1, 1.3999999999999999, 1.25, 0.1]
+    rng = np.random.default_rng(2024)
+    pairs = [(d, f) for d in edge_d for f in edge_f]
+    for _ in range(3000):
+        d = int(rng.integers(0, 1 << int(rng.choice([3, 10, 20, 31, 40, 50, 53, 54, 56]))))
+        f = float(rng.choice([rng.uniform(1.0, 1.4), rng.uniform(0.0, 3.0), rng.integers(1, 48) / 16]))
+        pairs.append((d, f))
+    S = len(pairs)
+    d = np.array([p[0] for p in pairs], np.int64)
+    f = np.array([p[1] for p in pairs], np.float64)
+    sc = W.Scenarios(dur=np.stack([d, d, np.zeros(S, np.int64)]), alpha_ns=np.full(S, 100.0),
+                     bw_intra=np.full(S, 50.0), lat_intra=np.full(S, 10.0), bw_inter=np.full(S, 5.0),
+                     lat_inter=np.full(S, 20.0), delta=np.zeros(S), slowdown=f[None, :].copy(),
+                     peak_flop_per_ns=np.ones(S))
+    got = run_gpu(g, sc, 1)
+    want = np.rint(d.astype(np.float64) * f).astype(np.int64)
+    want[d == 0] = 0
+    for v in (0, 1):
+        assert np.array_equal(got["finish"][v] - got["start"][v], want)
+    assert_same(got, oracle.compose(g, sc, refine_passes=1), g, 1)
+
+
 def test_gpt13b_all_ops_all_scenarios_bit_exact():
     c = W.config("gpt1.3b")
     g = W.build_gpt_graph(c)
