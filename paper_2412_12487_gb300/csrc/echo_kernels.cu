@@ -237,7 +237,20 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
   const int64_t *__restrict__ du = a.d_used + base;
   const bool same = a.d_orig == a.d_used;
   int32_t qreg = c0 + lane < c1 ? a.q_ops[c0 + lane] : 0;  // ops c0 .. c0+31 of the chunk
-  int64_t cur[NCMAX], end[NCMAX], sw[NCMAX], fw[NCMAX];
+  // per comm timeline: position, end, and interval of the cursor op; the cursor op
+  // always has positive length and finishes after the current op's start (or the
+  // cursor is at the end, with an interval that never overlaps)
+  int32_t cur[NCMAX], end[NCMAX];
+  int64_t sw[NCMAX], fw[NCMAX];
+  auto load = [&](int j) {
+    if (cur[j] < end[j]) {
+      const int64_t w = a.cq_ops[cur[j]];
+      fw[j] = f[w << sh];
+      sw[j] = fw[j] - du[w << sh];
+    } else {
+      sw[j] = fw[j] = INT64_MAX;
+    }
+  };
   {
     const int64_t v = __shfl_sync(0xffffffffu, qreg, 0);
     const int64_t sv = act ? f[v << sh] - du[v << sh] : 0;
@@ -246,20 +259,20 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
       cur[j] = end[j] = 0;
       sw[j] = fw[j] = INT64_MAX;
       if (j < nc && act) {
-        int64_t lo = a.cq_off[r * nc + j], hi = a.cq_off[r * nc + j + 1];
+        int32_t lo = (int32_t)a.cq_off[r * nc + j], hi = (int32_t)a.cq_off[r * nc + j + 1];
         end[j] = hi;
         while (lo < hi) {  // first comm op finishing after sv (finishes are sorted)
-          const int64_t mid = (lo + hi) >> 1;
+          const int32_t mid = (lo + hi) >> 1;
           if (f[(int64_t)a.cq_ops[mid] << sh] > sv)
             hi = mid;
           else
             lo = mid + 1;
         }
         cur[j] = lo;
-        if (lo < end[j]) {
-          const int64_t w = a.cq_ops[lo];
-          fw[j] = f[w << sh];
-          sw[j] = fw[j] - du[w << sh];
+        load(j);
+        while (cur[j] < end[j] && sw[j] >= fw[j]) {  // zero-length ops never overlap
+          ++cur[j];
+          load(j);
         }
       }
     }
@@ -287,15 +300,11 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
 #pragma unroll
         for (int j = 0; j < NCMAX; ++j) {
           if (j < nc) {
-            // skip comm ops that ended by sv or have zero length
-            while (cur[j] < end[j] && (fw[j] <= sv || sw[j] >= fw[j])) {
-              if (++cur[j] < end[j]) {
-                const int64_t w = a.cq_ops[cur[j]];
-                fw[j] = f[w << sh];
-                sw[j] = fw[j] - du[w << sh];
-              } else {
-                sw[j] = fw[j] = INT64_MAX;
-              }
+            if (fw[j] <= sv) {  // the cursor op ended before this op starts: move on
+              do {
+                ++cur[j];
+                load(j);
+              } while (cur[j] < end[j] && (fw[j] <= sv || sw[j] >= fw[j]));
             }
             hit |= sw[j] < fv;
           }
