@@ -258,7 +258,7 @@ def run_echo(args):
     e2e_value = units * world / (e2e_ms / 1e3)
 
     comp_launches, comp_ms = prof.get("compose", (0, 0.0))
-    launches = sum(n for n, _ in prof.values())
+    launches = sum(n for k, (n, _) in prof.items() if k != "dur_copy")  # kernels only
     peak, peak_kind = measured_peaks()
     b_pass = algorithmic_bytes_per_pass(g, info, S)
     per_launch_ms = comp_ms / max(comp_launches, 1)

@@ -219,6 +219,8 @@ typedef struct {
   int64_t n_ops, n_edges, n_levels, max_width, n_queue_entries, n_comm_ops, n_signatures;
   int64_t n_segments;        /* serial chains the composer contracts into one step each */
   int64_t n_segment_levels;  /* synchronized steps of one composition                   */
+  int64_t n_overlap_candidates; /* compute ops the validator tests (the others can never
+                                   overlap a comm op of their rank, whatever the durations) */
   int32_t n_ranks, n_streams, sigma; /* sigma: scenarios per thread block of the composer */
 } echo_graph_info;
 int echo_graph_info_get(echo_ctx *ctx, echo_graph_info *info);

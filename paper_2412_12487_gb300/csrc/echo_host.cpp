@@ -61,8 +61,10 @@ struct GraphBuild {
   std::vector<int32_t> q_ops_int;
   std::vector<CcSig> sigs;
   std::vector<int32_t> sig_count, comm_node, comm_sig, node_sig;
-  std::vector<int32_t> non_compute;   // internal ids of comm and memcpy ops
-  std::vector<int64_t> ov_chunks;     // (rank, first position) of compute-timeline chunks
+  std::vector<int64_t> cand_off;      // [R+1] overlap candidates of each rank (compute ops, issue order)
+  std::vector<int32_t> cand_ops;      // (internal ids)
+  std::vector<uint8_t> cand_flag;     // [V] 1 for an overlap candidate
+  std::vector<int64_t> ov_chunks;     // (rank, first candidate index) of the overlap test's chunks
   int32_t n_cq = 0;                   // comm timelines per rank in cq_off (max over ranks)
   std::vector<int64_t> cq_off;        // [R*n_cq+1] comm ops of each (rank, comm timeline)
   std::vector<int32_t> cq_ops;        // internal ids, in issue order
@@ -74,6 +76,94 @@ struct GraphBuild {
 };
 
 bool finite_nonneg(double x) { return std::isfinite(x) && x >= 0.0; }
+
+// Compute ops that can overlap a comm op of their rank in some scenario (the
+// validator of Sec. 3 tests only these).  A rank's compute timeline is a serial
+// chain, so for a comm op w on rank r the compute ops of r up to the latest one
+// that reaches w finish before w starts, and those from the earliest one that w
+// reaches on start after w ends: only positions in between, (anc(w), desc(w)),
+// can intersect w's interval, whatever the durations.  anc and desc follow the
+// edges among rank r's own ops (data edges and the order of r's timelines); paths
+// through other ranks are ignored, which only widens the ranges.  Needs the
+// internal numbering (a topological order), q_off/q_ops_int and dp.
+void overlap_candidates(GraphBuild &b) {
+  const int64_t V = b.V;
+  const int32_t R = b.R, NS = b.NS;
+  std::vector<int64_t> su_off(V + 1, 0);  // data successors
+  for (int64_t q = 0; q < b.dp_off[V]; ++q) su_off[b.dp[q] + 1]++;
+  for (int64_t v = 0; v < V; ++v) su_off[v + 1] += su_off[v];
+  std::vector<int32_t> su(std::max<int64_t>(su_off[V], 1));
+  {
+    std::vector<int64_t> fill(su_off.begin(), su_off.end() - 1);
+    for (int64_t v = 0; v < V; ++v)
+      for (int64_t q = b.dp_off[v]; q < b.dp_off[v + 1]; ++q) su[fill[b.dp[q]]++] = (int32_t)v;
+  }
+  std::vector<int32_t> loc(V, -1);
+  b.cand_off.assign(R + 1, 0);
+  b.cand_ops.clear();
+  b.cand_flag.assign(V, 0);
+  b.ov_chunks.clear();
+  std::vector<int32_t> nodes, cpos, prv, nxt, anc, desc;
+  std::vector<int64_t> cover;
+  for (int32_t r = 0; r < R; ++r) {
+    nodes.clear();
+    for (int32_t k = 0; k < NS; ++k)
+      for (int64_t i = b.q_off[(int64_t)r * NS + k]; i < b.q_off[(int64_t)r * NS + k + 1]; ++i)
+        nodes.push_back(b.q_ops_int[i]);
+    std::sort(nodes.begin(), nodes.end());  // a topological order
+    const int64_t m = (int64_t)nodes.size();
+    for (int64_t j = 0; j < m; ++j) loc[nodes[j]] = (int32_t)j;
+    const int64_t c0 = b.q_off[(int64_t)r * NS], n = b.q_off[(int64_t)r * NS + 1] - c0;
+    cpos.assign(m, -1);
+    prv.assign(m, -1);
+    nxt.assign(m, -1);
+    for (int64_t i = c0; i < c0 + n; ++i) cpos[loc[b.q_ops_int[i]]] = (int32_t)(i - c0);
+    for (int32_t k = 0; k < NS; ++k)
+      for (int64_t i = b.q_off[(int64_t)r * NS + k] + 1; i < b.q_off[(int64_t)r * NS + k + 1]; ++i) {
+        prv[loc[b.q_ops_int[i]]] = loc[b.q_ops_int[i - 1]];
+        nxt[loc[b.q_ops_int[i - 1]]] = loc[b.q_ops_int[i]];
+      }
+    anc.assign(m, -1);
+    for (int64_t j = 0; j < m; ++j) {  // latest compute position of r reaching the op
+      int32_t x = cpos[j];
+      if (prv[j] >= 0) x = std::max(x, anc[prv[j]]);
+      for (int64_t q = b.dp_off[nodes[j]]; q < b.dp_off[nodes[j] + 1]; ++q)
+        if (loc[b.dp[q]] >= 0) x = std::max(x, anc[loc[b.dp[q]]]);
+      anc[j] = x;
+    }
+    desc.assign(m, (int32_t)n);
+    for (int64_t j = m - 1; j >= 0; --j) {  // earliest compute position of r the op reaches
+      int32_t x = cpos[j] >= 0 ? cpos[j] : (int32_t)n;
+      if (nxt[j] >= 0) x = std::min(x, desc[nxt[j]]);
+      for (int64_t q = su_off[nodes[j]]; q < su_off[nodes[j] + 1]; ++q)
+        if (loc[su[q]] >= 0) x = std::min(x, desc[loc[su[q]]]);
+      desc[j] = x;
+    }
+    cover.assign(n + 1, 0);
+    for (int64_t j = 0; j < m; ++j)
+      if (b.is_comm[nodes[j]] && anc[j] + 1 < desc[j]) {
+        cover[anc[j] + 1]++;
+        cover[desc[j]]--;
+      }
+    const int64_t first = (int64_t)b.cand_ops.size();
+    int64_t run = 0;
+    for (int64_t p = 0; p < n; ++p) {
+      run += cover[p];
+      if (run > 0) {
+        const int32_t v = b.q_ops_int[c0 + p];
+        b.cand_ops.push_back(v);
+        b.cand_flag[v] = 1;
+      }
+    }
+    for (int64_t p = first; p < (int64_t)b.cand_ops.size(); p += echo::kOverlapChunk) {
+      b.ov_chunks.push_back(r);
+      b.ov_chunks.push_back(p);
+    }
+    b.cand_off[r + 1] = (int64_t)b.cand_ops.size();
+    for (int64_t j = 0; j < m; ++j) loc[nodes[j]] = -1;
+  }
+  if (b.cand_ops.empty()) b.cand_ops.push_back(0);
+}
 
 int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
   if (!g) return fail(e, ECHO_E_INVALID_ARG, "graph descriptor is NULL");
@@ -438,15 +528,8 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
       b.comm_sig.push_back(s);
       b.node_sig[i] = s;
     }
-    if (kd != ECHO_OP_COMPUTE) b.non_compute.push_back((int32_t)i);
   }
-  for (int32_t r = 0; r < R; ++r) {
-    const int64_t a = g->q_off[(int64_t)r * NS], z = g->q_off[(int64_t)r * NS + 1];
-    for (int64_t p = a; p < z; p += echo::kOverlapChunk) {
-      b.ov_chunks.push_back(r);
-      b.ov_chunks.push_back(p);
-    }
-  }
+  overlap_candidates(b);
   // the comm ops of each rank's timelines that hold any, in issue order
   for (int32_t r = 0; r < R; ++r) {
     int32_t n = 0;
@@ -597,7 +680,9 @@ struct echo_ctx {
   int64_t *seg_lvl_off = nullptr, *seg_node_off = nullptr, *nq_off = nullptr, *dp_off = nullptr, *q_off = nullptr;
   int64_t *ov_chunks = nullptr, *cq_off = nullptr;
   int32_t *cq_ops = nullptr;
-  int32_t *non_compute = nullptr;
+  int64_t *cand_off = nullptr;
+  int32_t *cand_ops = nullptr;
+  uint8_t *cand_flag = nullptr;
   int32_t *nq = nullptr, *dp = nullptr, *q_ops = nullptr, *int2ext = nullptr, *ext2int = nullptr;
   int32_t *node_sig = nullptr, *comm_node = nullptr, *comm_sig = nullptr, *sig_count = nullptr;
   uint8_t *kcl = nullptr, *local = nullptr;
@@ -893,7 +978,9 @@ int echo_load_graph(echo_ctx *c, const echo_graph_desc *g) {
   auto &o = c->graph_allocs;
   if ((rc = upload(c, o, &c->seg_lvl_off, B.seg_lvl_off)) || (rc = upload(c, o, &c->seg_node_off, B.seg_node_off)) ||
       (rc = upload(c, o, &c->ov_chunks, B.ov_chunks)) ||
-      (rc = upload(c, o, &c->cq_off, B.cq_off)) || (rc = upload(c, o, &c->cq_ops, B.cq_ops)) || (rc = upload(c, o, &c->non_compute, B.non_compute)) ||
+      (rc = upload(c, o, &c->cq_off, B.cq_off)) || (rc = upload(c, o, &c->cq_ops, B.cq_ops)) ||
+      (rc = upload(c, o, &c->cand_off, B.cand_off)) || (rc = upload(c, o, &c->cand_ops, B.cand_ops)) ||
+      (rc = upload(c, o, &c->cand_flag, B.cand_flag)) ||
       (rc = upload(c, o, &c->nq_off, B.nq_off)) ||
       (rc = upload(c, o, &c->nq, B.nq)) || (rc = upload(c, o, &c->dp_off, B.dp_off)) ||
       (rc = upload(c, o, &c->dp, B.dp)) || (rc = upload(c, o, &c->q_off, B.q_off)) ||
@@ -1136,8 +1223,8 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     o.n_streams = B.NS;
     o.n_chunks = (int64_t)B.ov_chunks.size() / 2;
     o.chunks = c->ov_chunks;
-    o.q_off = c->q_off;
-    o.q_ops = c->q_ops;
+    o.cand_off = c->cand_off;
+    o.cand_ops = c->cand_ops;
     o.n_cq = B.n_cq;
     o.cq_off = c->cq_off;
     o.cq_ops = c->cq_ops;
@@ -1148,11 +1235,11 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     o.sfx = c->sfx;
     o.d_next = c->deff[(p - 1) % 2];
     o.ov = nullptr;  // the decisions are recomputed on demand by echo_read_overlap
+    // ops that cannot overlap keep their durations; the test rewrites the candidates
+    CK(timed(c, "dur_copy", [&] {
+         return cudaMemcpyAsync(o.d_next, c->dur, c->scen_vs * sizeof(int64_t), cudaMemcpyDeviceToDevice, c->stream);
+       }), "duration copy");
     CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");
-    CK(timed(c, "copy_rows", [&] {
-         return echo::launch_copy_rows(c->non_compute, (int64_t)B.non_compute.size(), c->S, c->lay, c->dur,
-                                       o.d_next, c->stream);
-       }), "copy_rows launch");
     CK(compose_pass(o.d_next, c->f[p % 2]), "compose launch");
     d_used = o.d_next;
     c->last_ov = o;
@@ -1262,7 +1349,7 @@ int echo_read_overlap(echo_ctx *c, int64_t op0, int64_t op1, uint8_t *out) {
     int64_t n = (b - a) * S;
     uint8_t *d = static_cast<uint8_t *>(c->stage);
     CK(timed(c, "read_overlap", [&] {
-         return echo::launch_read_ov(c->ext2int, a, b, S, c->lay, ov, c->kcl, d, c->stream);
+         return echo::launch_read_ov(c->ext2int, a, b, S, c->lay, ov, c->cand_flag, d, c->stream);
        }), "read_overlap launch");
     CK(cudaMemcpyAsync(out + (a - op0) * S, d, n, cudaMemcpyDeviceToHost, c->stream), "D2H");
     CK(cudaStreamSynchronize(c->stream), "read_overlap");
@@ -1340,6 +1427,7 @@ int echo_graph_info_get(echo_ctx *c, echo_graph_info *info) {
   info->n_signatures = (int64_t)B.sigs.size();
   info->n_segments = B.n_seg;
   info->n_segment_levels = B.Ls;
+  info->n_overlap_candidates = B.cand_off.empty() ? 0 : B.cand_off.back();
   info->n_ranks = B.R;
   info->n_streams = B.NS;
   info->sigma = c->sigma;

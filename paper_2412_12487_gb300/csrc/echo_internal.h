@@ -119,15 +119,15 @@ __host__ __device__ inline StagedLayout staged_layout(int sigma, int vlog2, int 
   return L;
 }
 
-// Validator: for each compute op, whether its interval overlaps a comm op of its
-// rank, and the duration to use in the next composition.
+// Validator: for each overlap candidate (a compute op), whether its interval
+// overlaps a comm op of its rank, and the duration to use in the next composition.
 struct OverlapArgs {
   MatLayout lay;
   int32_t S, n_streams;
   int32_t n_cq;            // comm timelines per rank (lists of a rank with fewer are empty)
   int64_t n_chunks;
-  const int64_t *chunks;   // [n_chunks][2]: (rank, first compute-timeline position)
-  const int64_t *q_off; const int32_t *q_ops;    // timelines in internal ids (compute: stream 0)
+  const int64_t *chunks;   // [n_chunks][2]: (rank, first candidate index)
+  const int64_t *cand_off; const int32_t *cand_ops;  // [R+1]: each rank's overlap candidates, in issue order
   const int64_t *cq_off; const int32_t *cq_ops;  // [R*n_cq+1]: comm ops of each (rank, comm timeline)
   const uint8_t *kcl;      // [V]
   const int64_t *f;        // finish times of the last pass
@@ -154,15 +154,13 @@ cudaError_t launch_compose(const ComposeArgs &a, int sigma, cudaStream_t st);
 cudaError_t launch_compose_staged(const StagedArgs &a, int sigma, const StagedPlan &plan, cudaStream_t st);
 cudaError_t launch_compose_pipelined(const StagedArgs &a, int sigma, const StagedPlan &plan, cudaStream_t st);
 cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st);
-cudaError_t launch_copy_rows(const int32_t *rows, int64_t n_rows, int32_t S, MatLayout lay, const int64_t *src,
-                             int64_t *dst, cudaStream_t st);
 cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
                             const int64_t *f, const int64_t *d, int64_t *start, int64_t *finish,
                             cudaStream_t st);
 cudaError_t launch_read_cc(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S,
                            const int32_t *node_sig, const double *cc_ns, double *out, cudaStream_t st);
 cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
-                           const uint8_t *ov, const uint8_t *kcl, uint8_t *out, cudaStream_t st);
+                           const uint8_t *ov, const uint8_t *cand, uint8_t *out, cudaStream_t st);
 size_t compose_smem_bytes(int32_t n_queues, int sigma, bool *frontier_in_smem);
 
 }  // namespace echo

@@ -200,12 +200,15 @@ __global__ void permute_rows_kernel(const int64_t *__restrict__ raw, const int32
 }
 
 // ---------------------------------------------------------------------------------
-// B3: validator overlap test.  One thread per (chunk of a rank's compute timeline,
-// scenario); a warp covers 32 scenarios of one chunk and shares its op list.
+// B3: validator overlap test over the overlap candidates: the compute ops that
+// some comm op of their rank is neither an ancestor nor a descendant of (the
+// others can never overlap; their durations are copied unchanged).  One thread
+// per (chunk of a rank's candidates, which run in issue order, scenario); a warp
+// covers 32 scenarios of one chunk and shares its op list.
 // Every timeline of a rank runs its ops one after the other, so on each of the
 // rank's comm timelines the intervals are sorted and the compute ops' starts only
 // grow.  The thread keeps, per comm timeline, a cursor at the first comm op of
-// positive length that finishes after the current compute op starts, with that
+// positive length that finishes after the current candidate starts, with that
 // op's interval in registers: the compute op overlaps this timeline iff that
 // interval starts before the compute op finishes (any later comm op starts after
 // the cursor op ends).  A binary search places the cursors at the chunk's first
@@ -229,18 +232,18 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
   const int nc = a.n_cq;
   const int64_t r = a.chunks[2 * c];
   const int64_t c0 = a.chunks[2 * c + 1];
-  const int64_t c1 = min(a.q_off[r * a.n_streams + 1], c0 + kOverlapChunk);
+  const int64_t c1 = min(a.cand_off[r + 1], c0 + kOverlapChunk);
   // element (i, s) of a matrix sits at base + (i << sh)
   const int sh = a.lay.slog2;
   const int64_t base = a.lay.at(0, sl);
   const int64_t *__restrict__ f = a.f + base;
   const int64_t *__restrict__ du = a.d_used + base;
   const bool same = a.d_orig == a.d_used;
-  int32_t qreg = c0 + lane < c1 ? a.q_ops[c0 + lane] : 0;  // ops c0 .. c0+31 of the chunk
+  int32_t qreg = c0 + lane < c1 ? a.cand_ops[c0 + lane] : 0;  // ops c0 .. c0+31 of the chunk
   // per comm timeline: position, end, and interval of the cursor op; the cursor op
   // always has positive length and finishes after the current op's start (or the
   // cursor is at the end, with an interval that never overlaps)
-  int32_t cur[NCMAX], end[NCMAX];
+  int32_t cur[NCMAX] = {}, end[NCMAX] = {};
   int64_t sw[NCMAX], fw[NCMAX];
   auto load = [&](int j) {
     if (cur[j] < end[j]) {
@@ -279,7 +282,7 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
   }
   // groups of kOverlapBatch ops: their finish times and durations are loaded together
   for (int64_t i0 = c0; i0 < c1; i0 += kOverlapBatch) {
-    if (i0 > c0 && ((i0 - c0) & 31) == 0) qreg = i0 + lane < c1 ? a.q_ops[i0 + lane] : 0;
+    if (i0 > c0 && ((i0 - c0) & 31) == 0) qreg = i0 + lane < c1 ? a.cand_ops[i0 + lane] : 0;
     int64_t vb[kOverlapBatch], fb[kOverlapBatch], db[kOverlapBatch];
 #pragma unroll
     for (int u = 0; u < kOverlapBatch; ++u) {
@@ -321,17 +324,6 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
   }
 }
 
-__global__ void copy_rows_kernel(const int32_t *__restrict__ rows, int64_t n_rows, int32_t S, MatLayout lay,
-                                 const int64_t *__restrict__ src, int64_t *__restrict__ dst) {
-  int64_t total = n_rows * S;
-  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-       idx += (int64_t)gridDim.x * blockDim.x) {
-    int64_t k = idx / S;
-    int64_t at = lay.at(rows[k], (int32_t)(idx - k * S));
-    dst[at] = src[at];
-  }
-}
-
 // ---------------------------------------------------------------------------------
 // readback: internal order and blocked layout -> caller order, [op][scenario]
 // ---------------------------------------------------------------------------------
@@ -364,7 +356,7 @@ __global__ void read_cc_kernel(const int32_t *__restrict__ ext2int, int64_t op0,
 }
 
 __global__ void read_ov_kernel(const int32_t *__restrict__ ext2int, int64_t op0, int64_t op1, int32_t S,
-                               MatLayout lay, const uint8_t *__restrict__ ov, const uint8_t *__restrict__ kcl,
+                               MatLayout lay, const uint8_t *__restrict__ ov, const uint8_t *__restrict__ cand,
                                uint8_t *__restrict__ out) {
   int64_t total = (op1 - op0) * S;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
@@ -372,7 +364,7 @@ __global__ void read_ov_kernel(const int32_t *__restrict__ ext2int, int64_t op0,
     int64_t o = idx / S;
     int32_t s = (int32_t)(idx - o * S);
     int64_t i = ext2int[op0 + o];
-    out[idx] = (ov && kcl[i] != kNotSlowable) ? ov[lay.at(i, s)] : 0;  // only compute ops are tested
+    out[idx] = (ov && cand[i]) ? ov[lay.at(i, s)] : 0;  // only the candidates are tested
   }
 }
 
@@ -446,13 +438,6 @@ cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_copy_rows(const int32_t *rows, int64_t n_rows, int32_t S, MatLayout lay, const int64_t *src,
-                             int64_t *dst, cudaStream_t st) {
-  if (n_rows == 0 || S == 0) return cudaSuccess;
-  copy_rows_kernel<<<grid_for(n_rows * S, 256), 256, 0, st>>>(rows, n_rows, S, lay, src, dst);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
                             const int64_t *f, const int64_t *d, int64_t *start, int64_t *finish, cudaStream_t st) {
   int64_t n = (op1 - op0) * S;
@@ -470,10 +455,10 @@ cudaError_t launch_read_cc(const int32_t *ext2int, int64_t op0, int64_t op1, int
 }
 
 cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
-                           const uint8_t *ov, const uint8_t *kcl, uint8_t *out, cudaStream_t st) {
+                           const uint8_t *ov, const uint8_t *cand, uint8_t *out, cudaStream_t st) {
   int64_t n = (op1 - op0) * S;
   if (n <= 0) return cudaSuccess;
-  read_ov_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, lay, ov, kcl, out);
+  read_ov_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, lay, ov, cand, out);
   return cudaGetLastError();
 }
 

@@ -69,6 +69,7 @@ class GraphInfo(C.Structure):
     _fields_ = [("n_ops", C.c_int64), ("n_edges", C.c_int64), ("n_levels", C.c_int64),
                 ("max_width", C.c_int64), ("n_queue_entries", C.c_int64), ("n_comm_ops", C.c_int64),
                 ("n_signatures", C.c_int64), ("n_segments", C.c_int64), ("n_segment_levels", C.c_int64),
+                ("n_overlap_candidates", C.c_int64),
                 ("n_ranks", C.c_int32), ("n_streams", C.c_int32), ("sigma", C.c_int32)]
 
 
