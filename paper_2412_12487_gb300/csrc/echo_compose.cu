@@ -172,16 +172,31 @@ template <int SIGMA, int LANES>
 __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t ro, uint32_t i0, uint32_t seg0,
                                                  int32_t nseg, int sub, int step, int j0, int64_t *vr,
                                                  const int64_t *dr, const uint32_t *rr, uint32_t vmask,
-                                                 uint32_t dmask, uint32_t rmask, int64_t (&mk)[LANES]) {
+                                                 uint32_t dmask, uint32_t rmask, int64_t (&mk)[LANES],
+                                                 const int64_t *cr = nullptr, uint32_t cmask = 0) {
   int64_t *fb = a.f + ((int64_t)blockIdx.x * a.n_rows) * SIGMA;
   const uint32_t vr_a = saddr(vr) + j0 * 8, dr_a = saddr(dr) + j0 * 8;
   const uint32_t rr_a = saddr(rr);
+  const uint32_t cr_a = cr ? saddr(cr) + j0 * 8 : 0;
   constexpr uint32_t kRowBytes = SIGMA * 8;
   auto word = [&](uint32_t w) { return s_ld32(rr_a + (w & rmask) * 4); };
   for (int32_t k = sub; k < nseg; k += step) {
     const uint4 hd = s_ld128(rr_a + ((ro + 4 * k) & rmask) * 4);
     const uint32_t nin = hd.y & 0xFFFFu, nfar = hd.y >> 16;
-    const uint32_t len = hd.w;
+    const uint32_t len = hd.w & 0xFFFFu;
+    // chain positions whose duration the validator rewrote (second and later passes)
+    uint64_t cmask_bits = 0;
+    uint32_t c_first = 0;
+    if (cr && (hd.w >> 16)) {
+      const uint32_t ec = ro + hd.x + nin + nfar;
+      cmask_bits = (uint64_t)word(ec) | ((uint64_t)word(ec + 1) << 32);
+      c_first = word(ec + 2);
+    }
+    // a candidate's duration comes from the candidate ring instead of the duration ring
+    auto patch = [&](uint32_t t, int64_t (&d)[LANES]) {
+      if ((cmask_bits >> t) & 1)
+        s_load<LANES>(cr_a + ((c_first + (uint32_t)__popcll(cmask_bits & ((1ull << t) - 1))) & cmask) * kRowBytes, d);
+    };
     const uint32_t e = ro + hd.x;
     const uint32_t first = i0 + hd.z;
     int64_t fv[LANES];
@@ -213,6 +228,12 @@ __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t r
       s_load<LANES>(dr_a + ((first + t + 1) & dmask) * kRowBytes, d1);
       s_load<LANES>(dr_a + ((first + t + 2) & dmask) * kRowBytes, d2);
       s_load<LANES>(dr_a + ((first + t + 3) & dmask) * kRowBytes, d3);
+      if (cmask_bits) {
+        patch(t, d0);
+        patch(t + 1, d1);
+        patch(t + 2, d2);
+        patch(t + 3, d3);
+      }
 #pragma unroll
       for (int j = 0; j < LANES; ++j) fv[j] += d0[j];
       g_store<LANES>(gp, fv);
@@ -229,6 +250,7 @@ __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t r
     for (; t < len; ++t, gp += SIGMA) {
       int64_t d[LANES];
       s_load<LANES>(dr_a + ((first + t) & dmask) * kRowBytes, d);
+      if (cmask_bits) patch(t, d);
 #pragma unroll
       for (int j = 0; j < LANES; ++j) fv[j] += d[j];
       g_store<LANES>(gp, fv);
@@ -258,7 +280,7 @@ compose_staged_kernel(StagedArgs a) {
   const int32_t S = a.S;
   const int32_t s0 = blockIdx.x * SIGMA;
   const int tid = threadIdx.x;
-  const StagedLayout lay = staged_layout(SIGMA, a.vlog2, a.dlog2, a.rlog2);
+  const StagedLayout lay = staged_layout(SIGMA, a.vlog2, a.dlog2, a.rlog2, a.clog2);
   const uint32_t vmask = (1u << a.vlog2) - 1, dmask = (1u << a.dlog2) - 1, rmask = (1u << a.rlog2) - 1;
   const uint32_t RR = dmask + 1, RB = rmask + 1;
   int64_t *mk_s = reinterpret_cast<int64_t *>(sbuf);                  // [SIGMA]
@@ -412,17 +434,18 @@ compose_pipelined_kernel(StagedArgs a) {
   const int32_t S = a.S;
   const int32_t s0 = blockIdx.x * SIGMA;
   const int tid = threadIdx.x;
-  const StagedLayout lay = staged_layout(SIGMA, a.vlog2, a.dlog2, a.rlog2);
+  const StagedLayout lay = staged_layout(SIGMA, a.vlog2, a.dlog2, a.rlog2, a.clog2);
   const uint32_t vmask = (1u << a.vlog2) - 1, dmask = (1u << a.dlog2) - 1, rmask = (1u << a.rlog2) - 1;
-  const uint32_t RR = dmask + 1, RB = rmask + 1;
+  const uint32_t RR = dmask + 1, RB = rmask + 1, CRR = 1u << a.clog2;
   int64_t *mk_s = reinterpret_cast<int64_t *>(sbuf);                       // [SIGMA]
   uint64_t *full = reinterpret_cast<uint64_t *>(sbuf + lay.meta);          // [NB]
   uint64_t *empty = full + NB;                                              // [NB]
-  uint32_t *hist = reinterpret_cast<uint32_t *>(sbuf + lay.meta + 256);    // [NB][2] producer only
-  uint32_t *metas = reinterpret_cast<uint32_t *>(sbuf + lay.meta + 384);   // [NB][8]
+  uint32_t *hist = reinterpret_cast<uint32_t *>(sbuf + lay.meta + 256);    // [NB][4] producer only
+  uint32_t *metas = reinterpret_cast<uint32_t *>(sbuf + lay.meta + 512);   // [NB][8]
   int64_t *vr = reinterpret_cast<int64_t *>(sbuf + lay.vr);
   int64_t *dr = reinterpret_cast<int64_t *>(sbuf + lay.dr);
   uint32_t *rr = reinterpret_cast<uint32_t *>(sbuf + lay.rr);
+  int64_t *cr = reinterpret_cast<int64_t *>(sbuf + lay.cr);
 
   if (tid < SIGMA) mk_s[tid] = 0;
   if (tid == 0) {
@@ -440,7 +463,8 @@ compose_pipelined_kernel(StagedArgs a) {
     const int lane = tid - NCT;
     if (lane == 0) {
       const int64_t *durb = a.dur + ((int64_t)blockIdx.x * a.n_rows) * SIGMA;
-      const uint32_t emask = RR * SIGMA - 1;
+      const int64_t *cdb = a.cdur ? a.cdur + ((int64_t)blockIdx.x * a.n_cand) * SIGMA : nullptr;
+      const uint32_t emask = RR * SIGMA - 1, cemask = CRR * SIGMA - 1;
       int32_t c_known = 0;  // every level < c_known has been composed
       int32_t issued = 0;   // levels [0, issued) have been armed
       bool fail = false;
@@ -449,9 +473,10 @@ compose_pipelined_kernel(StagedArgs a) {
         const uint4 m0 = *reinterpret_cast<const uint4 *>(a.meta + 4 * l);
         const uint4 m1 = *reinterpret_cast<const uint4 *>(a.meta + 4 * (l + 1));
         const uint32_t ro = m0.x, i0 = m0.y, ro1 = m1.x, i1 = m1.y;
+        const uint32_t c0 = cdb ? m0.w : 0, c1 = cdb ? m1.w : 0;  // the level's candidate rows
         // ring space: level l overwrites rows and words of levels below c_known only
-        while (c_known < l && (l - c_known >= NB || i1 > hist[2 * (c_known % NB)] + RR ||
-                               ro1 > hist[2 * (c_known % NB) + 1] + RB)) {
+        while (c_known < l && (l - c_known >= NB || i1 > hist[4 * (c_known % NB)] + RR ||
+                               ro1 > hist[4 * (c_known % NB) + 1] + RB || c1 > hist[4 * (c_known % NB) + 2] + CRR)) {
           if (!mbar_wait(&empty[c_known % NB], (c_known / NB) & 1, a.wait_limit_cycles)) {
             fail = true;
             break;
@@ -459,11 +484,18 @@ compose_pipelined_kernel(StagedArgs a) {
           ++c_known;
         }
         if (fail) break;
-        hist[2 * (l % NB)] = i0;
-        hist[2 * (l % NB) + 1] = ro;
+        hist[4 * (l % NB)] = i0;
+        hist[4 * (l % NB) + 1] = ro;
+        hist[4 * (l % NB) + 2] = c0;
         uint64_t *bar = &full[l % NB];
         const uint32_t e0 = i0 * SIGMA, ne = (i1 - i0) * SIGMA, w0 = ro & rmask, nw = ro1 - ro;
-        mbar_arrive_expect_tx(bar, ne * 8 + nw * 4 + 32);
+        const uint32_t ce0 = c0 * SIGMA, nce = (c1 - c0) * SIGMA;
+        mbar_arrive_expect_tx(bar, ne * 8 + nw * 4 + 32 + nce * 8);
+        if (nce) {
+          const uint32_t nce1 = min(nce, cemask + 1 - (ce0 & cemask));
+          bulk_g2s(cr + (ce0 & cemask), cdb + ce0, nce1 * 8, bar);
+          if (nce1 < nce) bulk_g2s(cr, cdb + ce0 + nce1, (nce - nce1) * 8, bar);
+        }
         const uint32_t ne1 = min(ne, emask + 1 - (e0 & emask));
         bulk_g2s(dr + (e0 & emask), durb + e0, ne1 * 8, bar);
         if (ne1 < ne) bulk_g2s(dr, durb + e0 + ne1, (ne - ne1) * 8, bar);
@@ -490,7 +522,7 @@ compose_pipelined_kernel(StagedArgs a) {
         const uint32_t ro = mb[0], i0 = mb[1], seg0 = mb[2];
         const int32_t nseg = (int32_t)(mb[4 + 2] - seg0);
         compose_segments<SIGMA, LANES>(a, ro, i0, seg0, nseg, tid / TPN, NCT / TPN, j0, vr, dr, rr, vmask, dmask,
-                                       rmask, mk);
+                                       rmask, mk, a.cdur ? cr : nullptr, CRR - 1);
       }
       // every consumer learns, in the same barrier, whether any of them gave up
       if (named_barrier_or(1, NCT, !ok)) {

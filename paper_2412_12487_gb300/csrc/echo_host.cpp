@@ -64,6 +64,11 @@ struct GraphBuild {
   std::vector<int64_t> cand_off;      // [R+1] overlap candidates of each rank (compute ops, issue order)
   std::vector<int32_t> cand_ops;      // (internal ids)
   std::vector<uint8_t> cand_flag;     // [V] 1 for an overlap candidate
+  int64_t n_cand = 0;                 // overlap candidates
+  std::vector<int32_t> cidx;          // [V] level-order index of a candidate (by internal id), -1 otherwise
+  std::vector<int32_t> cand_cidx;     // level-order index of each entry of cand_ops
+  std::vector<int64_t> cand_lvl;      // [Ls+1] first level-order candidate index of each segment level
+  std::vector<int32_t> cand_node;     // internal id of each candidate, in level order
   std::vector<int64_t> ov_chunks;     // (rank, first candidate index) of the overlap test's chunks
   int32_t n_cq = 0;                   // comm timelines per rank in cq_off (max over ranks)
   std::vector<int64_t> cq_off;        // [R*n_cq+1] comm ops of each (rank, comm timeline)
@@ -162,7 +167,30 @@ void overlap_candidates(GraphBuild &b) {
     b.cand_off[r + 1] = (int64_t)b.cand_ops.size();
     for (int64_t j = 0; j < m; ++j) loc[nodes[j]] = -1;
   }
+  // level order of the candidates (by internal id): each segment level's candidates
+  // are then one contiguous range, and so are each segment's
+  b.n_cand = b.cand_off[R];
+  b.cidx.assign(V, -1);
+  b.cand_node.clear();
+  for (int64_t v = 0; v < V; ++v)
+    if (b.cand_flag[v]) {
+      b.cidx[v] = (int32_t)b.cand_node.size();
+      b.cand_node.push_back((int32_t)v);
+    }
+  if (b.cand_node.empty()) b.cand_node.push_back(0);
+  b.cand_cidx.resize(b.cand_ops.size());
+  for (size_t k = 0; k < b.cand_ops.size(); ++k) b.cand_cidx[k] = b.n_cand ? b.cidx[b.cand_ops[k]] : 0;
+  b.cand_lvl.assign(b.Ls + 1, 0);
+  {
+    int64_t k = 0;
+    for (int64_t l = 0; l < b.Ls; ++l) {
+      b.cand_lvl[l] = k;
+      for (int64_t v = b.seg_node_off[b.seg_lvl_off[l]]; v < b.seg_node_off[b.seg_lvl_off[l + 1]]; ++v) k += b.cand_flag[v];
+    }
+    b.cand_lvl[b.Ls] = k;
+  }
   if (b.cand_ops.empty()) b.cand_ops.push_back(0);
+  if (b.cand_cidx.empty()) b.cand_cidx.push_back(0);
 }
 
 int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
@@ -562,7 +590,9 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
     for (int64_t t = b.seg_lvl_off[l]; t < b.seg_lvl_off[l + 1]; ++t) {
       const int64_t nin = b.hin_off[t + 1] - b.hin_off[t];
       if (nin > 0xFFFF) b.stageable = false;
-      w += 4 + nin;
+      bool cand = false;
+      for (int64_t v = b.seg_node_off[t]; v < b.seg_node_off[t + 1]; ++v) cand = cand || b.cand_flag[v];
+      w += 4 + nin + (cand ? 3 : 0);
     }
     b.blk_words[l] = (w + 3) & ~(int64_t)3;
   }
@@ -582,9 +612,12 @@ echo::StagedPlan plan_staged(const GraphBuild &b, int sigma, size_t smem_cap) {
     while (((int64_t)1 << k) < x) ++k;
     return k;
   };
-  int64_t rows2 = 0, words2 = 0, segmax = 0, prow = 0, pword = 0;
+  int64_t rows2 = 0, words2 = 0, segmax = 0, prow = 0, pword = 0, crows2 = 0, pcand = 0;
   for (int64_t l = 0; l < b.Ls; ++l) {
     const int64_t r = b.seg_node_off[b.seg_lvl_off[l + 1]] - b.seg_node_off[b.seg_lvl_off[l]];
+    const int64_t nc = b.cand_lvl[l + 1] - b.cand_lvl[l];
+    crows2 = std::max(crows2, nc + pcand);
+    pcand = nc;
     rows2 = std::max(rows2, r + prow);
     words2 = std::max(words2, b.blk_words[l] + pword);
     segmax = std::max(segmax, b.seg_lvl_off[l + 1] - b.seg_lvl_off[l]);
@@ -592,16 +625,18 @@ echo::StagedPlan plan_staged(const GraphBuild &b, int sigma, size_t smem_cap) {
     pword = b.blk_words[l];
   }
   const int dmin = std::max(pow2(rows2), 4), rmin = std::max(pow2(words2), 4);
+  const int cring = std::max(pow2(crows2), 4);  // candidate ring: two levels' candidates
   const int vwant = std::min(std::max(pow2(4 * segmax), 6), 12);
   for (int d = dmin + 2; d >= dmin; --d)
     for (int v = vwant; v >= 6; --v)
       for (int r = rmin + 1; r >= rmin; --r) {
-        const size_t need = echo::staged_layout(sigma, v, d, r).total;
-        if (need <= smem_cap && d < 31 && r < 31) {
+        const size_t need = echo::staged_layout(sigma, v, d, r, cring).total;
+        if (need <= smem_cap && d < 31 && r < 31 && cring < 31) {
           best.ok = true;
           best.dring_log2 = d;
           best.vring_log2 = v;
           best.rring_log2 = r;
+          best.cring_log2 = cring;
           best.smem = need;
           return best;
         }
@@ -627,6 +662,7 @@ void build_records(const GraphBuild &b, int sigma, int vlog2, std::vector<uint32
     meta[4 * l] = (uint32_t)base;
     meta[4 * l + 1] = (uint32_t)i0;
     meta[4 * l + 2] = (uint32_t)s0;
+    meta[4 * l + 3] = (uint32_t)b.cand_lvl[l];
     recs.resize(base + 4 * (s1 - s0), 0);
     for (int64_t t = s0; t < s1; ++t) {
       const int64_t h = b.seg_node_off[t], z = b.seg_node_off[t + 1] - 1;
@@ -649,12 +685,28 @@ void build_records(const GraphBuild &b, int sigma, int vlog2, std::vector<uint32
       }
       recs.insert(recs.end(), far.begin(), far.end());
       recs[hd + 1] = nin | ((uint32_t)far.size() << 16);
+      // chain nodes that are overlap candidates: a 64-bit mask over the chain and the
+      // level-order index of the first of them
+      uint64_t mask = 0;
+      int64_t c_first = -1;
+      for (int64_t v = h; v <= z; ++v)
+        if (b.cand_flag[v]) {
+          mask |= 1ull << (v - h);
+          if (c_first < 0) c_first = b.cidx[v];
+        }
+      if (mask) {
+        recs[hd + 3] |= 1u << 16;
+        recs.push_back((uint32_t)mask);
+        recs.push_back((uint32_t)(mask >> 32));
+        recs.push_back((uint32_t)c_first);
+      }
     }
     while (recs.size() % 4) recs.push_back(0);
   }
   meta[4 * b.Ls] = (uint32_t)recs.size();
   meta[4 * b.Ls + 1] = (uint32_t)b.V;
   meta[4 * b.Ls + 2] = (uint32_t)b.n_seg;
+  meta[4 * b.Ls + 3] = (uint32_t)b.cand_lvl[b.Ls];
   if (recs.empty()) recs.assign(4, 0);
 }
 
@@ -698,14 +750,18 @@ struct echo_ctx {
   std::vector<uint64_t> h_sfx;
   int64_t *raw = nullptr, *dur = nullptr, *f[2] = {nullptr, nullptr}, *mk = nullptr, *cc_dur = nullptr;
   int64_t *gfrontier = nullptr;
-  int64_t *deff[2] = {nullptr, nullptr};  // durations of the validator's passes
+  int64_t *deff = nullptr;                // full validator durations, for kernels without a candidate ring
+  int64_t *cd[2] = {nullptr, nullptr};    // candidates' durations of the validator's passes (compact)
+  echo::MatLayout lay_c{0, 0};            // [n_cand][S] compact layout
+  size_t cd_elems = 0;                    // elements of each compact matrix
+  int32_t *cand_cidx = nullptr, *cidx = nullptr, *cand_node = nullptr;
   uint8_t *ov = nullptr;
   uint32_t *d_recs = nullptr, *d_meta = nullptr;
   echo::StagedPlan plan;
   uint32_t rec_words = 0;
   std::vector<double> h_sums, h_maxsf;
   int final_f = 0;
-  const int64_t *final_d = nullptr;
+  const int64_t *final_cd = nullptr;  // candidates' durations of the last composition (null: the original)
   bool have_ov = false;
   echo::OverlapArgs last_ov{};  // inputs of the last validator pass (to recompute its decisions)
   int kernel_choice = 0;            // 0 automatic, 1 direct, 2 staged, 3 pipelined (tuning and tests)
@@ -980,7 +1036,8 @@ int echo_load_graph(echo_ctx *c, const echo_graph_desc *g) {
       (rc = upload(c, o, &c->ov_chunks, B.ov_chunks)) ||
       (rc = upload(c, o, &c->cq_off, B.cq_off)) || (rc = upload(c, o, &c->cq_ops, B.cq_ops)) ||
       (rc = upload(c, o, &c->cand_off, B.cand_off)) || (rc = upload(c, o, &c->cand_ops, B.cand_ops)) ||
-      (rc = upload(c, o, &c->cand_flag, B.cand_flag)) ||
+      (rc = upload(c, o, &c->cand_flag, B.cand_flag)) || (rc = upload(c, o, &c->cand_cidx, B.cand_cidx)) ||
+      (rc = upload(c, o, &c->cidx, B.cidx)) || (rc = upload(c, o, &c->cand_node, B.cand_node)) ||
       (rc = upload(c, o, &c->nq_off, B.nq_off)) ||
       (rc = upload(c, o, &c->nq, B.nq)) || (rc = upload(c, o, &c->dp_off, B.dp_off)) ||
       (rc = upload(c, o, &c->dp, B.dp)) || (rc = upload(c, o, &c->q_off, B.q_off)) ||
@@ -1039,11 +1096,12 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     bool in_smem = true;
     echo::compose_smem_bytes(B.R * B.NS, sigma, &in_smem);
     int64_t nblk = (S + sigma - 1) / sigma;
+    const size_t CS = (size_t)std::max<int64_t>(B.n_cand, 1) * (size_t)nblk * sigma;  // compact matrices
     if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sfx, (size_t)C * S)) ||
         (rc = dalloc(c, o, &c->sums, (size_t)S)) || (rc = dalloc(c, o, &c->comm_sum, (size_t)S)) ||
         (rc = dalloc(c, o, &c->raw, (size_t)V * S)) || (rc = dalloc(c, o, &c->dur, VS)) ||
         (rc = dalloc(c, o, &c->f[0], VS)) || (rc = dalloc(c, o, &c->f[1], VS)) ||
-        (rc = dalloc(c, o, &c->deff[0], VS)) || (rc = dalloc(c, o, &c->ov, VS)) ||
+        (rc = dalloc(c, o, &c->cd[0], CS)) || (rc = dalloc(c, o, &c->ov, VS)) ||
         (rc = dalloc(c, o, &c->mk, (size_t)S)) || (rc = dalloc(c, o, &c->cc_ns, (size_t)G * S)) ||
         (rc = dalloc(c, o, &c->cc_dur, (size_t)G * S)) ||
         (!in_smem && (rc = dalloc(c, o, &c->gfrontier, (size_t)nblk * B.R * B.NS * sigma)))) {
@@ -1053,8 +1111,9 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     if (in_smem) c->gfrontier = nullptr;
     // padding lanes of the duration matrices stay zero
     CK(cudaMemsetAsync(c->dur, 0, VS * sizeof(int64_t), c->stream), "memset");
-    CK(cudaMemsetAsync(c->deff[0], 0, VS * sizeof(int64_t), c->stream), "memset");
-    c->deff[1] = nullptr;  // second validator buffer: allocated when refine_passes > 1
+    CK(cudaMemsetAsync(c->cd[0], 0, CS * sizeof(int64_t), c->stream), "memset");
+    c->cd[1] = nullptr;   // second compact buffer: allocated when refine_passes > 1
+    c->deff = nullptr;    // allocated when a kernel without a candidate ring composes a second pass
     // launch shape of the staged kernels (threads and blocks per SM may be overridden
     // for tuning: ECHO_STAGED_THREADS, ECHO_BLOCKS_PER_SM)
     int optin = 0, per_sm = 0;
@@ -1073,7 +1132,8 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
       int64_t max_bytes = 0;
       for (int64_t l = 0; l < B.Ls; ++l) {
         const int64_t rows = B.seg_node_off[B.seg_lvl_off[l + 1]] - B.seg_node_off[B.seg_lvl_off[l]];
-        max_bytes = std::max(max_bytes, rows * sigma * 8 + B.blk_words[l] * 4 + 32);
+        max_bytes = std::max(max_bytes, rows * sigma * 8 + B.blk_words[l] * 4 + 32 +
+                                            (B.cand_lvl[l + 1] - B.cand_lvl[l]) * sigma * 8);
       }
       c->plan.pipelined = sigma % 2 == 0 && max_bytes < (1 << 20);
       std::vector<uint32_t> recs, meta;
@@ -1089,6 +1149,8 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     c->C = C;
     c->sigma = sigma;
     c->lay = echo::MatLayout{V, slog2};
+    c->lay_c = echo::MatLayout{B.n_cand, slog2};
+    c->cd_elems = CS;
   }
   c->tbl = tbl;
   c->h_maxsf = maxsf;
@@ -1166,13 +1228,20 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   int32_t refine = opts ? opts->refine_passes : 1;
   if (refine < 0 || refine > 8) return set_err(c, ECHO_E_INVALID_ARG, "refine_passes outside [0, 8]");
   const GraphBuild &B = c->gb;
-  if (refine > 1 && !c->deff[1]) {
-    if ((rc = dalloc(c, c->scen_allocs, &c->deff[1], c->scen_vs))) return rc;
-    CK(cudaMemsetAsync(c->deff[1], 0, c->scen_vs * sizeof(int64_t), c->stream), "memset");
+  // the pipelined kernel reads the validator's durations of the candidates from a
+  // ring of its own; the others compose from a full matrix built for them
+  const bool ring = c->plan.ok && c->plan.pipelined && (c->kernel_choice == 0 || c->kernel_choice == 3);
+  if (refine > 1 && !c->cd[1]) {
+    if ((rc = dalloc(c, c->scen_allocs, &c->cd[1], c->cd_elems))) return rc;
+    CK(cudaMemsetAsync(c->cd[1], 0, c->cd_elems * sizeof(int64_t), c->stream), "memset");
+  }
+  if (refine > 0 && !ring && !c->deff) {
+    if ((rc = dalloc(c, c->scen_allocs, &c->deff, c->scen_vs))) return rc;
   }
   c->state = 3;
-  // one composition with durations `d` into `f`
-  auto compose_pass = [&](const int64_t *d, int64_t *f) -> cudaError_t {
+  // one composition with durations `d` (and, for the pipelined kernel, the
+  // candidates' durations `cdur`) into `f`
+  auto compose_pass = [&](const int64_t *d, const int64_t *cdur, int64_t *f) -> cudaError_t {
     if (c->plan.ok && c->kernel_choice != 1) {
       echo::StagedArgs a{};
       a.S = c->S;
@@ -1182,9 +1251,12 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       a.vlog2 = c->plan.vring_log2;
       a.dlog2 = c->plan.dring_log2;
       a.rlog2 = c->plan.rring_log2;
+      a.clog2 = c->plan.cring_log2;
       a.meta = c->d_meta;
       a.recs = c->d_recs;
       a.dur = d;
+      a.cdur = cdur;
+      a.n_cand = (uint32_t)B.n_cand;
       a.f = f;
       a.makespan = c->mk;
       a.status = c->status;
@@ -1214,38 +1286,46 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     return timed(c, "compose_direct", [&] { return echo::launch_compose(a, c->sigma, c->stream); });
   };
   CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
-  CK(compose_pass(c->dur, c->f[0]), "compose launch");
-  const int64_t *d_used = c->dur;
+  CK(compose_pass(c->dur, nullptr, c->f[0]), "compose launch");
+  const int64_t *cd_used = nullptr;
   for (int32_t p = 1; p <= refine; ++p) {
     echo::OverlapArgs o{};
     o.lay = c->lay;
+    o.lay_c = c->lay_c;
     o.S = c->S;
     o.n_streams = B.NS;
     o.n_chunks = (int64_t)B.ov_chunks.size() / 2;
     o.chunks = c->ov_chunks;
     o.cand_off = c->cand_off;
     o.cand_ops = c->cand_ops;
+    o.cand_cidx = c->cand_cidx;
     o.n_cq = B.n_cq;
     o.cq_off = c->cq_off;
     o.cq_ops = c->cq_ops;
     o.kcl = c->kcl;
     o.f = c->f[(p - 1) % 2];
-    o.d_used = d_used;
-    o.d_orig = c->dur;
+    o.dur = c->dur;
+    o.cd_used = cd_used;
     o.sfx = c->sfx;
-    o.d_next = c->deff[(p - 1) % 2];
+    o.cd_next = c->cd[(p - 1) % 2];
     o.ov = nullptr;  // the decisions are recomputed on demand by echo_read_overlap
-    // ops that cannot overlap keep their durations; the test rewrites the candidates
-    CK(timed(c, "dur_copy", [&] {
-         return cudaMemcpyAsync(o.d_next, c->dur, c->scen_vs * sizeof(int64_t), cudaMemcpyDeviceToDevice, c->stream);
-       }), "duration copy");
     CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");
-    CK(compose_pass(o.d_next, c->f[p % 2]), "compose launch");
-    d_used = o.d_next;
+    if (ring) {
+      CK(compose_pass(c->dur, o.cd_next, c->f[p % 2]), "compose launch");
+    } else {
+      CK(cudaMemcpyAsync(c->deff, c->dur, c->scen_vs * sizeof(int64_t), cudaMemcpyDeviceToDevice, c->stream),
+         "duration copy");
+      CK(timed(c, "scatter_candidates", [&] {
+           return echo::launch_scatter_candidates(c->cand_node, B.n_cand, c->S, c->lay, c->lay_c, o.cd_next, c->deff,
+                                                  c->stream);
+         }), "scatter launch");
+      CK(compose_pass(c->deff, nullptr, c->f[p % 2]), "compose launch");
+    }
+    cd_used = o.cd_next;
     c->last_ov = o;
   }
   c->final_f = refine % 2;
-  c->final_d = d_used;
+  c->final_cd = cd_used;
   c->have_ov = refine > 0;
   c->state = 4;
   return ECHO_OK;
@@ -1281,7 +1361,8 @@ int echo_read_times(echo_ctx *c, int64_t op0, int64_t op1, int64_t *start, int64
     int64_t *ds = static_cast<int64_t *>(c->stage);
     int64_t *df = ds + n;
     CK(timed(c, "readback", [&] {
-         return echo::launch_readback(c->ext2int, a, b, S, c->lay, c->f[c->final_f], c->final_d,
+         return echo::launch_readback(c->ext2int, a, b, S, c->lay, c->f[c->final_f], c->dur, c->cidx, c->lay_c,
+                                      c->final_cd,
                                       start ? ds : nullptr, finish ? df : nullptr, c->stream);
        }), "readback launch");
     if (start) CK(cudaMemcpyAsync(start + (a - op0) * S, ds, n * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream), "D2H");
@@ -1339,7 +1420,7 @@ int echo_read_overlap(echo_ctx *c, int64_t op0, int64_t op1, uint8_t *out) {
     // the last pass's inputs (its finish times and durations) are still intact:
     // run its overlap test again, keeping only the decisions
     echo::OverlapArgs o = c->last_ov;
-    o.d_next = nullptr;
+    o.cd_next = nullptr;
     o.ov = c->ov;
     CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");
     ov = c->ov;

@@ -77,17 +77,24 @@ struct ComposeArgs {
 // nin | nfar << 16, first node - level's first node, length}; entries = the
 // head's nin inputs held in the value ring (byte offsets of their slots), then its
 // nfar inputs too old for the ring (node ids, read from global memory).  Every
-// input is the tail of an earlier segment.  Blocks are padded to 4 words.
+// input is the tail of an earlier segment.  A segment whose chain holds overlap
+// candidates has bit 16 of its length word set and 3 more entries: a 64-bit mask
+// of those chain positions and the level-order index of the first.  Blocks are
+// padded to 4 words.  Metadata of a level: record word offset, first node, first
+// segment, first level-order candidate.
 struct StagedArgs {
   int32_t S, L;                  // L: segment levels
   uint32_t n_rows, n_words;      // nodes; words of all record blocks
   int32_t vlog2, dlog2, rlog2;   // log2 sizes: value ring (segments), duration ring (rows), record ring (words)
-  const uint32_t *meta;          // [4*(L+1)]: record word offset, first node, first segment, 0
+  const uint32_t *meta;          // [4*(L+1)]: record word offset, first node, first segment, first candidate
   const uint32_t *recs;          // record blocks
   const int64_t *dur;            // durations (MatLayout)
   int64_t *f;                    // finish times (MatLayout, out)
   int64_t *makespan;             // [S] (out)
   // pipelined kernel only
+  const int64_t *cdur;           // validator durations of the candidates ([n_cand] rows per block), or null
+  uint32_t n_cand;               // overlap candidates
+  int32_t clog2;                 // log2 rows of the candidate ring
   int32_t *status;               // device status word (kDevTimeout when a bounded wait gives up)
   long long wait_limit_cycles;   // bound of every mbarrier wait, in SM clock cycles
   int32_t skip_level;            // failure injection for tests: this level is never filled (-1: none)
@@ -99,43 +106,47 @@ struct StagedPlan {
   bool pipelined = false;  // bulk-copy producer warp (even sigma)
   int threads = 512;       // threads per block of the staged kernel
   int vring_log2 = 0, dring_log2 = 0, rring_log2 = 0;  // sizes (segments, rows, words)
+  int cring_log2 = 0;  // candidate ring (rows of the validator's durations, pipelined kernel)
   size_t smem = 0;
 };
 
 // Shared-memory layout of the staged kernels (byte offsets).  Every region starts
 // on a 16-byte boundary, as 16-byte copy destinations require.
 struct StagedLayout {
-  size_t hist, meta, vr, dr, rr, total;
+  size_t hist, meta, vr, dr, rr, cr, total;
 };
 __host__ __device__ inline size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
-__host__ __device__ inline StagedLayout staged_layout(int sigma, int vlog2, int dlog2, int rlog2) {
+__host__ __device__ inline StagedLayout staged_layout(int sigma, int vlog2, int dlog2, int rlog2, int clog2) {
   StagedLayout L;
   L.hist = 128;                        // [0, 128): per-scenario makespans
   L.meta = L.hist + 16 * 8;            // 16 copy-group extents
   L.vr = L.meta + round16((size_t)2 * kMetaCap * 16);
   L.dr = L.vr + round16(((size_t)1 << vlog2) * sigma * 8);
   L.rr = L.dr + round16(((size_t)1 << dlog2) * sigma * 8);
-  L.total = L.rr + round16(((size_t)1 << rlog2) * 4);
+  L.cr = L.rr + round16(((size_t)1 << rlog2) * 4);
+  L.total = L.cr + round16(((size_t)1 << clog2) * sigma * 8);
   return L;
 }
 
 // Validator: for each overlap candidate (a compute op), whether its interval
 // overlaps a comm op of its rank, and the duration to use in the next composition.
 struct OverlapArgs {
-  MatLayout lay;
+  MatLayout lay;           // [V][S] matrices
+  MatLayout lay_c;         // [n_cand][S] compact matrices (rows in level order)
   int32_t S, n_streams;
   int32_t n_cq;            // comm timelines per rank (lists of a rank with fewer are empty)
   int64_t n_chunks;
   const int64_t *chunks;   // [n_chunks][2]: (rank, first candidate index)
   const int64_t *cand_off; const int32_t *cand_ops;  // [R+1]: each rank's overlap candidates, in issue order
+  const int32_t *cand_cidx;                          // level-order index of each entry of cand_ops
   const int64_t *cq_off; const int32_t *cq_ops;  // [R*n_cq+1]: comm ops of each (rank, comm timeline)
   const uint8_t *kcl;      // [V]
   const int64_t *f;        // finish times of the last pass
-  const int64_t *d_used;   // durations of the last pass
-  const int64_t *d_orig;   // durations before any slowdown
+  const int64_t *dur;      // original durations
+  const int64_t *cd_used;  // candidates' durations in the last pass (compact), or null: the original ones
   const uint64_t *sfx;     // [C][S] slowdown factors, packed as (53-bit significand << 11) | (exponent + 1075)
-  int64_t *d_next;         // (out, compute rows; may be null)
-  uint8_t *ov;             // (out, compute rows; may be null)
+  int64_t *cd_next;        // (out, compact; may be null) candidates' durations for the next pass
+  uint8_t *ov;             // (out, [V][S] rows of the candidates; may be null)
 };
 
 // kernels.cu
@@ -155,8 +166,10 @@ cudaError_t launch_compose_staged(const StagedArgs &a, int sigma, const StagedPl
 cudaError_t launch_compose_pipelined(const StagedArgs &a, int sigma, const StagedPlan &plan, cudaStream_t st);
 cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st);
 cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
-                            const int64_t *f, const int64_t *d, int64_t *start, int64_t *finish,
-                            cudaStream_t st);
+                            const int64_t *f, const int64_t *d, const int32_t *cidx, MatLayout lay_c,
+                            const int64_t *cd, int64_t *start, int64_t *finish, cudaStream_t st);
+cudaError_t launch_scatter_candidates(const int32_t *cand_node, int64_t n_cand, int32_t S, MatLayout lay,
+                                      MatLayout lay_c, const int64_t *cd, int64_t *dst, cudaStream_t st);
 cudaError_t launch_read_cc(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S,
                            const int32_t *node_sig, const double *cc_ns, double *out, cudaStream_t st);
 cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,

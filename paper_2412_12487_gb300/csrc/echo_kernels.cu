@@ -214,7 +214,7 @@ __global__ void permute_rows_kernel(const int64_t *__restrict__ raw, const int32
 // the cursor op ends).  A binary search places the cursors at the chunk's first
 // op; from there they only move forward, and only then touch memory.  A compute
 // op of positive length that overlaps gets rint(d * slowdown) for the next
-// composition (d_next), others keep d; the decisions themselves are stored only
+// composition (cd_next, compact), others keep d; the decisions themselves are stored only
 // when `ov` is given.  The finish times and durations of 8 consecutive ops are
 // loaded together before they are tested.
 // ---------------------------------------------------------------------------------
@@ -237,9 +237,14 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
   const int sh = a.lay.slog2;
   const int64_t base = a.lay.at(0, sl);
   const int64_t *__restrict__ f = a.f + base;
-  const int64_t *__restrict__ du = a.d_used + base;
-  const bool same = a.d_orig == a.d_used;
-  int32_t qreg = c0 + lane < c1 ? a.cand_ops[c0 + lane] : 0;  // ops c0 .. c0+31 of the chunk
+  const int64_t *__restrict__ du = a.dur + base;  // comm ops' durations (never slowed)
+  // the candidates' durations in the pass that produced f: the original ones, or the
+  // previous validator pass's (compact [candidate][scenario] rows)
+  const int64_t *__restrict__ cu = a.cd_used ? a.cd_used + a.lay_c.at(0, sl) : nullptr;
+  int64_t *__restrict__ cn = a.cd_next ? a.cd_next + a.lay_c.at(0, sl) : nullptr;
+  int32_t qreg = c0 + lane < c1 ? a.cand_ops[c0 + lane] : 0;   // ops c0 .. c0+31 of the chunk
+  int32_t creg = c0 + lane < c1 ? a.cand_cidx[c0 + lane] : 0;  // and their level-order indices
+  auto cand_d = [&](int64_t v, int64_t ci) { return cu ? cu[ci << sh] : du[v << sh]; };
   // per comm timeline: position, end, and interval of the cursor op; the cursor op
   // always has positive length and finishes after the current op's start (or the
   // cursor is at the end, with an interval that never overlaps)
@@ -255,8 +260,8 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
     }
   };
   {
-    const int64_t v = __shfl_sync(0xffffffffu, qreg, 0);
-    const int64_t sv = act ? f[v << sh] - du[v << sh] : 0;
+    const int64_t v = __shfl_sync(0xffffffffu, qreg, 0), ci = __shfl_sync(0xffffffffu, creg, 0);
+    const int64_t sv = act ? f[v << sh] - cand_d(v, ci) : 0;
 #pragma unroll
     for (int j = 0; j < NCMAX; ++j) {
       cur[j] = end[j] = 0;
@@ -282,15 +287,19 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
   }
   // groups of kOverlapBatch ops: their finish times and durations are loaded together
   for (int64_t i0 = c0; i0 < c1; i0 += kOverlapBatch) {
-    if (i0 > c0 && ((i0 - c0) & 31) == 0) qreg = i0 + lane < c1 ? a.cand_ops[i0 + lane] : 0;
-    int64_t vb[kOverlapBatch], fb[kOverlapBatch], db[kOverlapBatch];
+    if (i0 > c0 && ((i0 - c0) & 31) == 0) {
+      qreg = i0 + lane < c1 ? a.cand_ops[i0 + lane] : 0;
+      creg = i0 + lane < c1 ? a.cand_cidx[i0 + lane] : 0;
+    }
+    int64_t vb[kOverlapBatch], cb[kOverlapBatch], fb[kOverlapBatch], db[kOverlapBatch];
 #pragma unroll
     for (int u = 0; u < kOverlapBatch; ++u) {
       vb[u] = __shfl_sync(0xffffffffu, qreg, (int)((i0 - c0 + u) & 31));
+      cb[u] = __shfl_sync(0xffffffffu, creg, (int)((i0 - c0 + u) & 31));
       fb[u] = db[u] = 0;
       if (act && i0 + u < c1) {
         fb[u] = f[vb[u] << sh];
-        db[u] = du[vb[u] << sh];
+        db[u] = cand_d(vb[u], cb[u]);
       }
     }
     if (!act) continue;
@@ -313,11 +322,10 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
           }
         }
         hit = hit && sv < fv;
-        const int64_t at = base + (v << sh);
-        if (a.ov) a.ov[at] = hit;
-        if (a.d_next) {
-          const int64_t d0 = same ? dv : a.d_orig[at];
-          a.d_next[at] = hit ? slowed(d0, a.sfx[(int64_t)a.kcl[v] * S + sl]) : d0;
+        if (a.ov) a.ov[base + (v << sh)] = hit;
+        if (cn) {
+          const int64_t d0 = cu ? du[v << sh] : dv;  // the original duration
+          cn[cb[u] << sh] = hit ? slowed(d0, a.sfx[(int64_t)a.kcl[v] * S + sl]) : d0;
         }
       }
     }
@@ -327,18 +335,39 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
 // ---------------------------------------------------------------------------------
 // readback: internal order and blocked layout -> caller order, [op][scenario]
 // ---------------------------------------------------------------------------------
+// start = finish - the duration the op had in the last composition: d, or for an
+// overlap candidate its row of the compact cd when given
 __global__ void readback_kernel(const int32_t *__restrict__ ext2int, int64_t op0, int64_t op1, int32_t S,
                                 MatLayout lay, const int64_t *__restrict__ f, const int64_t *__restrict__ d,
+                                const int32_t *__restrict__ cidx, MatLayout lay_c, const int64_t *__restrict__ cd,
                                 int64_t *__restrict__ start, int64_t *__restrict__ finish) {
   int64_t total = (op1 - op0) * S;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
        idx += (int64_t)gridDim.x * blockDim.x) {
     int64_t o = idx / S;
     int32_t s = (int32_t)(idx - o * S);
-    int64_t at = lay.at(ext2int[op0 + o], s);
+    const int32_t i = ext2int[op0 + o];
+    int64_t at = lay.at(i, s);
     int64_t fv = f[at];
-    if (start) start[idx] = fv - d[at];
+    if (start) {
+      const int32_t ci = cd ? cidx[i] : -1;
+      start[idx] = fv - (ci >= 0 ? cd[lay_c.at(ci, s)] : d[at]);
+    }
     if (finish) finish[idx] = fv;
+  }
+}
+
+// Full validator durations for the kernels without a candidate ring: the
+// candidates' rows of the compact cd into dst (which holds the original durations).
+__global__ void scatter_candidates_kernel(const int32_t *__restrict__ cand_node, int64_t n_cand, int32_t S,
+                                          MatLayout lay, MatLayout lay_c, const int64_t *__restrict__ cd,
+                                          int64_t *__restrict__ dst) {
+  const int64_t total = n_cand * S;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t k = idx / S;
+    const int32_t s = (int32_t)(idx - k * S);
+    dst[lay.at(cand_node[k], s)] = cd[lay_c.at(k, s)];
   }
 }
 
@@ -439,10 +468,19 @@ cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
 }
 
 cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
-                            const int64_t *f, const int64_t *d, int64_t *start, int64_t *finish, cudaStream_t st) {
+                            const int64_t *f, const int64_t *d, const int32_t *cidx, MatLayout lay_c,
+                            const int64_t *cd, int64_t *start, int64_t *finish, cudaStream_t st) {
   int64_t n = (op1 - op0) * S;
   if (n <= 0) return cudaSuccess;
-  readback_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, lay, f, d, start, finish);
+  readback_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, lay, f, d, cidx, lay_c, cd, start,
+                                                    finish);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scatter_candidates(const int32_t *cand_node, int64_t n_cand, int32_t S, MatLayout lay,
+                                      MatLayout lay_c, const int64_t *cd, int64_t *dst, cudaStream_t st) {
+  if (n_cand == 0 || S == 0) return cudaSuccess;
+  scatter_candidates_kernel<<<grid_for(n_cand * S, 256), 256, 0, st>>>(cand_node, n_cand, S, lay, lay_c, cd, dst);
   return cudaGetLastError();
 }
 
