@@ -60,6 +60,8 @@ enum { ECHO_OP_COMPUTE = 0, ECHO_OP_MEMCPY = 1, ECHO_OP_COLL = 2, ECHO_OP_P2P = 
 enum { ECHO_CC_ALLREDUCE = 0, ECHO_CC_ALLGATHER = 1, ECHO_CC_REDUCESCATTER = 2, ECHO_CC_SENDRECV = 3 };
 /* all-reduce algorithm (Sec. 5.1: NCCL runs ring or tree all-reduce; AUTO = the faster) */
 enum { ECHO_ALGO_RING = 0, ECHO_ALGO_TREE = 1, ECHO_ALGO_AUTO = 2 };
+/* collective cost models (echo_set_cc_model) */
+enum { ECHO_CC_MODEL_WHITEBOX = 0, ECHO_CC_MODEL_ALPHA_BETA = 1 };
 
 typedef struct echo_ctx echo_ctx;
 
@@ -162,6 +164,16 @@ int echo_load_scenarios(echo_ctx *ctx, const echo_scen_desc *sc);
  * largest member count on one node, log2(M) computed on the host.  A time that
  * could overflow the composition -> ECHO_E_OVERFLOW. */
 int echo_estimate_collectives(echo_ctx *ctx);
+
+/* Cost model of the next echo_estimate_collectives.  ECHO_CC_MODEL_WHITEBOX (the
+ * default) is Eqs. 2-5 above.  ECHO_CC_MODEL_ALPHA_BETA is the model Sec. 2.3
+ * describes for the simulators Echo is compared with (NCCL-Predictor, Sec. 8.3):
+ * message size over bandwidth plus latency, here on the group's bottleneck link
+ * (inter-node when the group spans nodes), 0 for N = 1 or 0 bytes, every
+ * collective type alike; comparing the two shows how the makespan depends on the
+ * estimator.  A context that had estimated must estimate again before composing.
+ * An unknown model -> ECHO_E_INVALID_ARG. */
+int echo_set_cc_model(echo_ctx *ctx, int model);
 
 /* Timeline composer (Sec. 4.2) over all scenarios, then `refine_passes` validator
  * passes (Sec. 3, 2.3): a compute op whose [start, finish) interval overlaps, with

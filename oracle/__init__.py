@@ -51,7 +51,7 @@ class _Scen(C.Structure):
                 ("dur", C.c_void_p), ("alpha_ns", C.c_void_p), ("bw_intra", C.c_void_p),
                 ("lat_intra", C.c_void_p), ("bw_inter", C.c_void_p), ("lat_inter", C.c_void_p),
                 ("delta", C.c_void_p), ("slowdown", C.c_void_p),
-                ("chunk_max_bytes", C.c_void_p), ("chunk_bytes", C.c_void_p)]
+                ("chunk_max_bytes", C.c_void_p), ("chunk_bytes", C.c_void_p), ("cc_model", C.c_int32)]
 
 
 def _load():
@@ -65,6 +65,8 @@ def _load():
             lib.oracle_cc_ns.restype = C.c_double
             lib.oracle_cc_ns.argtypes = [C.c_int, C.c_int, C.c_int64, C.c_int, C.c_int, C.c_int,
                                          C.c_double, C.c_void_p, C.c_int, C.c_void_p, C.c_void_p]
+            lib.oracle_cc_ns_alpha_beta.restype = C.c_double
+            lib.oracle_cc_ns_alpha_beta.argtypes = [C.c_int64, C.c_int, C.c_int, C.c_void_p]
             lib.oracle_compose.restype = C.c_int
             lib.oracle_compose.argtypes = [C.POINTER(_Graph), C.POINTER(_Scen), C.c_int32, C.c_int32,
                                            C.c_int32, C.c_uint64, C.c_void_p, C.c_void_p,
@@ -101,6 +103,13 @@ def cc_ns(cc_type: int, cc_algo: int, nbytes: int, N: int, M: int, K: int, lg: f
                                   _p(mx), _p(cb)))
 
 
+def cc_ns_alpha_beta(nbytes: int, N: int, M: int, alpha: float, bw_intra: float, lat_intra: float,
+                     bw_inter: float, lat_inter: float, delta: float) -> float:
+    lib = _load()
+    prm = np.array([alpha, bw_intra, lat_intra, bw_inter, lat_inter, delta], np.float64)
+    return float(lib.oracle_cc_ns_alpha_beta(int(nbytes), int(N), int(M), _p(prm)))
+
+
 class OracleResult:
     def __init__(self, start, finish, makespan, cc_ns, overlapped):
         self.start, self.finish, self.makespan = start, finish, makespan
@@ -108,8 +117,9 @@ class OracleResult:
 
 
 def compose(g, sc, refine_passes: int = 1, tie_seed: int = 0, threads: int = 1,
-            want_cc: bool = True, want_overlap: bool = True) -> OracleResult:
-    """Compose every scenario of ``sc`` on graph ``g`` (workloads.Graph/Scenarios)."""
+            want_cc: bool = True, want_overlap: bool = True, cc_model: int = 0) -> OracleResult:
+    """Compose every scenario of ``sc`` on graph ``g`` (workloads.Graph/Scenarios).
+    cc_model 0 takes collective times from Eqs. 2-5, 1 from the alpha-beta model."""
     lib = _load()
     V, S = g.n_ops, sc.n_scen
     keep = []
@@ -130,7 +140,7 @@ def compose(g, sc, refine_passes: int = 1, tie_seed: int = 0, threads: int = 1,
                arr(sc.bw_inter, np.float64), arr(sc.lat_inter, np.float64), arr(sc.delta, np.float64),
                arr(sc.slowdown, np.float64),
                arr(sc.chunk_max_bytes, np.int64) if n_chunk else None,
-               arr(sc.chunk_bytes, np.int64) if n_chunk else None)
+               arr(sc.chunk_bytes, np.int64) if n_chunk else None, int(cc_model))
     start = np.zeros((V, S), np.int64)
     finish = np.zeros((V, S), np.int64)
     mk = np.zeros(S, np.int64)

@@ -116,6 +116,17 @@ double oracle_cc_ns(int cc_type, int cc_algo, int64_t nbytes, int N, int M, int 
   return (t < r) ? t : r;
 }
 
+/* The alpha-beta model that Sec. 2.3 describes for the simulators Echo compares
+ * against (NCCL-Predictor, Sec. 8.3): a collective takes its message size over the
+ * bandwidth plus the latency.  Read here on the group's bottleneck link, the
+ * inter-node one when the group spans nodes; N = 1 or 0 bytes costs 0. */
+double oracle_cc_ns_alpha_beta(int64_t nbytes, int N, int M, const double *prm) {
+  if (N <= 1 || nbytes <= 0) return 0.0;
+  double L = (M > 1) ? prm[4] : prm[2];
+  double B = (M > 1) ? prm[3] : prm[1];
+  return L + (double)nbytes / B;
+}
+
 /* ------------------------------------------------------------------------------ */
 /* event-driven timeline composer (Sec. 4.2)                                      */
 /* ------------------------------------------------------------------------------ */
@@ -322,8 +333,10 @@ int oracle_compose(const oracle_graph *g, const oracle_scen *sc, int32_t s0, int
       uint8_t k = g->kind[v];
       if (k == K_COLL || k == K_P2P) {
         int32_t gi = g->group[v];
-        double T = oracle_cc_ns(g->cc_type[v], g->cc_algo[v], g->cc_bytes[v], gN[gi], gM[gi], gK[gi],
-                                glg[gi], prm, sc->n_chunk, sc->chunk_max_bytes, sc->chunk_bytes);
+        double T = sc->cc_model == 1
+                       ? oracle_cc_ns_alpha_beta(g->cc_bytes[v], gN[gi], gM[gi], prm)
+                       : oracle_cc_ns(g->cc_type[v], g->cc_algo[v], g->cc_bytes[v], gN[gi], gM[gi], gK[gi],
+                                      glg[gi], prm, sc->n_chunk, sc->chunk_max_bytes, sc->chunk_bytes);
         if (cc_ns) cc_ns[v * S + s] = T;
         d0[v] = llrint(T);
       } else {

@@ -32,6 +32,7 @@ typedef struct {
   const double *alpha_ns, *bw_intra, *lat_intra, *bw_inter, *lat_inter, *delta; /* [n_scen] */
   const double *slowdown;                                                      /* [n_kclass][n_scen] */
   const int64_t *chunk_max_bytes, *chunk_bytes; /* [n_chunk]; n_chunk = 0 -> Table 6 */
+  int32_t cc_model; /* 0: Eqs. 2-5 (white box), 1: alpha-beta */
 } oracle_scen;
 
 int64_t oracle_chunk_bytes(int64_t nbytes, int n_chunk, const int64_t *max_bytes,
@@ -41,6 +42,9 @@ int64_t oracle_chunk_bytes(int64_t nbytes, int n_chunk, const int64_t *max_bytes
 double oracle_cc_ns(int cc_type, int cc_algo, int64_t nbytes, int N, int M, int K, double lg,
                     const double *prm, int n_chunk, const int64_t *max_bytes,
                     const int64_t *chunk_bytes);
+
+/* prm as above; message size over bandwidth plus latency on the bottleneck link */
+double oracle_cc_ns_alpha_beta(int64_t nbytes, int N, int M, const double *prm);
 
 /* Composes scenarios [s0, s1).  Outputs are [n_ops][n_scen] (only the columns in
  * range are written); any output pointer may be NULL. */

@@ -765,6 +765,7 @@ struct echo_ctx {
   bool have_ov = false;
   echo::OverlapArgs last_ov{};  // inputs of the last validator pass (to recompute its decisions)
   int kernel_choice = 0;            // 0 automatic, 1 direct, 2 staged, 3 pipelined (tuning and tests)
+  int cc_model = ECHO_CC_MODEL_WHITEBOX;
   long long wait_limit_cycles = 0;  // bound of every device-side wait
   int32_t skip_level = -1;          // failure injection for tests
   // scratch for readback / queries
@@ -1200,7 +1201,7 @@ int echo_estimate_collectives(echo_ctx *c) {
   CK(cudaMemsetAsync(c->comm_sum, 0, S * sizeof(double), c->stream), "memset");
   CK(timed(c, "cc_estimate", [&] {
        return echo::launch_cc_estimate(c->sigs, G, p, S, c->tbl, c->sig_count, c->cc_ns, c->cc_dur,
-                                       c->comm_sum, c->status, c->stream);
+                                       c->comm_sum, c->status, c->cc_model, c->stream);
      }), "cc_estimate launch");
   CK(timed(c, "cc_scatter", [&] {
        return echo::launch_cc_scatter(c->comm_node, c->comm_sig, (int64_t)B.comm_node.size(), c->cc_dur, S,
@@ -1512,6 +1513,16 @@ int echo_graph_info_get(echo_ctx *c, echo_graph_info *info) {
   info->n_ranks = B.R;
   info->n_streams = B.NS;
   info->sigma = c->sigma;
+  return ECHO_OK;
+}
+
+int echo_set_cc_model(echo_ctx *c, int model) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (model != ECHO_CC_MODEL_WHITEBOX && model != ECHO_CC_MODEL_ALPHA_BETA)
+    return set_err(c, ECHO_E_INVALID_ARG, "unknown collective cost model");
+  c->cc_model = model;
+  if (c->state > 2) c->state = 2;  // the estimates must be made again
   return ECHO_OK;
 }
 

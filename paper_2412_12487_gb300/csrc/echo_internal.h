@@ -152,7 +152,7 @@ struct OverlapArgs {
 // kernels.cu
 cudaError_t launch_cc_estimate(const CcSig *sig, int32_t G, ScenParams p, int32_t S,
                                const ChunkTable &tbl, const int32_t *sig_count, double *cc_ns,
-                               int64_t *cc_dur, double *comm_sum, int32_t *status, cudaStream_t st);
+                               int64_t *cc_dur, double *comm_sum, int32_t *status, int model, cudaStream_t st);
 cudaError_t launch_cc_scatter(const int32_t *comm_node, const int32_t *comm_sig, int64_t n_comm,
                               const int64_t *cc_dur, int32_t S, MatLayout lay, int64_t *dur, cudaStream_t st);
 cudaError_t launch_cc_query(int64_t n, const uint8_t *type, const uint8_t *algo, const int64_t *nbytes,

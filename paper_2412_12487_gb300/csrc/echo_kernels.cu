@@ -130,13 +130,22 @@ __device__ __forceinline__ void set_status(int32_t *status, int32_t code) {
 __global__ void cc_estimate_kernel(const CcSig *__restrict__ sig, int32_t G, ScenParams p, int32_t S,
                                    ChunkTable tbl, const int32_t *__restrict__ sig_count,
                                    double *__restrict__ cc_ns, int64_t *__restrict__ cc_dur,
-                                   double *__restrict__ comm_sum, int32_t *status) {
+                                   double *__restrict__ comm_sum, int32_t *status, int model) {
   int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)G * S) return;
   int32_t g = (int32_t)(idx / S), s = (int32_t)(idx % S);
   CcSig q = sig[g];
-  double T = cc_ns_of(q.type, q.algo, q.nbytes, q.N, q.M, q.K, q.lg, p.alpha[s], p.bwa[s], p.lata[s],
-                      p.bwe[s], p.late[s], p.delta[s], tbl);
+  double T;
+  if (model == 1) {
+    // alpha-beta comparison model (Sec. 2.3): size over bandwidth plus latency on
+    // the bottleneck link
+    T = (q.N <= 1 || q.nbytes <= 0)
+            ? 0.0
+            : __dadd_rn(q.M > 1 ? p.late[s] : p.lata[s], __ddiv_rn((double)q.nbytes, q.M > 1 ? p.bwe[s] : p.bwa[s]));
+  } else {
+    T = cc_ns_of(q.type, q.algo, q.nbytes, q.N, q.M, q.K, q.lg, p.alpha[s], p.bwa[s], p.lata[s], p.bwe[s],
+                 p.late[s], p.delta[s], tbl);
+  }
   int64_t d = 0;
   if (T >= 0.0 && T < 2305843009213693952.0) {  // 2^61
     d = __double2ll_rn(T);
@@ -408,13 +417,13 @@ int grid_for(int64_t n, int threads) {
 
 cudaError_t launch_cc_estimate(const CcSig *sig, int32_t G, ScenParams p, int32_t S, const ChunkTable &tbl,
                                const int32_t *sig_count, double *cc_ns, int64_t *cc_dur, double *comm_sum,
-                               int32_t *status, cudaStream_t st) {
+                               int32_t *status, int model, cudaStream_t st) {
   int64_t n = (int64_t)G * S;
   if (n == 0) return cudaSuccess;
   int threads = 256;
   int64_t blocks = (n + threads - 1) / threads;
   cc_estimate_kernel<<<(unsigned)blocks, threads, 0, st>>>(sig, G, p, S, tbl, sig_count, cc_ns, cc_dur,
-                                                          comm_sum, status);
+                                                          comm_sum, status, model);
   return cudaGetLastError();
 }
 

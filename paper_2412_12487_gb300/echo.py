@@ -23,7 +23,7 @@ STATUS_NAMES = {0: "ECHO_OK", 1: "ECHO_E_INVALID_ARG", 2: "ECHO_E_BAD_GRAPH", 3:
 EXPORTS = ["echo_create", "echo_destroy", "echo_check_graph", "echo_load_graph", "echo_load_scenarios",
            "echo_estimate_collectives", "echo_compose", "echo_read_times", "echo_read_makespan",
            "echo_read_cc", "echo_read_overlap", "echo_cc_query", "echo_cc_query_noalloc",
-           "echo_graph_info_get",
+           "echo_graph_info_get", "echo_set_cc_model",
            "echo_set_profiling", "echo_read_profile", "echo_strerror", "echo_last_error"]
 
 
@@ -34,6 +34,7 @@ class EchoError(RuntimeError):
 
 
 CUDA_STREAM_LEGACY = 0x1  # cudaStreamLegacy
+CC_MODEL_WHITEBOX, CC_MODEL_ALPHA_BETA = 0, 1
 
 
 class GraphDesc(C.Structure):
@@ -110,6 +111,7 @@ def load_library(path: Optional[str] = None):
         "echo_cc_query": ([vp, C.POINTER(CCQueryDesc), vp], C.c_int),
         "echo_cc_query_noalloc": ([C.POINTER(CCQueryDesc), vp, vp], C.c_int),
         "echo_graph_info_get": ([vp, C.POINTER(GraphInfo)], C.c_int),
+        "echo_set_cc_model": ([vp, C.c_int], C.c_int),
         "echo_set_profiling": ([vp, C.c_int], C.c_int),
         "echo_read_profile": ([vp, C.POINTER(KernelStat), C.c_int, C.POINTER(C.c_int)], C.c_int),
         "echo_strerror": ([C.c_int], C.c_char_p),
@@ -293,6 +295,10 @@ class Echo:
         gi = GraphInfo()
         self._check(self.lib.echo_graph_info_get(self.h, C.byref(gi)))
         return {k: int(getattr(gi, k)) for k, _ in GraphInfo._fields_}
+
+    def set_cc_model(self, model: int):
+        """CC_MODEL_WHITEBOX (Eqs. 2-5, default) or CC_MODEL_ALPHA_BETA for the next estimate."""
+        self._check(self.lib.echo_set_cc_model(self.h, int(model)))
 
     def set_profiling(self, on: bool):
         self._check(self.lib.echo_set_profiling(self.h, 1 if on else 0))

@@ -121,6 +121,33 @@ def test_slowdown_rounding_is_exact():
     assert_same(got, oracle.compose(g, sc, refine_passes=1), g, 1)
 
 
+def test_alpha_beta_cost_model_bit_exact():
+    """The alpha-beta comparison model (size / bandwidth + latency) through
+    echo_set_cc_model, against the oracle's; then back to Eqs. 2-5."""
+    from paper_2412_12487_gb300.echo import CC_MODEL_ALPHA_BETA, CC_MODEL_WHITEBOX
+    c = W.config("tiny")
+    c = W.GPTConfig(**{**c.__dict__, "fixed_scenario": False})
+    rng = np.random.default_rng(4242)
+    cases = [(W.build_gpt_graph(c), None)]
+    for _ in range(12):
+        cases.append((SG.random_graph(rng, int(rng.integers(5, 60)), max_ranks=5, max_streams=4, p_edge=0.08),
+                      None))
+    e = Echo(0)
+    try:
+        for k, (g, _) in enumerate(cases):
+            sc = W.make_scenarios(g, c, n_scen=6) if k == 0 else SG.random_scenarios(rng, g, 37, max_dur=50)
+            e.set_cc_model(CC_MODEL_ALPHA_BETA)
+            got = run_gpu(g, sc, 1, ctx=e)
+            assert_same(got, oracle.compose(g, sc, refine_passes=1, cc_model=1), g, 1)
+            e.set_cc_model(CC_MODEL_WHITEBOX)
+            got = run_gpu(g, sc, 1, ctx=e)
+            assert_same(got, oracle.compose(g, sc, refine_passes=1, cc_model=0), g, 1)
+        with pytest.raises(EchoError):
+            e.set_cc_model(7)
+    finally:
+        e.close()
+
+
 def test_gpt13b_all_ops_all_scenarios_bit_exact():
     c = W.config("gpt1.3b")
     g = W.build_gpt_graph(c)

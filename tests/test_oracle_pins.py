@@ -196,6 +196,35 @@ def test_reduction_term_and_degenerate_cases():
             assert _cc(t, 2, S, 1, 1, 1, p) == 0.0
 
 
+def test_alpha_beta_model_is_size_over_bandwidth_plus_latency():
+    """The comparison model of Sec. 2.3: message size / bandwidth + latency, on the
+    intra-node link inside a node and the inter-node one across nodes; setup
+    (alpha) and reduction (delta) costs play no part, nor does the chunk table."""
+    # 1 MiB at 50 B/ns with a 5 us latency: 5000 + 20971.52 ns
+    assert oracle.cc_ns_alpha_beta(1 << 20, 8, 1, 10000.0, 50.0, 5000.0, 6.25, 9000.0, 1e-3) == 25971.52
+    # across nodes: 1 MiB at 6.25 B/ns with 9 us: 9000 + 167772.16 ns
+    assert oracle.cc_ns_alpha_beta(1 << 20, 16, 2, 10000.0, 50.0, 5000.0, 6.25, 9000.0, 1e-3) == 176772.16
+    assert oracle.cc_ns_alpha_beta(1 << 20, 1, 1, 10000.0, 50.0, 5000.0, 6.25, 9000.0, 1e-3) == 0.0
+    assert oracle.cc_ns_alpha_beta(0, 8, 2, 10000.0, 50.0, 5000.0, 6.25, 9000.0, 1e-3) == 0.0
+
+
+def test_alpha_beta_composition_times_every_collective_by_the_model():
+    g = W.build_gpt_graph(W.config("tiny"))
+    sc = W.make_scenarios(g, W.config("tiny"), n_scen=1)
+    r = oracle.compose(g, sc, refine_passes=0, cc_model=1)
+    comm = np.nonzero((g.kind == W.KIND_COLL) | (g.kind == W.KIND_P2P))[0]
+    assert len(comm) > 10
+    for v in comm:
+        members = g.grp_rank[g.grp_off[g.group[v]]:g.grp_off[g.group[v] + 1]]
+        nodes = len(set(int(m) // g.gpus_per_node for m in members))
+        B, L = (sc.bw_inter[0], sc.lat_inter[0]) if nodes > 1 else (sc.bw_intra[0], sc.lat_intra[0])
+        want = 0 if len(members) <= 1 or g.cc_bytes[v] == 0 else int(np.rint(L + g.cc_bytes[v] / B))
+        assert r.finish[v, 0] - r.start[v, 0] == want
+    # the white-box times differ from these
+    w = oracle.compose(g, sc, refine_passes=0, cc_model=0)
+    assert not np.array_equal(w.finish[comm] - w.start[comm], r.finish[comm] - r.start[comm])
+
+
 def test_auto_takes_the_faster_algorithm():
     rng = np.random.default_rng(13)
     for _ in range(300):
