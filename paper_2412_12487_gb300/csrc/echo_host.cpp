@@ -82,6 +82,9 @@ struct GraphBuild {
 
 bool finite_nonneg(double x) { return std::isfinite(x) && x >= 0.0; }
 
+constexpr int64_t kStepNodes = 2048;     // nodes of one composition step (a level or a part of one)
+constexpr int64_t kStepSegments = 1024;  // segments of one composition step
+
 // Compute ops that can overlap a comm op of their rank in some scenario (the
 // validator of Sec. 3 tests only these).  A rank's compute timeline is a serial
 // chain, so for a comm op w on rank r the compute ops of r up to the latest one
@@ -462,6 +465,27 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
       }
     }
     b.seg_node_off[NSg] = i;
+  }
+  // The segments of one level are independent, so a wide level may run as several
+  // consecutive steps: each step holds at most kStepNodes nodes and kStepSegments
+  // segments, so that two consecutive steps fit the shared-memory rings of the
+  // staged kernels (the numbering stays as it is).
+  {
+    std::vector<int64_t> off{0};
+    for (int64_t l = 0; l < Ls; ++l) {
+      int64_t t = b.seg_lvl_off[l];
+      while (t < b.seg_lvl_off[l + 1]) {
+        int64_t u = t + 1;  // one segment always fits (at most kMaxSegment nodes)
+        while (u < b.seg_lvl_off[l + 1] && u - t < kStepSegments &&
+               b.seg_node_off[u + 1] - b.seg_node_off[t] <= kStepNodes)
+          ++u;
+        off.push_back(u);
+        t = u;
+      }
+    }
+    b.seg_lvl_off = off;
+    Ls = (int64_t)off.size() - 1;
+    b.Ls = Ls;
   }
   // Inputs of every segment head: its distinct predecessors over data and issue
   // order (each the tail of an earlier segment, as a chain only continues through
