@@ -115,7 +115,8 @@ typedef struct {
   int32_t n_scen;                  /* S >= 1                                          */
   int32_t n_kclass;                /* rows of slowdown; > every compute op's kclass   */
   int32_t n_chunk;                 /* entries of the chunk table, 0 = Table 6 default */
-  const int64_t *dur;              /* [V][S] ns >= 0; entries of COLL/P2P ops ignored */
+  const void *dur;                 /* [V][S] ns >= 0 (int64, or int32 when dur_bits is
+                                      32); entries of COLL/P2P ops ignored            */
   const double *alpha_ns;          /* [S] >= 0                                        */
   const double *bw_intra;          /* [S] > 0, intra-node link                        */
   const double *lat_intra;         /* [S] >= 0                                        */
@@ -126,6 +127,9 @@ typedef struct {
   const int64_t *chunk_max_bytes;  /* [n_chunk] ascending: messages <= max use ...    */
   const int64_t *chunk_bytes;      /* [n_chunk] ... this chunk size (> 0); larger
                                       messages use the last entry                     */
+  int32_t dur_bits;                /* width of the dur entries: 64 (0 means 64) or 32;
+                                      32 halves the upload when every duration fits;
+                                      the composition computes in int64 either way    */
 } echo_scen_desc;
 
 typedef struct {

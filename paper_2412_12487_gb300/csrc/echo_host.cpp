@@ -1092,6 +1092,8 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   if (sc->n_kclass < 1 || sc->n_kclass <= B.max_kclass)
     return set_err(c, ECHO_E_INVALID_ARG, "n_kclass must exceed every compute op's kclass");
   if (V > 0 && !sc->dur) return set_err(c, ECHO_E_INVALID_ARG, "dur is NULL");
+  if (sc->dur_bits != 0 && sc->dur_bits != 32 && sc->dur_bits != 64)
+    return set_err(c, ECHO_E_INVALID_ARG, "dur_bits must be 32 or 64");
   if (!sc->slowdown) return set_err(c, ECHO_E_INVALID_ARG, "slowdown is NULL");
   if ((rc = check_params(c, S, sc->alpha_ns, sc->bw_intra, sc->lat_intra, sc->bw_inter, sc->lat_inter, sc->delta)))
     return rc;
@@ -1196,11 +1198,12 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   CK(cudaMemsetAsync(c->sums, 0, S * sizeof(double), c->stream), "memset");
   CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
   if (V > 0) {
-    CK(cudaMemcpyAsync(c->raw, sc->dur, (size_t)V * S * sizeof(int64_t), cudaMemcpyHostToDevice, c->stream),
+    const int bits = sc->dur_bits == 32 ? 32 : 64;
+    CK(cudaMemcpyAsync(c->raw, sc->dur, (size_t)V * S * (bits / 8), cudaMemcpyHostToDevice, c->stream),
        "duration upload");
     CK(timed(c, "permute_rows", [&] {
-         return echo::launch_permute_rows(c->raw, c->int2ext, c->local, V, S, c->lay, c->dur, c->sums, c->status,
-                                          c->stream);
+         return echo::launch_permute_rows(c->raw, bits, c->int2ext, c->local, V, S, c->lay, c->dur, c->sums,
+                                          c->status, c->stream);
        }), "permute_rows launch");
   }
   c->h_sums.assign(S, 0.0);

@@ -158,7 +158,7 @@ cudaError_t launch_cc_scatter(const int32_t *comm_node, const int32_t *comm_sig,
 cudaError_t launch_cc_query(int64_t n, const uint8_t *type, const uint8_t *algo, const int64_t *nbytes,
                             const int32_t *N, const int32_t *M, const double *lg, ScenParams p,
                             const ChunkTable &tbl, double *out, cudaStream_t st);
-cudaError_t launch_permute_rows(const int64_t *raw, const int32_t *int2ext, const uint8_t *local,
+cudaError_t launch_permute_rows(const void *raw, int bits, const int32_t *int2ext, const uint8_t *local,
                                 int64_t V, int32_t S, MatLayout lay, int64_t *dur, double *sums, int32_t *status,
                                 cudaStream_t st);
 cudaError_t launch_compose(const ComposeArgs &a, int sigma, cudaStream_t st);

@@ -187,7 +187,8 @@ __global__ void cc_query_kernel(int64_t n, const uint8_t *__restrict__ type, con
 // load: caller-order rows -> internal order and blocked layout, with validation
 // and per-scenario sums
 // ---------------------------------------------------------------------------------
-__global__ void permute_rows_kernel(const int64_t *__restrict__ raw, const int32_t *__restrict__ int2ext,
+template <typename T>
+__global__ void permute_rows_kernel(const T *__restrict__ raw, const int32_t *__restrict__ int2ext,
                                     const uint8_t *__restrict__ local, int64_t V, int32_t S, MatLayout lay,
                                     int64_t *__restrict__ dur, double *__restrict__ sums, int32_t *status) {
   int32_t s = blockIdx.x * blockDim.x + threadIdx.x;
@@ -198,7 +199,7 @@ __global__ void permute_rows_kernel(const int64_t *__restrict__ raw, const int32
     int64_t e = int2ext[i];
     int64_t d = 0;
     if (local[i]) {
-      d = raw[e * S + s];
+      d = (int64_t)raw[e * S + s];
       neg |= d < 0;
       acc += (double)d;
     }
@@ -442,7 +443,7 @@ cudaError_t launch_cc_query(int64_t n, const uint8_t *type, const uint8_t *algo,
   return cudaGetLastError();
 }
 
-cudaError_t launch_permute_rows(const int64_t *raw, const int32_t *int2ext, const uint8_t *local, int64_t V,
+cudaError_t launch_permute_rows(const void *raw, int bits, const int32_t *int2ext, const uint8_t *local, int64_t V,
                                 int32_t S, MatLayout lay, int64_t *dur, double *sums, int32_t *status,
                                 cudaStream_t st) {
   if (V == 0 || S == 0) return cudaSuccess;
@@ -450,7 +451,12 @@ cudaError_t launch_permute_rows(const int64_t *raw, const int32_t *int2ext, cons
   dim3 block(tx);
   int64_t gy = V < 8192 ? V : 8192;
   dim3 grid((S + tx - 1) / tx, (unsigned)gy);
-  permute_rows_kernel<<<grid, block, 0, st>>>(raw, int2ext, local, V, S, lay, dur, sums, status);
+  if (bits == 32)
+    permute_rows_kernel<int32_t><<<grid, block, 0, st>>>(static_cast<const int32_t *>(raw), int2ext, local, V, S,
+                                                         lay, dur, sums, status);
+  else
+    permute_rows_kernel<int64_t><<<grid, block, 0, st>>>(static_cast<const int64_t *>(raw), int2ext, local, V, S,
+                                                         lay, dur, sums, status);
   return cudaGetLastError();
 }
 

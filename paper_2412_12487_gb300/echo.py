@@ -51,7 +51,7 @@ class ScenDesc(C.Structure):
                 ("dur", C.c_void_p), ("alpha_ns", C.c_void_p), ("bw_intra", C.c_void_p),
                 ("lat_intra", C.c_void_p), ("bw_inter", C.c_void_p), ("lat_inter", C.c_void_p),
                 ("delta", C.c_void_p), ("slowdown", C.c_void_p), ("chunk_max_bytes", C.c_void_p),
-                ("chunk_bytes", C.c_void_p)]
+                ("chunk_bytes", C.c_void_p), ("dur_bits", C.c_int32)]
 
 
 class ComposeOpts(C.Structure):
@@ -219,7 +219,8 @@ class Echo:
         self.n_ops = int(g.kind.shape[0])
 
     def load_scenarios(self, sc, dur=None):
-        """``dur`` overrides ``sc.dur`` (e.g. a pinned torch tensor of the same shape)."""
+        """``dur`` overrides ``sc.dur`` (e.g. a pinned torch tensor of the same shape).
+        int32 durations (numpy or torch) are uploaded as such, half the bytes of int64."""
         keep: list = []
 
         def a(x, dt):
@@ -228,8 +229,9 @@ class Echo:
             return y.ctypes.data
 
         D = sc.dur if dur is None else dur
+        bits = 32 if str(getattr(D, "dtype", "")) in ("int32", "torch.int32") else 64
         if isinstance(D, np.ndarray):
-            D = _c(D, np.int64)
+            D = _c(D, np.int32 if bits == 32 else np.int64)
             keep.append(D)
         S = int(sc.alpha_ns.shape[0])
         n_chunk = 0 if sc.chunk_max_bytes is None else len(sc.chunk_max_bytes)
@@ -238,7 +240,7 @@ class Echo:
                      a(sc.bw_inter, np.float64), a(sc.lat_inter, np.float64), a(sc.delta, np.float64),
                      a(sc.slowdown, np.float64),
                      a(sc.chunk_max_bytes, np.int64) if n_chunk else None,
-                     a(sc.chunk_bytes, np.int64) if n_chunk else None)
+                     a(sc.chunk_bytes, np.int64) if n_chunk else None, bits)
         self._check(self.lib.echo_load_scenarios(self.h, C.byref(d)))
         self.n_scen = S
 

@@ -148,6 +148,30 @@ def test_alpha_beta_cost_model_bit_exact():
         e.close()
 
 
+def test_int32_durations_give_the_same_timelines():
+    """Durations passed as int32 (half the upload) compose exactly like int64 ones."""
+    import dataclasses
+    c = W.config("gpt1.3b")
+    g = W.build_gpt_graph(c)
+    sc = W.make_scenarios(g, c, n_scen=40)
+    assert sc.dur.max() < 2**31
+    sc32 = dataclasses.replace(sc, dur=sc.dur.astype(np.int32))
+    e = Echo(0)
+    try:
+        a = run_gpu(g, sc, 2, ctx=e)
+        b = run_gpu(g, sc32, 2, ctx=e)
+        for k in ("start", "finish", "makespan", "ov"):
+            assert np.array_equal(a[k], b[k]), k
+        np.testing.assert_array_equal(a["cc"], b["cc"])
+        bad = sc32.dur.copy()
+        bad[int(np.nonzero(g.kind == W.KIND_COMPUTE)[0][7]), 3] = -1
+        with pytest.raises(EchoError) as ei:
+            e.load_scenarios(dataclasses.replace(sc32, dur=bad))
+        assert ei.value.code == 1
+    finally:
+        e.close()
+
+
 def test_gpt13b_all_ops_all_scenarios_bit_exact():
     c = W.config("gpt1.3b")
     g = W.build_gpt_graph(c)
