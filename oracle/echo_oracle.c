@@ -116,6 +116,33 @@ double oracle_cc_ns(int cc_type, int cc_algo, int64_t nbytes, int N, int M, int 
   return (t < r) ? t : r;
 }
 
+/* Total length covered by the intervals [lo[i], hi[i]) (their union): sort by
+ * start, then sweep, counting each stretch once. */
+static void sort_intervals(int64_t *lo, int64_t *hi, int64_t m) {
+  for (int64_t i = 1; i < m; ++i) { /* insertion sort: the lists are short */
+    int64_t a = lo[i], b = hi[i], j = i - 1;
+    while (j >= 0 && lo[j] > a) {
+      lo[j + 1] = lo[j];
+      hi[j + 1] = hi[j];
+      --j;
+    }
+    lo[j + 1] = a;
+    hi[j + 1] = b;
+  }
+}
+static int64_t union_length(int64_t *lo, int64_t *hi, int64_t m) {
+  sort_intervals(lo, hi, m);
+  int64_t total = 0, covered = INT64_MIN;
+  for (int64_t i = 0; i < m; ++i) {
+    int64_t a = lo[i] > covered ? lo[i] : covered;
+    if (hi[i] > a) {
+      total += hi[i] - a;
+      covered = hi[i];
+    }
+  }
+  return total;
+}
+
 /* The alpha-beta model that Sec. 2.3 describes for the simulators Echo compares
  * against (NCCL-Predictor, Sec. 8.3): a collective takes its message size over the
  * bandwidth plus the latency.  Read here on the group's bottleneck link, the
@@ -279,13 +306,17 @@ int oracle_compose(const oracle_graph *g, const oracle_scen *sc, int32_t s0, int
   uint8_t *ov = calloc((size_t)(V > 0 ? V : 1), 1);
   int64_t *cst = malloc((size_t)(QE > 0 ? QE : 1) * sizeof(int64_t)); /* one rank's comm intervals */
   int64_t *cfn = malloc((size_t)(QE > 0 ? QE : 1) * sizeof(int64_t));
+  int64_t *clo = malloc((size_t)(QE > 0 ? QE : 1) * sizeof(int64_t)); /* clipped to one kernel */
+  int64_t *chi = malloc((size_t)(QE > 0 ? QE : 1) * sizeof(int64_t));
+  int64_t *olen = calloc((size_t)(V > 0 ? V : 1), sizeof(int64_t)); /* overlapped length */
   int32_t G = g->n_groups;
   int32_t *gN = calloc((size_t)(G > 0 ? G : 1), sizeof(int32_t));
   int32_t *gM = calloc((size_t)(G > 0 ? G : 1), sizeof(int32_t));
   int32_t *gK = calloc((size_t)(G > 0 ? G : 1), sizeof(int32_t));
   double *glg = calloc((size_t)(G > 0 ? G : 1), sizeof(double));
   if (!sim.succ_off || !sim.succ_idx || !sim.opq_off || !sim.opq_q || !sim.opq_pos || !sim.cnt ||
-      !sim.heap || !fill || !d0 || !d || !st || !fn || !ov || !cst || !cfn || !gN || !gM || !gK || !glg) {
+      !sim.heap || !fill || !d0 || !d || !st || !fn || !ov || !cst || !cfn || !clo || !chi || !olen || !gN || !gM ||
+      !gK || !glg) {
     rc = ORACLE_E_NOMEM;
     goto out;
   }
@@ -363,20 +394,32 @@ int oracle_compose(const oracle_graph *g, const oracle_scen *sc, int32_t s0, int
         for (int64_t i = g->q_off[qa]; i < g->q_off[qb]; ++i) {
           int32_t v = g->q_ops[i];
           if (g->kind[v] != K_COMPUTE) continue;
-          uint8_t hit = 0;
-          for (int64_t j = 0; j < nc && !hit; ++j) {
+          /* the parts of the rank's comm intervals inside the kernel's interval; the
+           * kernel is overlapped when they cover a positive length */
+          int64_t m = 0;
+          for (int64_t j = 0; j < nc; ++j) {
             int64_t lo = st[v] > cst[j] ? st[v] : cst[j];
             int64_t hi = fn[v] < cfn[j] ? fn[v] : cfn[j];
-            if (lo < hi) hit = 1;
+            if (lo < hi) {
+              clo[m] = lo;
+              chi[m] = hi;
+              m++;
+            }
           }
-          ov[v] = hit;
+          ov[v] = m > 0;
+          olen[v] = union_length(clo, chi, m);
         }
       }
       for (int64_t v = 0; v < V; ++v) {
-        if (g->kind[v] == K_COMPUTE && ov[v])
-          d[v] = llrint((double)d0[v] * sc->slowdown[(int64_t)g->kclass[v] * S + s]);
-        else
+        if (g->kind[v] == K_COMPUTE && ov[v]) {
+          double f = sc->slowdown[(int64_t)g->kclass[v] * S + s];
+          if (sc->overlap_model == 1) /* the overlapped part of the kernel runs f times longer */
+            d[v] = llrint((double)d0[v] + (f - 1.0) * (double)olen[v]);
+          else /* the whole kernel does (Sec. 2.3) */
+            d[v] = llrint((double)d0[v] * f);
+        } else {
           d[v] = d0[v];
+        }
       }
       rc = simulate(&sim, d, st, fn);
       if (rc) goto out;
@@ -407,6 +450,9 @@ out:
   free(ov);
   free(cst);
   free(cfn);
+  free(clo);
+  free(chi);
+  free(olen);
   free(gN);
   free(gM);
   free(gK);

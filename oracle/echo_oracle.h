@@ -33,6 +33,8 @@ typedef struct {
   const double *slowdown;                                                      /* [n_kclass][n_scen] */
   const int64_t *chunk_max_bytes, *chunk_bytes; /* [n_chunk]; n_chunk = 0 -> Table 6 */
   int32_t cc_model; /* 0: Eqs. 2-5 (white box), 1: alpha-beta */
+  int32_t overlap_model; /* 0: an overlapped kernel takes d * factor;
+                            1: d + (factor - 1) * (length of its overlap) */
 } oracle_scen;
 
 int64_t oracle_chunk_bytes(int64_t nbytes, int n_chunk, const int64_t *max_bytes,

@@ -225,6 +225,63 @@ def test_alpha_beta_composition_times_every_collective_by_the_model():
     assert not np.array_equal(w.finish[comm] - w.start[comm], r.finish[comm] - r.start[comm])
 
 
+def _overlap_case(two_streams):
+    """Rank 0 runs kernel c (100 ns) from 0; on its comm timeline(s) a memcpy (50 or
+    70 ns) precedes a send/recv with rank 1 of 1000 B at 10 B/ns (100 ns, no setup
+    or latency), so the send/recv runs [50, 150) (and the second one [70, 170))."""
+    ops = [{"kind": W.KIND_COMPUTE, "kclass": 0},
+           {"kind": W.KIND_MEMCPY},
+           {"kind": W.KIND_P2P, "group": 0, "cc_type": W.CC_SENDRECV, "cc_bytes": 1000}]
+    queues = {(0, 0): [0], (0, 1): [1, 2], (1, 1): [2]}
+    groups = [[0, 1]]
+    if two_streams:
+        ops += [{"kind": W.KIND_MEMCPY},
+                {"kind": W.KIND_P2P, "group": 1, "cc_type": W.CC_SENDRECV, "cc_bytes": 1000}]
+        queues.update({(0, 2): [3, 4], (1, 2): [4]})
+        groups.append([0, 1])
+    g = SG.graph_from_lists(2, 3 if two_streams else 2, ops, queues, groups, gpus_per_node=2)
+    dur = np.zeros((len(ops), 1), np.int64)
+    dur[0, 0], dur[1, 0] = 100, 50
+    if two_streams:
+        dur[3, 0] = 70
+    sc = W.Scenarios(dur=dur, alpha_ns=np.zeros(1), bw_intra=np.full(1, 10.0), lat_intra=np.zeros(1),
+                     bw_inter=np.full(1, 10.0), lat_inter=np.zeros(1), delta=np.zeros(1),
+                     slowdown=np.full((1, 1), 1.5), peak_flop_per_ns=np.ones(1))
+    return g, sc
+
+
+def test_whole_kernel_and_proportional_slowdown_by_hand():
+    g, sc = _overlap_case(False)
+    r = oracle.compose(g, sc, refine_passes=1, overlap_model=0)
+    assert (r.start[2, 0], r.finish[2, 0]) == (50, 150)
+    assert r.overlapped[0, 0] == 1 and r.finish[0, 0] - r.start[0, 0] == 150  # 100 * 1.5
+    r = oracle.compose(g, sc, refine_passes=1, overlap_model=1)
+    assert r.finish[0, 0] - r.start[0, 0] == 125  # 100 + 0.5 * 50 (overlap [50, 100))
+
+
+def test_proportional_slowdown_counts_overlapping_comm_once():
+    g, sc = _overlap_case(True)
+    r = oracle.compose(g, sc, refine_passes=1, overlap_model=1)
+    assert (r.start[4, 0], r.finish[4, 0]) == (70, 170)
+    # [50, 100) and [70, 100) cover [50, 100): 50 ns, not 80
+    assert r.finish[0, 0] - r.start[0, 0] == 125
+    r = oracle.compose(g, sc, refine_passes=1, overlap_model=0)
+    assert r.finish[0, 0] - r.start[0, 0] == 150
+
+
+def test_proportional_model_never_exceeds_whole_kernel_model():
+    rng = np.random.default_rng(31)
+    for _ in range(200):
+        g = SG.random_graph(rng, int(rng.integers(2, 30)), max_ranks=3, max_streams=4, p_edge=0.1)
+        sc = SG.random_scenarios(rng, g, 3, max_dur=40)
+        a = oracle.compose(g, sc, refine_passes=1, overlap_model=0)
+        b = oracle.compose(g, sc, refine_passes=1, overlap_model=1)
+        assert np.array_equal(a.overlapped, b.overlapped)  # same decisions from the same first pass
+        comp = g.kind == W.KIND_COMPUTE
+        # slowdown factors are >= 1: the overlapped part is at most the whole kernel
+        assert ((b.finish - b.start)[comp] <= (a.finish - a.start)[comp]).all()
+
+
 def test_auto_takes_the_faster_algorithm():
     rng = np.random.default_rng(13)
     for _ in range(300):
