@@ -138,7 +138,13 @@ typedef struct {
    * recomputes the overlap from pass k's times and always slows the ORIGINAL
    * durations.  At most 8. */
   int32_t refine_passes;
+  /* how an overlapped kernel is slowed: ECHO_OVERLAP_WHOLE (default) multiplies its
+   * duration by its factor (Sec. 2.3: the factor is the ratio of its times with and
+   * without overlapping communication); ECHO_OVERLAP_PROPORTIONAL adds (factor - 1)
+   * times the length of its interval covered by its rank's comm intervals. */
+  int32_t overlap_model;
 } echo_compose_opts;
+enum { ECHO_OVERLAP_WHOLE = 0, ECHO_OVERLAP_PROPORTIONAL = 1 };
 
 /* Create a context on `device`, enqueuing on `cuda_stream` (a cudaStream_t; NULL =
  * a new non-blocking stream owned by the context; the legacy default stream is

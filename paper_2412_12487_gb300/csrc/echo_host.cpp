@@ -771,6 +771,7 @@ struct echo_ctx {
   ChunkTable tbl{};
   double *prm = nullptr, *sums = nullptr, *comm_sum = nullptr, *cc_ns = nullptr;
   uint64_t *sfx = nullptr;  // packed slowdown factors [C][S]
+  double *sf = nullptr;     // slowdown factors [C][S]
   std::vector<uint64_t> h_sfx;
   int64_t *raw = nullptr, *dur = nullptr, *f[2] = {nullptr, nullptr}, *mk = nullptr, *cc_dur = nullptr;
   int64_t *gfrontier = nullptr;
@@ -1124,7 +1125,7 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     echo::compose_smem_bytes(B.R * B.NS, sigma, &in_smem);
     int64_t nblk = (S + sigma - 1) / sigma;
     const size_t CS = (size_t)std::max<int64_t>(B.n_cand, 1) * (size_t)nblk * sigma;  // compact matrices
-    if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sfx, (size_t)C * S)) ||
+    if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sfx, (size_t)C * S)) || (rc = dalloc(c, o, &c->sf, (size_t)C * S)) ||
         (rc = dalloc(c, o, &c->sums, (size_t)S)) || (rc = dalloc(c, o, &c->comm_sum, (size_t)S)) ||
         (rc = dalloc(c, o, &c->raw, (size_t)V * S)) || (rc = dalloc(c, o, &c->dur, VS)) ||
         (rc = dalloc(c, o, &c->f[0], VS)) || (rc = dalloc(c, o, &c->f[1], VS)) ||
@@ -1195,6 +1196,8 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   }
   CK(cudaMemcpyAsync(c->sfx, c->h_sfx.data(), c->h_sfx.size() * sizeof(uint64_t), cudaMemcpyHostToDevice, c->stream),
      "slowdown upload");
+  CK(cudaMemcpyAsync(c->sf, sc->slowdown, (size_t)C * S * sizeof(double), cudaMemcpyHostToDevice, c->stream),
+     "slowdown upload");
   CK(cudaMemsetAsync(c->sums, 0, S * sizeof(double), c->stream), "memset");
   CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
   if (V > 0) {
@@ -1255,6 +1258,9 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   if (c->state < 3) return set_err(c, ECHO_E_STATE, "estimate the collectives first");
   int32_t refine = opts ? opts->refine_passes : 1;
   if (refine < 0 || refine > 8) return set_err(c, ECHO_E_INVALID_ARG, "refine_passes outside [0, 8]");
+  const int32_t model = opts ? opts->overlap_model : ECHO_OVERLAP_WHOLE;
+  if (model != ECHO_OVERLAP_WHOLE && model != ECHO_OVERLAP_PROPORTIONAL)
+    return set_err(c, ECHO_E_INVALID_ARG, "unknown overlap model");
   const GraphBuild &B = c->gb;
   // the pipelined kernel reads the validator's durations of the candidates from a
   // ring of its own; the others compose from a full matrix built for them
@@ -1335,6 +1341,8 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     o.dur = c->dur;
     o.cd_used = cd_used;
     o.sfx = c->sfx;
+    o.sf = c->sf;
+    o.model = model;
     o.cd_next = c->cd[(p - 1) % 2];
     o.ov = nullptr;  // the decisions are recomputed on demand by echo_read_overlap
     CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");

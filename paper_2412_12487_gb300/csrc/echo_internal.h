@@ -145,6 +145,8 @@ struct OverlapArgs {
   const int64_t *dur;      // original durations
   const int64_t *cd_used;  // candidates' durations in the last pass (compact), or null: the original ones
   const uint64_t *sfx;     // [C][S] slowdown factors, packed as (53-bit significand << 11) | (exponent + 1075)
+  const double *sf;        // [C][S] the same factors (proportional model)
+  int32_t model;           // 0: d * factor; 1: d + (factor - 1) * overlapped length
   int64_t *cd_next;        // (out, compact; may be null) candidates' durations for the next pass
   uint8_t *ov;             // (out, [V][S] rows of the candidates; may be null)
 };

@@ -335,7 +335,48 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
         if (a.ov) a.ov[base + (v << sh)] = hit;
         if (cn) {
           const int64_t d0 = cu ? du[v << sh] : dv;  // the original duration
-          cn[cb[u] << sh] = hit ? slowed(d0, a.sfx[(int64_t)a.kcl[v] * S + sl]) : d0;
+          int64_t dn = d0;
+          if (hit && a.model == 1) {
+            // proportional model: the length of [sv, fv) covered by the union of the
+            // comm intervals, swept in start order across the timelines.  Later
+            // candidates start no earlier than fv, so a cursor moves past every
+            // interval that ends by fv; one reaching beyond fv stays.
+            int64_t len = 0, covered = sv;
+            uint32_t held = 0;  // timelines whose cursor interval reaches beyond fv
+            while (true) {
+              int jb = -1;
+              int64_t first = fv;
+#pragma unroll
+              for (int j = 0; j < NCMAX; ++j)
+                if (j < nc && !((held >> j) & 1) && sw[j] < first) {
+                  first = sw[j];
+                  jb = j;
+                }
+              if (jb < 0) break;
+#pragma unroll
+              for (int j = 0; j < NCMAX; ++j) {  // (j == jb, in registers)
+                if (j != jb) continue;
+                const int64_t lo = max(sw[j], covered), hi = min(fw[j], fv);
+                if (hi > lo) {
+                  len += hi - lo;
+                  covered = hi;
+                }
+                if (fw[j] > fv) {
+                  held |= 1u << j;
+                } else {
+                  do {
+                    ++cur[j];
+                    load(j);
+                  } while (cur[j] < end[j] && sw[j] >= fw[j]);
+                }
+              }
+            }
+            const double f = a.sf[(int64_t)a.kcl[v] * S + sl];
+            dn = __double2ll_rn(__dadd_rn((double)d0, __dmul_rn(__dsub_rn(f, 1.0), (double)len)));
+          } else if (hit) {
+            dn = slowed(d0, a.sfx[(int64_t)a.kcl[v] * S + sl]);
+          }
+          cn[cb[u] << sh] = dn;
         }
       }
     }

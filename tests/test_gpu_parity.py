@@ -19,13 +19,13 @@ CC_RTOL = 1e-9
 THREADS = max(1, min(16, os.cpu_count() or 1))
 
 
-def run_gpu(g, sc, refine=1, ctx=None):
+def run_gpu(g, sc, refine=1, ctx=None, overlap_model=0):
     e = ctx or Echo(0)
     try:
         e.load_graph(g)
         e.load_scenarios(sc)
         e.estimate_collectives()
-        e.compose(refine_passes=refine)
+        e.compose(refine_passes=refine, overlap_model=overlap_model)
         st, fn = e.read_times()
         return dict(start=st, finish=fn, makespan=e.read_makespan(), cc=e.read_cc(),
                     ov=e.read_overlap(), info=e.info())
@@ -168,6 +168,30 @@ def test_int32_durations_give_the_same_timelines():
         with pytest.raises(EchoError) as ei:
             e.load_scenarios(dataclasses.replace(sc32, dur=bad))
         assert ei.value.code == 1
+    finally:
+        e.close()
+
+
+def test_proportional_overlap_model_bit_exact():
+    """Overlapped kernels lengthened by (factor - 1) x the covered length of their
+    interval (union over the rank's comm intervals), against the oracle."""
+    rng = np.random.default_rng(5150)
+    e = Echo(0)
+    try:
+        for case in range(14):
+            g = SG.random_graph(rng, int(rng.integers(20, 400)), max_ranks=4, max_streams=16,
+                                min_streams=2 if case % 2 else 5, p_edge=0.01)
+            sc = SG.random_scenarios(rng, g, 45, max_dur=60)
+            for refine in (1, 2):
+                got = run_gpu(g, sc, refine, ctx=e, overlap_model=1)
+                assert_same(got, oracle.compose(g, sc, refine_passes=refine, overlap_model=1), g, refine)
+        c = W.config("gpt1.3b")
+        g = W.build_gpt_graph(c)
+        sc = W.make_scenarios(g, c, n_scen=24)
+        got = run_gpu(g, sc, 1, ctx=e, overlap_model=1)
+        assert_same(got, oracle.compose(g, sc, refine_passes=1, overlap_model=1, threads=THREADS), g, 1)
+        with pytest.raises(EchoError):
+            e.compose(refine_passes=1, overlap_model=5)
     finally:
         e.close()
 
