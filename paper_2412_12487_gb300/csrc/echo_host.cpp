@@ -67,13 +67,12 @@ struct GraphBuild {
   int64_t n_cand = 0;                 // overlap candidates
   std::vector<int32_t> cidx;          // [V] level-order index of a candidate (by internal id), -1 otherwise
   std::vector<int32_t> cand_cidx;     // level-order index of each entry of cand_ops
-  std::vector<int64_t> cand_lvl;      // [Ls+1] first level-order candidate index of each segment level
   std::vector<int32_t> cand_node;     // internal id of each candidate, in level order
   std::vector<int64_t> ov_chunks;     // (rank, first candidate index) of the overlap test's chunks
   int32_t n_cq = 0;                   // comm timelines per rank in cq_off (max over ranks)
   std::vector<int64_t> cq_off;        // [R*n_cq+1] comm ops of each (rank, comm timeline)
   std::vector<int32_t> cq_ops;        // internal ids, in issue order
-  std::vector<int64_t> blk_words;     // record block size of each segment level (words, padded)
+  std::vector<int64_t> seg_words;     // [n_seg] record words of each segment
   std::vector<int64_t> hin_off;       // [n_seg+1] inputs of each segment's head
   std::vector<int32_t> hin;           // (internal ids, each the tail of an earlier segment)
   int32_t max_kclass = -1;
@@ -183,15 +182,6 @@ void overlap_candidates(GraphBuild &b) {
   if (b.cand_node.empty()) b.cand_node.push_back(0);
   b.cand_cidx.resize(b.cand_ops.size());
   for (size_t k = 0; k < b.cand_ops.size(); ++k) b.cand_cidx[k] = b.n_cand ? b.cidx[b.cand_ops[k]] : 0;
-  b.cand_lvl.assign(b.Ls + 1, 0);
-  {
-    int64_t k = 0;
-    for (int64_t l = 0; l < b.Ls; ++l) {
-      b.cand_lvl[l] = k;
-      for (int64_t v = b.seg_node_off[b.seg_lvl_off[l]]; v < b.seg_node_off[b.seg_lvl_off[l + 1]]; ++v) k += b.cand_flag[v];
-    }
-    b.cand_lvl[b.Ls] = k;
-  }
   if (b.cand_ops.empty()) b.cand_ops.push_back(0);
   if (b.cand_cidx.empty()) b.cand_cidx.push_back(0);
 }
@@ -466,27 +456,6 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
     }
     b.seg_node_off[NSg] = i;
   }
-  // The segments of one level are independent, so a wide level may run as several
-  // consecutive steps: each step holds at most kStepNodes nodes and kStepSegments
-  // segments, so that two consecutive steps fit the shared-memory rings of the
-  // staged kernels (the numbering stays as it is).
-  {
-    std::vector<int64_t> off{0};
-    for (int64_t l = 0; l < Ls; ++l) {
-      int64_t t = b.seg_lvl_off[l];
-      while (t < b.seg_lvl_off[l + 1]) {
-        int64_t u = t + 1;  // one segment always fits (at most kMaxSegment nodes)
-        while (u < b.seg_lvl_off[l + 1] && u - t < kStepSegments &&
-               b.seg_node_off[u + 1] - b.seg_node_off[t] <= kStepNodes)
-          ++u;
-        off.push_back(u);
-        t = u;
-      }
-    }
-    b.seg_lvl_off = off;
-    Ls = (int64_t)off.size() - 1;
-    b.Ls = Ls;
-  }
   // Inputs of every segment head: its distinct predecessors over data and issue
   // order (each the tail of an earlier segment, as a chain only continues through
   // an op's single consumer), less any that is itself a direct predecessor of
@@ -608,17 +577,24 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
     for (; j < b.n_cq; ++j) b.cq_off[(size_t)r * b.n_cq + j + 1] = (int64_t)b.cq_ops.size();
   }
   if (b.cq_ops.empty()) b.cq_ops.push_back(0);
-  b.blk_words.assign(Ls, 0);
-  for (int64_t l = 0; l < Ls; ++l) {
-    int64_t w = 0;
-    for (int64_t t = b.seg_lvl_off[l]; t < b.seg_lvl_off[l + 1]; ++t) {
-      const int64_t nin = b.hin_off[t + 1] - b.hin_off[t];
-      if (nin > 0xFFFF) b.stageable = false;
-      bool cand = false;
-      for (int64_t v = b.seg_node_off[t]; v < b.seg_node_off[t + 1]; ++v) cand = cand || b.cand_flag[v];
-      w += 4 + nin + (cand ? 3 : 0);
-    }
-    b.blk_words[l] = (w + 3) & ~(int64_t)3;
+  b.seg_words.assign(NSg, 0);
+  for (int64_t t = 0; t < NSg; ++t) {
+    const int64_t nin = b.hin_off[t + 1] - b.hin_off[t];
+    if (nin > 0xFFFF) b.stageable = false;
+    bool cand = false;
+    for (int64_t v = b.seg_node_off[t]; v < b.seg_node_off[t + 1]; ++v) cand = cand || b.cand_flag[v];
+    b.seg_words[t] = 4 + nin + (cand ? 3 : 0);
+  }
+  // every input of a segment comes from an earlier level (the kernels' contract)
+  {
+    std::vector<int32_t> lvl(NSg, 0);
+    for (int64_t l = 0; l < Ls; ++l)
+      for (int64_t t = b.seg_lvl_off[l]; t < b.seg_lvl_off[l + 1]; ++t) lvl[t] = (int32_t)l;
+    for (int64_t t = 0; t < NSg; ++t)
+      for (int64_t q = b.hin_off[t]; q < b.hin_off[t + 1]; ++q)
+        if (lvl[b.seg_int[b.hin[q]]] >= lvl[t])
+          return fail(e, ECHO_E_BAD_GRAPH, "internal: segment %lld reads level %d from level %d", (long long)t,
+                      lvl[b.seg_int[b.hin[q]]], lvl[t]);
   }
   return ECHO_OK;
 }
@@ -628,25 +604,62 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
 // being composed and the one before it, which slower threads may still read);
 // whatever more they hold is prefetch look-ahead.  Preference: a larger duration
 // ring, then a larger value ring (more predecessors served from shared memory).
-echo::StagedPlan plan_staged(const GraphBuild &b, int sigma, size_t smem_cap) {
+// The steps of the staged kernels for scenario blocks of `sigma`.  The segments of
+// one level are independent, so a wide level may run as several consecutive
+// steps: each step holds at most `cap` nodes and kStepSegments segments, so that
+// two consecutive steps fit the shared-memory rings (the numbering stays as it is).
+struct Steps {
+  int64_t L = 0;
+  std::vector<int64_t> off;    // [L+1] segments of each step
+  std::vector<int64_t> words;  // [L] record block words (padded to 4)
+  std::vector<int64_t> cand;   // [L+1] first level-order candidate of each step
+};
+
+Steps make_steps(const GraphBuild &b, int64_t cap) {
+  Steps st;
+  st.off.assign(1, 0);
+  for (int64_t l = 0; l < b.Ls; ++l) {
+    int64_t t = b.seg_lvl_off[l];
+    while (t < b.seg_lvl_off[l + 1]) {
+      int64_t u = t + 1;  // one segment always fits (at most kMaxSegment nodes)
+      while (u < b.seg_lvl_off[l + 1] && u - t < kStepSegments && b.seg_node_off[u + 1] - b.seg_node_off[t] <= cap)
+        ++u;
+      st.off.push_back(u);
+      t = u;
+    }
+  }
+  st.L = (int64_t)st.off.size() - 1;
+  st.words.assign(st.L, 0);
+  st.cand.assign(st.L + 1, b.n_cand);
+  for (int64_t l = 0; l < st.L; ++l) {
+    int64_t w = 0;
+    for (int64_t t = st.off[l]; t < st.off[l + 1]; ++t) w += b.seg_words[t];
+    st.words[l] = (w + 3) & ~(int64_t)3;
+    const int32_t first = (int32_t)b.seg_node_off[st.off[l]];
+    st.cand[l] = std::lower_bound(b.cand_node.begin(), b.cand_node.begin() + b.n_cand, first) - b.cand_node.begin();
+  }
+  return st;
+}
+
+echo::StagedPlan plan_staged(const GraphBuild &b, const Steps &st, int sigma, size_t smem_cap) {
   echo::StagedPlan best;
-  if (!b.stageable || b.Ls == 0) return best;
+  if (!b.stageable || st.L == 0) return best;
   auto pow2 = [](int64_t x) {
     int k = 0;
     while (((int64_t)1 << k) < x) ++k;
     return k;
   };
   int64_t rows2 = 0, words2 = 0, segmax = 0, prow = 0, pword = 0, crows2 = 0, pcand = 0;
-  for (int64_t l = 0; l < b.Ls; ++l) {
-    const int64_t r = b.seg_node_off[b.seg_lvl_off[l + 1]] - b.seg_node_off[b.seg_lvl_off[l]];
-    const int64_t nc = b.cand_lvl[l + 1] - b.cand_lvl[l];
+  for (int64_t l = 0; l < st.L; ++l) {
+    const int64_t r = b.seg_node_off[st.off[l + 1]] - b.seg_node_off[st.off[l]];
+    const int64_t nc = st.cand[l + 1] - st.cand[l];
     crows2 = std::max(crows2, nc + pcand);
     pcand = nc;
     rows2 = std::max(rows2, r + prow);
-    words2 = std::max(words2, b.blk_words[l] + pword);
-    segmax = std::max(segmax, b.seg_lvl_off[l + 1] - b.seg_lvl_off[l]);
+    words2 = std::max(words2, st.words[l] + pword);
+    segmax = std::max(segmax, st.off[l + 1] - st.off[l]);
     prow = r;
-    pword = b.blk_words[l];
+    pword = st.words[l];
   }
   const int dmin = std::max(pow2(rows2), 4), rmin = std::max(pow2(words2), 4);
   const int cring = std::max(pow2(crows2), 4);  // candidate ring: two levels' candidates
@@ -672,21 +685,21 @@ echo::StagedPlan plan_staged(const GraphBuild &b, int sigma, size_t smem_cap) {
 // ring of 2^vlog2 segments, and the per-level metadata (word offset of the block,
 // first node, first segment).  A head's inputs recent enough to be in the value
 // ring become byte offsets of their slots, the others node ids.
-void build_records(const GraphBuild &b, int sigma, int vlog2, std::vector<uint32_t> &recs,
+void build_records(const GraphBuild &b, const Steps &stp, int sigma, int vlog2, std::vector<uint32_t> &recs,
                    std::vector<uint32_t> &meta) {
   const int64_t R = (int64_t)1 << vlog2;
   const uint32_t row = (uint32_t)sigma * 8;
   recs.clear();
-  meta.assign(4 * (b.Ls + 1), 0);
+  meta.assign(4 * (stp.L + 1), 0);
   std::vector<uint32_t> far;
-  for (int64_t l = 0; l < b.Ls; ++l) {
-    const int64_t s0 = b.seg_lvl_off[l], s1 = b.seg_lvl_off[l + 1];
+  for (int64_t l = 0; l < stp.L; ++l) {
+    const int64_t s0 = stp.off[l], s1 = stp.off[l + 1];
     const int64_t i0 = b.seg_node_off[s0];
     const size_t base = recs.size();
     meta[4 * l] = (uint32_t)base;
     meta[4 * l + 1] = (uint32_t)i0;
     meta[4 * l + 2] = (uint32_t)s0;
-    meta[4 * l + 3] = (uint32_t)b.cand_lvl[l];
+    meta[4 * l + 3] = (uint32_t)stp.cand[l];
     recs.resize(base + 4 * (s1 - s0), 0);
     for (int64_t t = s0; t < s1; ++t) {
       const int64_t h = b.seg_node_off[t], z = b.seg_node_off[t + 1] - 1;
@@ -727,10 +740,10 @@ void build_records(const GraphBuild &b, int sigma, int vlog2, std::vector<uint32
     }
     while (recs.size() % 4) recs.push_back(0);
   }
-  meta[4 * b.Ls] = (uint32_t)recs.size();
-  meta[4 * b.Ls + 1] = (uint32_t)b.V;
-  meta[4 * b.Ls + 2] = (uint32_t)b.n_seg;
-  meta[4 * b.Ls + 3] = (uint32_t)b.cand_lvl[b.Ls];
+  meta[4 * stp.L] = (uint32_t)recs.size();
+  meta[4 * stp.L + 1] = (uint32_t)b.V;
+  meta[4 * stp.L + 2] = (uint32_t)b.n_seg;
+  meta[4 * stp.L + 3] = (uint32_t)stp.cand[stp.L];
   if (recs.empty()) recs.assign(4, 0);
 }
 
@@ -783,6 +796,7 @@ struct echo_ctx {
   uint8_t *ov = nullptr;
   uint32_t *d_recs = nullptr, *d_meta = nullptr;
   echo::StagedPlan plan;
+  Steps steps;  // composition steps of the staged kernels
   uint32_t rec_words = 0;
   std::vector<double> h_sums, h_maxsf;
   int final_f = 0;
@@ -1152,21 +1166,26 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     if (const char *e = std::getenv("ECHO_STAGED_THREADS")) threads = std::atoi(e);
     if (const char *e = std::getenv("ECHO_BLOCKS_PER_SM")) bps = std::max(1, std::atoi(e));
     const size_t cap = std::min((size_t)std::max(optin - 1024, 0), (size_t)(per_sm / bps) - 1024);
-    c->plan = plan_staged(B, sigma, cap);
+    // the widest steps whose rings fit
+    for (int64_t step_cap = kStepNodes;; step_cap /= 2) {
+      c->steps = make_steps(B, step_cap);
+      c->plan = plan_staged(B, c->steps, sigma, cap);
+      if (c->plan.ok || step_cap <= 2 * echo::kMaxSegment) break;
+    }
+    const Steps &st = c->steps;
     c->plan.threads = threads;
     if (c->plan.ok) {
-      // the pipelined kernel moves whole rows of even width and arms each level's
+      // the pipelined kernel moves whole rows of even width and arms each step's
       // byte count on one mbarrier (transaction counts stay below 2^20)
       int64_t max_bytes = 0;
-      for (int64_t l = 0; l < B.Ls; ++l) {
-        const int64_t rows = B.seg_node_off[B.seg_lvl_off[l + 1]] - B.seg_node_off[B.seg_lvl_off[l]];
-        max_bytes = std::max(max_bytes, rows * sigma * 8 + B.blk_words[l] * 4 + 32 +
-                                            (B.cand_lvl[l + 1] - B.cand_lvl[l]) * sigma * 8);
+      for (int64_t l = 0; l < st.L; ++l) {
+        const int64_t rows = B.seg_node_off[st.off[l + 1]] - B.seg_node_off[st.off[l]];
+        max_bytes = std::max(max_bytes, rows * sigma * 8 + st.words[l] * 4 + 32 + (st.cand[l + 1] - st.cand[l]) * sigma * 8);
       }
       c->plan.pipelined = sigma % 2 == 0 && max_bytes < (1 << 20);
       std::vector<uint32_t> recs, meta;
-      build_records(B, sigma, c->plan.vring_log2, recs, meta);
-      c->rec_words = meta[4 * B.Ls];
+      build_records(B, st, sigma, c->plan.vring_log2, recs, meta);
+      c->rec_words = meta[4 * st.L];
       if ((rc = upload(c, o, &c->d_recs, recs)) || (rc = upload(c, o, &c->d_meta, meta))) {
         free_all(c->scen_allocs);
         return rc;
@@ -1279,7 +1298,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     if (c->plan.ok && c->kernel_choice != 1) {
       echo::StagedArgs a{};
       a.S = c->S;
-      a.L = (int32_t)B.Ls;
+      a.L = (int32_t)c->steps.L;
       a.n_rows = (uint32_t)B.V;
       a.n_words = c->rec_words;
       a.vlog2 = c->plan.vring_log2;
