@@ -52,7 +52,7 @@ class _Scen(C.Structure):
                 ("lat_intra", C.c_void_p), ("bw_inter", C.c_void_p), ("lat_inter", C.c_void_p),
                 ("delta", C.c_void_p), ("slowdown", C.c_void_p),
                 ("chunk_max_bytes", C.c_void_p), ("chunk_bytes", C.c_void_p), ("cc_model", C.c_int32),
-                ("overlap_model", C.c_int32)]
+                ("overlap_model", C.c_int32), ("comm_interval", C.c_int32)]
 
 
 def _load():
@@ -119,11 +119,13 @@ class OracleResult:
 
 def compose(g, sc, refine_passes: int = 1, tie_seed: int = 0, threads: int = 1,
             want_cc: bool = True, want_overlap: bool = True, cc_model: int = 0,
-            overlap_model: int = 0) -> OracleResult:
+            overlap_model: int = 0, comm_interval: int = 0) -> OracleResult:
     """Compose every scenario of ``sc`` on graph ``g`` (workloads.Graph/Scenarios).
     cc_model 0 takes collective times from Eqs. 2-5, 1 from the alpha-beta model.
     overlap_model 0 slows an overlapped kernel to d * factor, 1 to
-    d + (factor - 1) * (length of its overlap with the rank's communication)."""
+    d + (factor - 1) * (length of its overlap with the rank's communication).
+    comm_interval 0 takes a comm op's execution interval [start, finish) on each
+    member rank, 1 the interval from the rank's own launch of it to its finish."""
     lib = _load()
     V, S = g.n_ops, sc.n_scen
     keep = []
@@ -144,7 +146,8 @@ def compose(g, sc, refine_passes: int = 1, tie_seed: int = 0, threads: int = 1,
                arr(sc.bw_inter, np.float64), arr(sc.lat_inter, np.float64), arr(sc.delta, np.float64),
                arr(sc.slowdown, np.float64),
                arr(sc.chunk_max_bytes, np.int64) if n_chunk else None,
-               arr(sc.chunk_bytes, np.int64) if n_chunk else None, int(cc_model), int(overlap_model))
+               arr(sc.chunk_bytes, np.int64) if n_chunk else None, int(cc_model), int(overlap_model),
+               int(comm_interval))
     start = np.zeros((V, S), np.int64)
     finish = np.zeros((V, S), np.int64)
     mk = np.zeros(S, np.int64)

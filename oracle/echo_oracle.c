@@ -27,7 +27,9 @@
  *   time is int64 ns, sources start at 0; a rank has any number of serial streams
  *   (its compute timeline plus comm/memcpy timelines); overlap means
  *   a positive-length intersection of [start, finish) intervals and slows the
- *   whole kernel; the bare "(N-1)" inside Eqs. 3-4 is read as a per-step latency,
+ *   whole kernel (variants: only the overlapped length is slowed; a comm op's
+ *   interval on rank r opens when r has launched it, the latest finish among its
+ *   launch conditions on r, rather than when the last member has); the bare "(N-1)" inside Eqs. 3-4 is read as a per-step latency,
  *   so every ring step costs L + p/B; send/recv costs eta chunk transfers over the
  *   intra- or inter-node link; AUTO all-reduce takes the faster of ring and tree
  *   (ties to ring); N = 1 or 0 bytes costs 0; slowed duration = rint(d * factor).
@@ -309,13 +311,14 @@ int oracle_compose(const oracle_graph *g, const oracle_scen *sc, int32_t s0, int
   int64_t *clo = malloc((size_t)(QE > 0 ? QE : 1) * sizeof(int64_t)); /* clipped to one kernel */
   int64_t *chi = malloc((size_t)(QE > 0 ? QE : 1) * sizeof(int64_t));
   int64_t *olen = calloc((size_t)(V > 0 ? V : 1), sizeof(int64_t)); /* overlapped length */
+  uint8_t *onr = calloc((size_t)(V > 0 ? V : 1), 1); /* op runs on the rank at hand */
   int32_t G = g->n_groups;
   int32_t *gN = calloc((size_t)(G > 0 ? G : 1), sizeof(int32_t));
   int32_t *gM = calloc((size_t)(G > 0 ? G : 1), sizeof(int32_t));
   int32_t *gK = calloc((size_t)(G > 0 ? G : 1), sizeof(int32_t));
   double *glg = calloc((size_t)(G > 0 ? G : 1), sizeof(double));
   if (!sim.succ_off || !sim.succ_idx || !sim.opq_off || !sim.opq_q || !sim.opq_pos || !sim.cnt ||
-      !sim.heap || !fill || !d0 || !d || !st || !fn || !ov || !cst || !cfn || !clo || !chi || !olen || !gN || !gM ||
+      !sim.heap || !fill || !d0 || !d || !st || !fn || !ov || !cst || !cfn || !clo || !chi || !olen || !onr || !gN || !gM ||
       !gK || !glg) {
     rc = ORACLE_E_NOMEM;
     goto out;
@@ -383,14 +386,28 @@ int oracle_compose(const oracle_graph *g, const oracle_scen *sc, int32_t s0, int
        * with positive length, the interval of any comm op that rank r takes part in */
       for (int32_t r = 0; r < g->n_ranks; ++r) {
         int64_t qa = (int64_t)g->n_streams * r, qb = qa + g->n_streams, nc = 0;
-        for (int64_t j = g->q_off[qa]; j < g->q_off[qb]; ++j) {
-          int32_t w = g->q_ops[j];
-          if (g->kind[w] == K_COLL || g->kind[w] == K_P2P) {
-            cst[nc] = st[w];
+        for (int64_t j = g->q_off[qa]; j < g->q_off[qb]; ++j) onr[g->q_ops[j]] = 1;
+        for (int64_t q = qa; q < qb; ++q)
+          for (int64_t j = g->q_off[q]; j < g->q_off[q + 1]; ++j) {
+            int32_t w = g->q_ops[j];
+            if (g->kind[w] != K_COLL && g->kind[w] != K_P2P) continue;
+            if (sc->comm_interval == 1) {
+              /* rank r has launched w once the op before it on this timeline and
+               * its data producers that run on r have finished */
+              int64_t t = 0;
+              if (j > g->q_off[q] && fn[g->q_ops[j - 1]] > t) t = fn[g->q_ops[j - 1]];
+              for (int64_t e = g->pred_off[w]; e < g->pred_off[w + 1]; ++e) {
+                int32_t u = g->pred_idx[e];
+                if (onr[u] && fn[u] > t) t = fn[u];
+              }
+              cst[nc] = t;
+            } else {
+              cst[nc] = st[w];
+            }
             cfn[nc] = fn[w];
             nc++;
           }
-        }
+        for (int64_t j = g->q_off[qa]; j < g->q_off[qb]; ++j) onr[g->q_ops[j]] = 0;
         for (int64_t i = g->q_off[qa]; i < g->q_off[qb]; ++i) {
           int32_t v = g->q_ops[i];
           if (g->kind[v] != K_COMPUTE) continue;
@@ -453,6 +470,7 @@ out:
   free(clo);
   free(chi);
   free(olen);
+  free(onr);
   free(gN);
   free(gM);
   free(gK);

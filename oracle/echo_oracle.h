@@ -35,6 +35,10 @@ typedef struct {
   int32_t cc_model; /* 0: Eqs. 2-5 (white box), 1: alpha-beta */
   int32_t overlap_model; /* 0: an overlapped kernel takes d * factor;
                             1: d + (factor - 1) * (length of its overlap) */
+  int32_t comm_interval; /* what counts as a comm op's interval on a member rank r:
+                            0: its execution [start, finish);
+                            1: [launch on r, finish), launch = when r's own launch
+                               conditions of it hold */
 } oracle_scen;
 
 int64_t oracle_chunk_bytes(int64_t nbytes, int n_chunk, const int64_t *max_bytes,

@@ -157,9 +157,30 @@ def op_ranks(g: W.Graph):
     return out
 
 
-def brute_compose(g: W.Graph, sc: W.Scenarios, s: int, refine_passes: int, cc_fn):
+def launch_preds(g: W.Graph):
+    """{(comm op w, member rank r): the ops whose finish rank r waits for before it
+    launches w}: the op just before w on r's timeline that holds w, and w's data
+    producers that run on r."""
+    ranks = op_ranks(g)
+    out = {}
+    for q in range(len(g.q_off) - 1):
+        r = q // g.n_streams
+        ops = g.q_ops[g.q_off[q]:g.q_off[q + 1]].tolist()
+        for k, w in enumerate(ops):
+            if g.kind[w] not in (W.KIND_COLL, W.KIND_P2P):
+                continue
+            ps = {u for u in g.pred_idx[g.pred_off[w]:g.pred_off[w + 1]].tolist() if r in ranks[u]}
+            if k > 0:
+                ps.add(ops[k - 1])
+            out[(w, r)] = ps
+    return out
+
+
+def brute_compose(g: W.Graph, sc: W.Scenarios, s: int, refine_passes: int, cc_fn, comm_interval: int = 0):
     """Brute-force reference of one scenario: CC durations from ``cc_fn`` (pinned on
-    its own), composition by path enumeration, overlap by checking every pair."""
+    its own), composition by path enumeration, overlap by checking every pair.  A
+    comm op's interval on rank r starts at its start (comm_interval 0) or when r
+    has launched it (1: the latest finish among ``launch_preds``)."""
     V = g.n_ops
     d0 = np.zeros(V, np.int64)
     for v in range(V):
@@ -172,6 +193,7 @@ def brute_compose(g: W.Graph, sc: W.Scenarios, s: int, refine_passes: int, cc_fn
         else:
             d0[v] = sc.dur[v, s]
     ranks = op_ranks(g)
+    lp = launch_preds(g)
     d = d0.copy()
     fin = brute_finish(g, d)
     ov = np.zeros(V, np.uint8)
@@ -182,8 +204,9 @@ def brute_compose(g: W.Graph, sc: W.Scenarios, s: int, refine_passes: int, cc_fn
                 continue
             hit = 0
             for w in range(V):
-                if g.kind[w] in (W.KIND_COLL, W.KIND_P2P) and ranks[v] & ranks[w]:
-                    if max(st[v], st[w]) < min(fin[v], fin[w]):
+                for r in ranks[v] & ranks[w] if g.kind[w] in (W.KIND_COLL, W.KIND_P2P) else ():
+                    lo = st[w] if comm_interval == 0 else max([0] + [int(fin[u]) for u in lp[(w, r)]])
+                    if max(st[v], lo) < min(fin[v], fin[w]):
                         hit = 1
             ov[v] = hit
         d = d0.copy()

@@ -282,6 +282,82 @@ def test_proportional_model_never_exceeds_whole_kernel_model():
         assert ((b.finish - b.start)[comp] <= (a.finish - a.start)[comp]).all()
 
 
+def _launch_case(d_b):
+    """Rank 0 runs kernels a (10 ns) then b; rank 1 runs kernel c (200 ns).  An
+    all-reduce of ranks 0 and 1 needs a's and c's outputs: 500 B at 10 B/ns, no
+    setup, latency or reduction cost, so it runs [200, 250).  Rank 0 has launched
+    it at 10, rank 1 at 200."""
+    ops = [{"kind": W.KIND_COMPUTE, "kclass": 0}, {"kind": W.KIND_COMPUTE, "kclass": 0},
+           {"kind": W.KIND_COMPUTE, "kclass": 0},
+           {"kind": W.KIND_COLL, "group": 0, "cc_type": W.CC_ALLREDUCE, "cc_algo": W.ALGO_RING,
+            "cc_bytes": 500, "preds": [0, 2]}]
+    queues = {(0, 0): [0, 1], (1, 0): [2], (0, 1): [3], (1, 1): [3]}
+    g = SG.graph_from_lists(2, 2, ops, queues, [[0, 1]], gpus_per_node=2)
+    dur = np.array([[10], [d_b], [200], [0]], np.int64)
+    sc = W.Scenarios(dur=dur, alpha_ns=np.zeros(1), bw_intra=np.full(1, 10.0), lat_intra=np.zeros(1),
+                     bw_inter=np.full(1, 10.0), lat_inter=np.zeros(1), delta=np.zeros(1),
+                     slowdown=np.full((1, 1), 1.5), peak_flop_per_ns=np.ones(1))
+    return g, sc
+
+
+def test_launch_interval_by_hand():
+    g, sc = _launch_case(100)
+    r = oracle.compose(g, sc, refine_passes=1, comm_interval=0)
+    assert (r.start[3, 0], r.finish[3, 0]) == (200, 250)
+    assert r.overlapped[:, 0].tolist() == [0, 0, 0, 0]  # b runs [10, 110)
+    for model in (0, 1):
+        r = oracle.compose(g, sc, refine_passes=1, overlap_model=model, comm_interval=1)
+        # on rank 0 the all-reduce holds [10, 250): b overlaps it over its whole length;
+        # on rank 1 it holds [200, 250), which only touches c
+        assert r.overlapped[:, 0].tolist() == [0, 1, 0, 0]
+        assert r.finish[1, 0] - r.start[1, 0] == 150  # 100 * 1.5 = 100 + 0.5 * 100
+    g, sc = _launch_case(300)  # b runs [10, 310)
+    assert oracle.compose(g, sc, overlap_model=1, comm_interval=0).finish[1, 0] == 10 + 325  # 300 + 0.5 * 50
+    assert oracle.compose(g, sc, overlap_model=1, comm_interval=1).finish[1, 0] == 10 + 420  # 300 + 0.5 * 240
+    assert oracle.compose(g, sc, overlap_model=0, comm_interval=1).finish[1, 0] == 10 + 450
+
+
+def test_launch_interval_on_one_rank_is_the_execution_interval():
+    # with one rank every launch condition of a comm op is that rank's, so it
+    # launches exactly when it starts
+    rng = np.random.default_rng(37)
+    for _ in range(200):
+        g = SG.random_graph(rng, int(rng.integers(2, 30)), max_ranks=1, max_streams=4, p_edge=0.1)
+        sc = SG.random_scenarios(rng, g, 3, max_dur=40)
+        for model in (0, 1):
+            a = oracle.compose(g, sc, refine_passes=2, overlap_model=model, comm_interval=0)
+            b = oracle.compose(g, sc, refine_passes=2, overlap_model=model, comm_interval=1)
+            assert np.array_equal(a.finish, b.finish) and np.array_equal(a.overlapped, b.overlapped)
+
+
+def test_launch_interval_only_adds_overlaps():
+    # the same first composition, and every launch interval holds the execution one
+    rng = np.random.default_rng(41)
+    grew = 0
+    for _ in range(300):
+        g = SG.random_graph(rng, int(rng.integers(2, 30)), max_ranks=3, max_streams=4, p_edge=0.1)
+        sc = SG.random_scenarios(rng, g, 3, max_dur=40)
+        a = oracle.compose(g, sc, refine_passes=1, comm_interval=0)
+        b = oracle.compose(g, sc, refine_passes=1, comm_interval=1)
+        assert (b.overlapped >= a.overlapped).all()
+        grew += int((b.overlapped > a.overlapped).any())
+    assert grew > 10  # the variant does change decisions on multi-rank graphs
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_brute_force_launch_intervals(seed):
+    rng = np.random.default_rng(2000 + seed)
+    for case in range(400):
+        g = SG.random_graph(rng, int(rng.integers(1, 11)))
+        sc = SG.random_scenarios(rng, g, 2)
+        for passes in (1, 2):
+            r = oracle.compose(g, sc, refine_passes=passes, comm_interval=1)
+            for s in range(sc.n_scen):
+                st, fn, ov = SG.brute_compose(g, sc, s, passes, oracle.cc_ns, comm_interval=1)
+                assert (r.finish[:, s] == fn).all(), (seed, case, passes)
+                assert (r.overlapped[:, s] == ov).all(), (seed, case, passes)
+
+
 def test_auto_takes_the_faster_algorithm():
     rng = np.random.default_rng(13)
     for _ in range(300):
