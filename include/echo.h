@@ -143,8 +143,16 @@ typedef struct {
    * without overlapping communication); ECHO_OVERLAP_PROPORTIONAL adds (factor - 1)
    * times the length of its interval covered by its rank's comm intervals. */
   int32_t overlap_model;
+  /* the interval of a comm op on a member rank r that the validator tests:
+   * ECHO_COMM_EXECUTION (default) its execution [start, finish), the same on every
+   * member (Sec. 5.2: it starts once the last member has launched it);
+   * ECHO_COMM_LAUNCH [launch on r, finish), where r has launched it once the op
+   * before it on r's timeline and its data producers that run on r have finished:
+   * the comm kernel is resident on r while it waits for the other members. */
+  int32_t comm_interval;
 } echo_compose_opts;
 enum { ECHO_OVERLAP_WHOLE = 0, ECHO_OVERLAP_PROPORTIONAL = 1 };
+enum { ECHO_COMM_EXECUTION = 0, ECHO_COMM_LAUNCH = 1 };
 
 /* Create a context on `device`, enqueuing on `cuda_stream` (a cudaStream_t; NULL =
  * a new non-blocking stream owned by the context; the legacy default stream is

@@ -72,6 +72,8 @@ struct GraphBuild {
   int32_t n_cq = 0;                   // comm timelines per rank in cq_off (max over ranks)
   std::vector<int64_t> cq_off;        // [R*n_cq+1] comm ops of each (rank, comm timeline)
   std::vector<int32_t> cq_ops;        // internal ids, in issue order
+  std::vector<int32_t> lq_off;        // [cq_ops+1] launch conditions of each cq_ops entry on its rank
+  std::vector<int32_t> lq_ops;        // (internal ids; the latest one on each of the rank's timelines)
   std::vector<int64_t> seg_words;     // [n_seg] record words of each segment
   std::vector<int64_t> hin_off;       // [n_seg+1] inputs of each segment's head
   std::vector<int32_t> hin;           // (internal ids, each the tail of an earlier segment)
@@ -564,19 +566,54 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
     }
     b.n_cq = std::max(b.n_cq, n);
   }
+  // With each entry, the ops whose finish its rank waits for before it launches
+  // the comm op (for the validator variant that counts a comm op's interval on a
+  // rank from that rank's launch): the op before it on its timeline and its data
+  // producers that run on the rank.  A timeline is serial, so only the latest of
+  // them on each of the rank's timelines is kept.
   b.cq_off.assign((size_t)R * b.n_cq + 1, 0);
-  for (int32_t r = 0; r < R; ++r) {
-    int32_t j = 0;
-    for (int32_t k = 1; k < NS; ++k) {
-      const int64_t q = (int64_t)r * NS + k;
-      const size_t before = b.cq_ops.size();
-      for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i)
-        if (b.is_comm[b.q_ops_int[i]]) b.cq_ops.push_back(b.q_ops_int[i]);
-      if (b.cq_ops.size() > before) b.cq_off[(size_t)r * b.n_cq + ++j] = (int64_t)b.cq_ops.size();
+  b.lq_off.assign(1, 0);
+  b.lq_ops.clear();
+  {
+    std::vector<int32_t> tl(V, -1);  // timeline of an op of the rank at hand
+    std::vector<int64_t> tpos(V, 0), best(NS);
+    for (int32_t r = 0; r < R; ++r) {
+      for (int32_t k = 0; k < NS; ++k)
+        for (int64_t i = g->q_off[(int64_t)r * NS + k]; i < g->q_off[(int64_t)r * NS + k + 1]; ++i) {
+          tl[b.q_ops_int[i]] = k;
+          tpos[b.q_ops_int[i]] = i;
+        }
+      int32_t j = 0;
+      for (int32_t k = 1; k < NS; ++k) {
+        const int64_t q = (int64_t)r * NS + k;
+        const size_t before = b.cq_ops.size();
+        for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i) {
+          const int32_t w = b.q_ops_int[i];
+          if (!b.is_comm[w]) continue;
+          b.cq_ops.push_back(w);
+          std::fill(best.begin(), best.end(), -1);
+          if (i > g->q_off[q]) best[k] = i - 1;
+          for (int64_t e = b.dp_off[w]; e < b.dp_off[w + 1]; ++e) {
+            const int32_t u = b.dp[e];
+            if (tl[u] >= 0) best[tl[u]] = std::max(best[tl[u]], tpos[u]);
+          }
+          for (int32_t kk = 0; kk < NS; ++kk)
+            if (best[kk] >= 0) b.lq_ops.push_back(b.q_ops_int[best[kk]]);
+          b.lq_off.push_back((int32_t)b.lq_ops.size());
+        }
+        if (b.cq_ops.size() > before) b.cq_off[(size_t)r * b.n_cq + ++j] = (int64_t)b.cq_ops.size();
+      }
+      for (; j < b.n_cq; ++j) b.cq_off[(size_t)r * b.n_cq + j + 1] = (int64_t)b.cq_ops.size();
+      for (int32_t k = 0; k < NS; ++k)
+        for (int64_t i = g->q_off[(int64_t)r * NS + k]; i < g->q_off[(int64_t)r * NS + k + 1]; ++i)
+          tl[b.q_ops_int[i]] = -1;
     }
-    for (; j < b.n_cq; ++j) b.cq_off[(size_t)r * b.n_cq + j + 1] = (int64_t)b.cq_ops.size();
   }
-  if (b.cq_ops.empty()) b.cq_ops.push_back(0);
+  if (b.cq_ops.empty()) {
+    b.cq_ops.push_back(0);
+    b.lq_off.push_back(0);
+  }
+  if (b.lq_ops.empty()) b.lq_ops.push_back(0);
   b.seg_words.assign(NSg, 0);
   for (int64_t t = 0; t < NSg; ++t) {
     const int64_t nin = b.hin_off[t + 1] - b.hin_off[t];
@@ -768,7 +805,7 @@ struct echo_ctx {
   // device graph
   int64_t *seg_lvl_off = nullptr, *seg_node_off = nullptr, *nq_off = nullptr, *dp_off = nullptr, *q_off = nullptr;
   int64_t *ov_chunks = nullptr, *cq_off = nullptr;
-  int32_t *cq_ops = nullptr;
+  int32_t *cq_ops = nullptr, *lq_off = nullptr, *lq_ops = nullptr;
   int64_t *cand_off = nullptr;
   int32_t *cand_ops = nullptr;
   uint8_t *cand_flag = nullptr;
@@ -1075,6 +1112,7 @@ int echo_load_graph(echo_ctx *c, const echo_graph_desc *g) {
   if ((rc = upload(c, o, &c->seg_lvl_off, B.seg_lvl_off)) || (rc = upload(c, o, &c->seg_node_off, B.seg_node_off)) ||
       (rc = upload(c, o, &c->ov_chunks, B.ov_chunks)) ||
       (rc = upload(c, o, &c->cq_off, B.cq_off)) || (rc = upload(c, o, &c->cq_ops, B.cq_ops)) ||
+      (rc = upload(c, o, &c->lq_off, B.lq_off)) || (rc = upload(c, o, &c->lq_ops, B.lq_ops)) ||
       (rc = upload(c, o, &c->cand_off, B.cand_off)) || (rc = upload(c, o, &c->cand_ops, B.cand_ops)) ||
       (rc = upload(c, o, &c->cand_flag, B.cand_flag)) || (rc = upload(c, o, &c->cand_cidx, B.cand_cidx)) ||
       (rc = upload(c, o, &c->cidx, B.cidx)) || (rc = upload(c, o, &c->cand_node, B.cand_node)) ||
@@ -1280,6 +1318,9 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   const int32_t model = opts ? opts->overlap_model : ECHO_OVERLAP_WHOLE;
   if (model != ECHO_OVERLAP_WHOLE && model != ECHO_OVERLAP_PROPORTIONAL)
     return set_err(c, ECHO_E_INVALID_ARG, "unknown overlap model");
+  const int32_t civ = opts ? opts->comm_interval : ECHO_COMM_EXECUTION;
+  if (civ != ECHO_COMM_EXECUTION && civ != ECHO_COMM_LAUNCH)
+    return set_err(c, ECHO_E_INVALID_ARG, "unknown comm interval");
   const GraphBuild &B = c->gb;
   // the pipelined kernel reads the validator's durations of the candidates from a
   // ring of its own; the others compose from a full matrix built for them
@@ -1355,6 +1396,8 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     o.n_cq = B.n_cq;
     o.cq_off = c->cq_off;
     o.cq_ops = c->cq_ops;
+    o.lq_off = civ == ECHO_COMM_LAUNCH ? c->lq_off : nullptr;
+    o.lq_ops = c->lq_ops;
     o.kcl = c->kcl;
     o.f = c->f[(p - 1) % 2];
     o.dur = c->dur;

@@ -140,6 +140,9 @@ struct OverlapArgs {
   const int64_t *cand_off; const int32_t *cand_ops;  // [R+1]: each rank's overlap candidates, in issue order
   const int32_t *cand_cidx;                          // level-order index of each entry of cand_ops
   const int64_t *cq_off; const int32_t *cq_ops;  // [R*n_cq+1]: comm ops of each (rank, comm timeline)
+  // launch conditions of each entry of cq_ops on its rank (CSR); null: a comm op's
+  // interval is its execution [start, finish), else [latest of them, finish)
+  const int32_t *lq_off, *lq_ops;
   const uint8_t *kcl;      // [V]
   const int64_t *f;        // finish times of the last pass
   const int64_t *dur;      // original durations

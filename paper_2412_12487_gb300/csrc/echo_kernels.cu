@@ -1,6 +1,7 @@
 // echo_kernels.cu -- sm_103a kernels of the CC estimator, the validator and the
 // readbacks.  All floating point that decides an integer is written with explicit
 // round-to-nearest intrinsics (no contraction), so results do not depend on -fmad.
+#include <type_traits>
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -230,7 +231,9 @@ __global__ void permute_rows_kernel(const T *__restrict__ raw, const int32_t *__
 // ---------------------------------------------------------------------------------
 constexpr int kOverlapThreads = 128;
 constexpr int kOverlapBatch = 8;  // divides 32 (the shuffled op list's width)
-template <int NCMAX>
+// LAUNCH: a comm op's interval on the rank opens at the rank's launch of it
+// (a.lq_off), else at its start
+template <int NCMAX, bool LAUNCH>
 __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a) {
   const int32_t S = a.S;
   const int32_t s = blockIdx.x * blockDim.x + threadIdx.x;
@@ -264,7 +267,13 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
     if (cur[j] < end[j]) {
       const int64_t w = a.cq_ops[cur[j]];
       fw[j] = f[w << sh];
-      sw[j] = fw[j] - du[w << sh];
+      if (LAUNCH) {  // from the rank's launch: its launch conditions' latest finish
+        int64_t t = 0;
+        for (int32_t k = a.lq_off[cur[j]]; k < a.lq_off[cur[j] + 1]; ++k) t = max(t, f[(int64_t)a.lq_ops[k] << sh]);
+        sw[j] = t;
+      } else {
+        sw[j] = fw[j] - du[w << sh];
+      }
     } else {
       sw[j] = fw[j] = INT64_MAX;
     }
@@ -508,18 +517,25 @@ cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
   int64_t gy = a.n_chunks < 65535 ? a.n_chunks : 65535;
   int64_t gz = (a.n_chunks + gy - 1) / gy;
   dim3 grid((a.S + tx - 1) / tx, (unsigned)gy, (unsigned)gz);
-  if (a.n_cq <= 1)
-    overlap_kernel<1><<<grid, tx, 0, st>>>(a);
-  else if (a.n_cq <= 2)
-    overlap_kernel<2><<<grid, tx, 0, st>>>(a);
-  else if (a.n_cq <= 3)
-    overlap_kernel<3><<<grid, tx, 0, st>>>(a);
-  else if (a.n_cq <= 4)
-    overlap_kernel<4><<<grid, tx, 0, st>>>(a);
-  else if (a.n_cq <= 8)
-    overlap_kernel<8><<<grid, tx, 0, st>>>(a);
+  auto go = [&](auto launch) {
+    constexpr bool L = decltype(launch)::value;
+    if (a.n_cq <= 1)
+      overlap_kernel<1, L><<<grid, tx, 0, st>>>(a);
+    else if (a.n_cq <= 2)
+      overlap_kernel<2, L><<<grid, tx, 0, st>>>(a);
+    else if (a.n_cq <= 3)
+      overlap_kernel<3, L><<<grid, tx, 0, st>>>(a);
+    else if (a.n_cq <= 4)
+      overlap_kernel<4, L><<<grid, tx, 0, st>>>(a);
+    else if (a.n_cq <= 8)
+      overlap_kernel<8, L><<<grid, tx, 0, st>>>(a);
+    else
+      overlap_kernel<kMaxStreams, L><<<grid, tx, 0, st>>>(a);
+  };
+  if (a.lq_off)
+    go(std::true_type{});
   else
-    overlap_kernel<kMaxStreams><<<grid, tx, 0, st>>>(a);
+    go(std::false_type{});
   return cudaGetLastError();
 }
 

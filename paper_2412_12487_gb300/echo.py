@@ -36,6 +36,7 @@ class EchoError(RuntimeError):
 CUDA_STREAM_LEGACY = 0x1  # cudaStreamLegacy
 CC_MODEL_WHITEBOX, CC_MODEL_ALPHA_BETA = 0, 1
 OVERLAP_WHOLE, OVERLAP_PROPORTIONAL = 0, 1
+COMM_EXECUTION, COMM_LAUNCH = 0, 1
 
 
 class GraphDesc(C.Structure):
@@ -56,7 +57,7 @@ class ScenDesc(C.Structure):
 
 
 class ComposeOpts(C.Structure):
-    _fields_ = [("refine_passes", C.c_int32), ("overlap_model", C.c_int32)]
+    _fields_ = [("refine_passes", C.c_int32), ("overlap_model", C.c_int32), ("comm_interval", C.c_int32)]
 
 
 class CCQueryDesc(C.Structure):
@@ -248,10 +249,11 @@ class Echo:
     def estimate_collectives(self):
         self._check(self.lib.echo_estimate_collectives(self.h))
 
-    def compose(self, refine_passes: int = 1, overlap_model: int = 0):
+    def compose(self, refine_passes: int = 1, overlap_model: int = 0, comm_interval: int = 0):
         """overlap_model: OVERLAP_WHOLE (d * factor) or OVERLAP_PROPORTIONAL
-        (d + (factor - 1) * overlapped length)."""
-        o = ComposeOpts(int(refine_passes), int(overlap_model))
+        (d + (factor - 1) * overlapped length).  comm_interval: COMM_EXECUTION (a
+        comm op's [start, finish)) or COMM_LAUNCH (from each member rank's launch)."""
+        o = ComposeOpts(int(refine_passes), int(overlap_model), int(comm_interval))
         self._check(self.lib.echo_compose(self.h, C.byref(o)))
 
     def read_times(self, op0: int = 0, op1: Optional[int] = None, start=True, finish=True):

@@ -19,13 +19,13 @@ CC_RTOL = 1e-9
 THREADS = max(1, min(16, os.cpu_count() or 1))
 
 
-def run_gpu(g, sc, refine=1, ctx=None, overlap_model=0):
+def run_gpu(g, sc, refine=1, ctx=None, overlap_model=0, comm_interval=0):
     e = ctx or Echo(0)
     try:
         e.load_graph(g)
         e.load_scenarios(sc)
         e.estimate_collectives()
-        e.compose(refine_passes=refine, overlap_model=overlap_model)
+        e.compose(refine_passes=refine, overlap_model=overlap_model, comm_interval=comm_interval)
         st, fn = e.read_times()
         return dict(start=st, finish=fn, makespan=e.read_makespan(), cc=e.read_cc(),
                     ov=e.read_overlap(), info=e.info())
@@ -192,6 +192,42 @@ def test_proportional_overlap_model_bit_exact():
         assert_same(got, oracle.compose(g, sc, refine_passes=1, overlap_model=1, threads=THREADS), g, 1)
         with pytest.raises(EchoError):
             e.compose(refine_passes=1, overlap_model=5)
+    finally:
+        e.close()
+
+
+def test_launch_interval_bit_exact():
+    """Comm intervals counted from each member rank's launch, with either overlap
+    model, against the oracle: random multi-rank graphs (up to 16 timelines), the
+    hand-built case, and GPT-1.3B."""
+    from tests.test_oracle_pins import _launch_case
+    rng = np.random.default_rng(6160)
+    e = Echo(0)
+    try:
+        for d_b in (100, 300):
+            g, sc = _launch_case(d_b)
+            for model in (0, 1):
+                got = run_gpu(g, sc, 1, ctx=e, overlap_model=model, comm_interval=1)
+                assert_same(got, oracle.compose(g, sc, overlap_model=model, comm_interval=1), g, 1)
+        for case in range(16):
+            g = SG.random_graph(rng, int(rng.integers(20, 400)), max_ranks=4, max_streams=16,
+                                min_streams=2 if case % 2 else 5, p_edge=0.01 if case % 4 < 2 else 0.05)
+            sc = SG.random_scenarios(rng, g, 37, max_dur=60)
+            for refine, model in ((1, 0), (2, 1), (2, 0)):
+                got = run_gpu(g, sc, refine, ctx=e, overlap_model=model, comm_interval=1)
+                want = oracle.compose(g, sc, refine_passes=refine, overlap_model=model, comm_interval=1)
+                assert_same(got, want, g, refine)
+        c = W.config("gpt1.3b")
+        g = W.build_gpt_graph(c)
+        sc = W.make_scenarios(g, c, n_scen=24)
+        for model in (0, 1):
+            got = run_gpu(g, sc, 1, ctx=e, overlap_model=model, comm_interval=1)
+            want = oracle.compose(g, sc, refine_passes=1, overlap_model=model, comm_interval=1, threads=THREADS)
+            assert_same(got, want, g, 1)
+        base = oracle.compose(g, sc, refine_passes=1, threads=THREADS)
+        assert (want.overlapped >= base.overlapped).all() and (want.overlapped > base.overlapped).any()
+        with pytest.raises(EchoError):
+            e.compose(refine_passes=1, comm_interval=2)
     finally:
         e.close()
 
