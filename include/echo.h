@@ -101,7 +101,24 @@ typedef struct {
   const int32_t *q_ops;    /* [q_off[n_ranks*n_streams]] op ids in issue order          */
   const int64_t *grp_off;  /* [n_groups+1] CSR of group members, grp_off[0] = 0         */
   const int32_t *grp_rank; /* [grp_off[n_groups]] member ranks, no repeats; P2P: 1 or 2 */
+  const int32_t *replica_of; /* [n_ranks] or NULL: replica folding, see below         */
 } echo_graph_desc;
+
+/*
+ * Replica folding (Sec. 8.5: in DDP mode Echo simulates one copy of the workload
+ * per DP group).  replica_of[b] = a marks rank b as a replica of rank a, and
+ * replica_of[a] = a marks a representative.  A replica runs the same ops as its
+ * representative, timeline by timeline and position by position: the op at
+ * position i of b's timeline k is either an op that a representative also runs
+ * (then it is the same op, e.g. a DP all-reduce shared by the replicas) or a copy
+ * of the op at position i of a's timeline k with the same kind, kernel class,
+ * message, group shape, data producers (up to the same mapping) and launch
+ * conditions.  echo_load_graph checks this (ECHO_E_BAD_GRAPH otherwise) and
+ * composes only the representatives' ops while every scenario batch gives each
+ * copied compute or memcpy op the durations of its original (checked on the
+ * device by echo_load_scenarios; a batch that does not runs the full graph).  The
+ * times are exactly those of the full graph: a copy reports its original's.
+ */
 
 /*
  * S what-if scenarios.  All arrays are host memory; dur is row-major [V][S]
@@ -165,6 +182,11 @@ int echo_destroy(echo_ctx *ctx);
  * echo_load_graph performs, without a device.  Writes the number of levels and
  * the widest level (either pointer may be NULL). */
 int echo_check_graph(const echo_graph_desc *g, int64_t *n_levels, int64_t *max_width);
+
+/* Host-only check of a graph with replica_of: the validation echo_load_graph
+ * performs, and the number of ops the folded graph composes (n_ops when
+ * replica_of is NULL or marks no replica).  Errors as echo_load_graph. */
+int echo_check_replicas(const echo_graph_desc *g, int64_t *n_ops_folded);
 
 /* Validate, level (ASAP depth over data + issue-order dependencies), renumber in
  * level order and upload the graph.  Errors: ECHO_E_INVALID_ARG, ECHO_E_BAD_GRAPH,
@@ -244,14 +266,18 @@ int echo_cc_query(echo_ctx *ctx, const echo_cc_query_desc *q, double *out_ns);
  *     and the call returns ECHO_E_INVALID_ARG; other queries are still estimated. */
 int echo_cc_query_noalloc(const echo_cc_query_desc *q, double *out_ns, void *cuda_stream);
 
-/* Shape of the loaded graph (after echo_load_graph). */
+/* Shape of the loaded graph (after echo_load_graph).  n_ops counts the caller's
+ * ops; every other count describes the graph being composed, the folded one while
+ * replicas are folded (replicas_folded = 1, see replica_of). */
 typedef struct {
   int64_t n_ops, n_edges, n_levels, max_width, n_queue_entries, n_comm_ops, n_signatures;
   int64_t n_segments;        /* serial chains the composer contracts into one step each */
   int64_t n_segment_levels;  /* synchronized steps of one composition                   */
   int64_t n_overlap_candidates; /* compute ops the validator tests (the others can never
                                    overlap a comm op of their rank, whatever the durations) */
+  int64_t n_ops_composed;    /* ops of the graph being composed                       */
   int32_t n_ranks, n_streams, sigma; /* sigma: scenarios per thread block of the composer */
+  int32_t replicas_folded;
 } echo_graph_info;
 int echo_graph_info_get(echo_ctx *ctx, echo_graph_info *info);
 

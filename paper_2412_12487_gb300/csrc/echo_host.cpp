@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <array>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -46,6 +47,7 @@ int fail(Err &e, int code, const char *fmt, ...) {
 // Everything derived from a graph on the host.
 struct GraphBuild {
   int64_t V = 0, E = 0, QE = 0, L = 0, max_width = 0;
+  int64_t V_ext = 0;  // the caller's ops (more than V when replicas are folded)
   int32_t R = 0, NS = 0, gpn = 1;
   std::vector<int32_t> int2ext, ext2int;
   int64_t Ls = 0, n_seg = 0;           // segment levels, segments
@@ -188,7 +190,10 @@ void overlap_candidates(GraphBuild &b) {
   if (b.cand_cidx.empty()) b.cand_cidx.push_back(0);
 }
 
-int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
+// `shape`, when given, replaces the (N, M, K) of every group computed from its
+// members (a folded graph keeps the shapes of the caller's groups).
+using Shape = std::array<int32_t, 3>;
+int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e, const std::vector<Shape> *shape = nullptr) {
   if (!g) return fail(e, ECHO_E_INVALID_ARG, "graph descriptor is NULL");
   const int64_t V = g->n_ops;
   if (V < 0 || V >= INT32_MAX) return fail(e, ECHO_E_INVALID_ARG, "n_ops %lld out of range", (long long)V);
@@ -341,6 +346,7 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
   int64_t L = 0;
   for (int64_t v = 0; v < V; ++v) L = std::max<int64_t>(L, level[v] + 1);
   b.V = V;
+  b.V_ext = V;
   b.E = E;
   b.QE = QE;
   b.L = L;
@@ -514,6 +520,11 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
     gN[gi] = (int32_t)members[gi].size();
     gM[gi] = (int32_t)per_node.size();
     gK[gi] = K;
+    if (shape) {
+      gN[gi] = (*shape)[gi][0];
+      gM[gi] = (*shape)[gi][1];
+      gK[gi] = (*shape)[gi][2];
+    }
   }
   std::map<std::tuple<int32_t, int32_t, int64_t, int32_t, int32_t, int32_t>, int32_t> sig_of;
   for (int64_t i = 0; i < V; ++i) {
@@ -641,6 +652,255 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e) {
 // being composed and the one before it, which slower threads may still read);
 // whatever more they hold is prefetch look-ahead.  Preference: a larger duration
 // ring, then a larger value ring (more predecessors served from shared memory).
+// Replica folding.  In DDP mode Echo composes a single copy of the workload of
+// each DP group (Sec. 8.5).  Generalised here: the caller marks rank b as a
+// replica of a representative rank a (replica_of[b] = a), meaning that b runs the
+// same ops as a, timeline by timeline and position by position.  rho maps every
+// op to its representative: an op that runs on some representative rank is its
+// own (a DP all-reduce shared by the replicas, say); an op that runs only on
+// replica ranks maps to the op at the same place on the representatives.  When
+//   (i)   d(x) = d(rho x) for every op (checked per scenario batch, on the device),
+//   (ii)  rho(preds(x)) = rho(preds(rho x)) as sets, and
+//   (iii) the folded graph -- the representatives, with predecessors rho(preds) --
+//         is acyclic,
+// the folded longest-path times t satisfy the full graph's recurrence through
+// f(x) = t(rho x), and as that recurrence has one solution, f(x) = t(rho x)
+// exactly.  (ii) holds for issue order by the positional mapping and is checked
+// here for data dependencies; the validator additionally needs a replica rank's
+// launch conditions to mirror those of its representative, also checked.
+struct Fold {
+  std::vector<int32_t> rho;     // [V] representative of each op (caller ids)
+  std::vector<int32_t> keep;    // folded id -> caller id
+  std::vector<int32_t> red;     // [V] caller id -> folded id of its representative
+  std::vector<int32_t> pairs;   // (replica op, representative) of every local replica-only op
+  std::vector<uint8_t> kind, kclass, cc_type, cc_algo;
+  std::vector<int32_t> group, pred_idx, q_ops, grp_rank;
+  std::vector<int64_t> cc_bytes, pred_off, q_off, grp_off;
+  std::vector<Shape> shape;     // [folded groups] (N, M, K) of the caller's group
+  echo_graph_desc desc{};
+};
+
+// Checks `replica_of` against the graph `g` (already validated) and builds the
+// folded graph in F.  F.keep stays empty when no rank is marked as a replica.
+int build_fold(const echo_graph_desc *g, const int32_t *replica_of, Fold &F, Err &e) {
+  const int64_t V = g->n_ops;
+  const int32_t R = g->n_ranks, NS = g->n_streams;
+  const int64_t NQ = (int64_t)R * NS, QE = g->q_off[NQ];
+  bool any = false;
+  for (int32_t r = 0; r < R; ++r) {
+    const int32_t a = replica_of[r];
+    if (a < 0 || a >= R) return fail(e, ECHO_E_INVALID_ARG, "replica_of[%d] = %d out of range", r, a);
+    if (replica_of[a] != a)
+      return fail(e, ECHO_E_BAD_GRAPH, "replica_of: rank %d mirrors rank %d, which is itself a replica", r, a);
+    any = any || a != r;
+  }
+  if (!any) return ECHO_OK;
+  auto is_rep = [&](int32_t r) { return replica_of[r] == r; };
+  // ranks of each op, ascending (CSR), and whether it runs on a representative
+  std::vector<int64_t> ro_off(V + 1, 0);
+  for (int64_t i = 0; i < QE; ++i) ro_off[g->q_ops[i] + 1]++;
+  for (int64_t v = 0; v < V; ++v) ro_off[v + 1] += ro_off[v];
+  std::vector<int32_t> ro(std::max<int64_t>(QE, 1));
+  std::vector<uint8_t> on_rep(V, 0);
+  {
+    std::vector<int64_t> fill(ro_off.begin(), ro_off.end() - 1);
+    for (int64_t q = 0; q < NQ; ++q)
+      for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i) {
+        const int32_t v = g->q_ops[i], r = (int32_t)(q / NS);
+        ro[fill[v]++] = r;
+        if (is_rep(r)) on_rep[v] = 1;
+      }
+  }
+  auto runs_on = [&](int32_t u, int32_t r) {
+    return std::binary_search(ro.data() + ro_off[u], ro.data() + ro_off[u + 1], r);
+  };
+  // the positional mapping
+  F.rho.assign(V, -1);
+  for (int32_t b = 0; b < R; ++b) {
+    const int32_t a = replica_of[b];
+    if (a == b) continue;
+    for (int32_t k = 0; k < NS; ++k) {
+      const int64_t qa = (int64_t)a * NS + k, qb = (int64_t)b * NS + k;
+      const int64_t n = g->q_off[qb + 1] - g->q_off[qb];
+      if (n != g->q_off[qa + 1] - g->q_off[qa])
+        return fail(e, ECHO_E_BAD_GRAPH, "replica_of: timeline %d of rank %d holds %lld ops, of rank %d %lld", k, b,
+                    (long long)n, a, (long long)(g->q_off[qa + 1] - g->q_off[qa]));
+      for (int64_t i = 0; i < n; ++i) {
+        const int32_t x = g->q_ops[g->q_off[qb] + i], y = g->q_ops[g->q_off[qa] + i];
+        if (on_rep[x] ? x != y : (F.rho[x] >= 0 && F.rho[x] != y))
+          return fail(e, ECHO_E_BAD_GRAPH, "replica_of: op %d (rank %d, timeline %d, position %lld) does not mirror op %d of rank %d",
+                      x, b, k, (long long)i, y, a);
+        if (!on_rep[x]) F.rho[x] = y;
+      }
+    }
+  }
+  for (int64_t v = 0; v < V; ++v)
+    if (on_rep[v]) F.rho[v] = (int32_t)v;
+  // group shapes of the caller's groups
+  std::vector<Shape> gshape(g->n_groups);
+  for (int32_t gi = 0; gi < g->n_groups; ++gi) {
+    std::map<int32_t, int32_t> per_node;
+    for (int64_t k = g->grp_off[gi]; k < g->grp_off[gi + 1]; ++k) per_node[g->grp_rank[k] / g->gpus_per_node]++;
+    int32_t K = 0;
+    for (auto &kv : per_node) K = std::max(K, kv.second);
+    gshape[gi] = {(int32_t)(g->grp_off[gi + 1] - g->grp_off[gi]), (int32_t)per_node.size(), K};
+  }
+  auto is_comm = [&](int64_t v) { return g->kind[v] == ECHO_OP_COLL || g->kind[v] == ECHO_OP_P2P; };
+  std::vector<int32_t> s1, s2;
+  auto rho_set = [&](int32_t v, std::vector<int32_t> &out, int32_t on_rank) {
+    out.clear();
+    for (int64_t k = g->pred_off[v]; k < g->pred_off[v + 1]; ++k) {
+      const int32_t u = g->pred_idx[k];
+      if (on_rank < 0 || runs_on(u, on_rank)) out.push_back(F.rho[u]);
+    }
+    std::sort(out.begin(), out.end());
+    out.erase(std::unique(out.begin(), out.end()), out.end());
+  };
+  for (int64_t x = 0; x < V; ++x) {
+    if (on_rep[x]) continue;
+    const int32_t y = F.rho[x];
+    // same op
+    bool same = g->kind[x] == g->kind[y] && (g->kind[x] != ECHO_OP_COMPUTE || g->kclass[x] == g->kclass[y]);
+    if (same && is_comm(x))
+      same = g->cc_type[x] == g->cc_type[y] && g->cc_bytes[x] == g->cc_bytes[y] &&
+             (g->cc_type[x] != ECHO_CC_ALLREDUCE || g->cc_algo[x] == g->cc_algo[y]) &&
+             gshape[g->group[x]] == gshape[g->group[y]];
+    if (!same) return fail(e, ECHO_E_BAD_GRAPH, "replica_of: op %lld differs from its representative %d", (long long)x, y);
+    // it runs on the replicas of exactly the representative ranks that run y
+    s1.clear();
+    for (int64_t k = ro_off[x]; k < ro_off[x + 1]; ++k) s1.push_back(replica_of[ro[k]]);
+    std::sort(s1.begin(), s1.end());
+    s2.clear();
+    for (int64_t k = ro_off[y]; k < ro_off[y + 1]; ++k)
+      if (is_rep(ro[k])) s2.push_back(ro[k]);
+    if (std::adjacent_find(s1.begin(), s1.end()) != s1.end() || s1 != s2)
+      return fail(e, ECHO_E_BAD_GRAPH, "replica_of: op %lld and its representative %d run on different ranks", (long long)x, y);
+    // (ii) for data dependencies
+    rho_set((int32_t)x, s1, -1);
+    rho_set(y, s2, -1);
+    if (s1 != s2)
+      return fail(e, ECHO_E_BAD_GRAPH, "replica_of: the producers of op %lld do not mirror those of op %d", (long long)x, y);
+  }
+  // launch conditions on each replica rank mirror those on its representative
+  for (int32_t b = 0; b < R; ++b) {
+    const int32_t a = replica_of[b];
+    if (a == b) continue;
+    for (int32_t k = 1; k < NS; ++k) {
+      const int64_t qa = (int64_t)a * NS + k, qb = (int64_t)b * NS + k;
+      for (int64_t i = 0; i < g->q_off[qb + 1] - g->q_off[qb]; ++i) {
+        const int32_t x = g->q_ops[g->q_off[qb] + i], y = g->q_ops[g->q_off[qa] + i];
+        if (!is_comm(x)) continue;
+        rho_set(x, s1, b);
+        rho_set(y, s2, a);
+        if (s1 != s2)
+          return fail(e, ECHO_E_BAD_GRAPH, "replica_of: the producers of op %d on rank %d do not mirror those on rank %d", x, b, a);
+      }
+    }
+  }
+  // the folded graph
+  F.red.assign(V, -1);
+  F.keep.clear();
+  for (int64_t v = 0; v < V; ++v)
+    if (F.rho[v] == v) {
+      F.red[v] = (int32_t)F.keep.size();
+      F.keep.push_back((int32_t)v);
+    }
+  for (int64_t v = 0; v < V; ++v) F.red[v] = F.red[F.rho[v]];
+  const int64_t Vf = (int64_t)F.keep.size();
+  std::vector<int32_t> gmap(g->n_groups, -1);
+  F.grp_off.assign(1, 0);
+  F.grp_rank.clear();
+  F.shape.clear();
+  F.kind.resize(Vf);
+  F.kclass.resize(Vf);
+  F.cc_type.resize(Vf);
+  F.cc_algo.resize(Vf);
+  F.group.resize(Vf);
+  F.cc_bytes.resize(Vf);
+  F.pred_off.assign(Vf + 1, 0);
+  F.pred_idx.clear();
+  for (int64_t j = 0; j < Vf; ++j) {
+    const int32_t v = F.keep[j];
+    F.kind[j] = g->kind[v];
+    F.kclass[j] = g->kclass[v];
+    F.cc_type[j] = g->cc_type[v];
+    F.cc_algo[j] = g->cc_algo[v];
+    F.cc_bytes[j] = g->cc_bytes[v];
+    F.group[j] = 0;
+    if (is_comm(v)) {
+      const int32_t gi = g->group[v];
+      if (gmap[gi] < 0) {  // the group's representative members
+        gmap[gi] = (int32_t)F.shape.size();
+        for (int64_t k = g->grp_off[gi]; k < g->grp_off[gi + 1]; ++k)
+          if (is_rep(g->grp_rank[k])) F.grp_rank.push_back(g->grp_rank[k]);
+        F.grp_off.push_back((int64_t)F.grp_rank.size());
+        F.shape.push_back(gshape[gi]);
+      }
+      F.group[j] = gmap[gi];
+    }
+    s1.clear();
+    for (int64_t k = g->pred_off[v]; k < g->pred_off[v + 1]; ++k) s1.push_back(F.red[g->pred_idx[k]]);
+    std::sort(s1.begin(), s1.end());
+    s1.erase(std::unique(s1.begin(), s1.end()), s1.end());
+    F.pred_idx.insert(F.pred_idx.end(), s1.begin(), s1.end());
+    F.pred_off[j + 1] = (int64_t)F.pred_idx.size();
+  }
+  F.q_off.assign(NQ + 1, 0);
+  F.q_ops.clear();
+  for (int64_t q = 0; q < NQ; ++q) {
+    if (is_rep((int32_t)(q / NS)))
+      for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i) F.q_ops.push_back(F.red[g->q_ops[i]]);
+    F.q_off[q + 1] = (int64_t)F.q_ops.size();
+  }
+  F.pairs.clear();
+  for (int64_t x = 0; x < V; ++x)
+    if (F.rho[x] != x && !is_comm(x)) {
+      F.pairs.push_back((int32_t)x);
+      F.pairs.push_back(F.rho[x]);
+    }
+  echo_graph_desc &d = F.desc;
+  d = echo_graph_desc{};
+  d.n_ops = Vf;
+  d.n_ranks = R;
+  d.n_streams = NS;
+  d.gpus_per_node = g->gpus_per_node;
+  d.n_groups = (int32_t)F.shape.size();
+  d.kind = F.kind.data();
+  d.kclass = F.kclass.data();
+  d.group = F.group.data();
+  d.cc_type = F.cc_type.data();
+  d.cc_algo = F.cc_algo.data();
+  d.cc_bytes = F.cc_bytes.data();
+  d.pred_off = F.pred_off.data();
+  d.pred_idx = F.pred_idx.data();
+  d.q_off = F.q_off.data();
+  d.q_ops = F.q_ops.data();
+  d.grp_off = F.grp_off.data();
+  d.grp_rank = F.grp_rank.data();
+  d.replica_of = nullptr;
+  return ECHO_OK;
+}
+
+// The folded graph of `g` when its replica_of marks replicas: `fb` composes it,
+// with int2ext / ext2int / V_ext in the caller's ids.  Returns ECHO_OK with
+// *folded = false when there is nothing to fold.
+int build_folded(const echo_graph_desc *g, GraphBuild &fb, Fold &F, bool *folded, Err &e) {
+  *folded = false;
+  if (!g->replica_of) return ECHO_OK;
+  int rc = build_fold(g, g->replica_of, F, e);
+  if (rc || F.keep.empty()) return rc;
+  Err e2;
+  rc = build_graph(&F.desc, fb, e2, &F.shape);
+  if (rc) return fail(e, ECHO_E_BAD_GRAPH, "replica_of: the folded graph is not valid (%s)", e2.msg.c_str());
+  for (auto &x : fb.int2ext) x = F.keep[x];
+  std::vector<int32_t> e2i(g->n_ops);
+  for (int64_t v = 0; v < g->n_ops; ++v) e2i[v] = fb.ext2int[F.red[v]];
+  fb.ext2int.swap(e2i);
+  fb.V_ext = g->n_ops;
+  *folded = true;
+  return ECHO_OK;
+}
+
 // The steps of the staged kernels for scenario blocks of `sigma`.  The segments of
 // one level are independent, so a wide level may run as several consecutive
 // steps: each step holds at most `cap` nodes and kStepSegments segments, so that
@@ -802,6 +1062,15 @@ struct echo_ctx {
   int state = 0;  // 0 empty, 1 graph, 2 scenarios, 3 estimated, 4 composed
   GraphBuild gb;
   std::vector<void *> graph_allocs, scen_allocs;
+  // replica folding: the other build of the graph (the full one while the folded
+  // one is active, and the reverse), pairs of rows whose durations must match
+  bool fold_ok = false, fold_active = false;
+  GraphBuild gb_alt;
+  std::vector<void *> fold_allocs;
+  int32_t *fold_pairs = nullptr, *fold_flag = nullptr;
+  int64_t n_fold_pairs = 0;
+  std::vector<void *> raw_allocs;  // the caller's durations as uploaded
+  size_t raw_cap = 0;
   // device graph
   int64_t *seg_lvl_off = nullptr, *seg_node_off = nullptr, *nq_off = nullptr, *dp_off = nullptr, *q_off = nullptr;
   int64_t *ov_chunks = nullptr, *cq_off = nullptr;
@@ -823,7 +1092,8 @@ struct echo_ctx {
   uint64_t *sfx = nullptr;  // packed slowdown factors [C][S]
   double *sf = nullptr;     // slowdown factors [C][S]
   std::vector<uint64_t> h_sfx;
-  int64_t *raw = nullptr, *dur = nullptr, *f[2] = {nullptr, nullptr}, *mk = nullptr, *cc_dur = nullptr;
+  void *raw = nullptr;
+  int64_t *dur = nullptr, *f[2] = {nullptr, nullptr}, *mk = nullptr, *cc_dur = nullptr;
   int64_t *gfrontier = nullptr;
   int64_t *deff = nullptr;                // full validator durations, for kernels without a candidate ring
   int64_t *cd[2] = {nullptr, nullptr};    // candidates' durations of the validator's passes (compact)
@@ -993,6 +1263,45 @@ int make_table(echo_ctx *c, int32_t n, const int64_t *mx, const int64_t *cb, Chu
   return ECHO_OK;
 }
 
+// Device copies of the active graph build c->gb.
+int upload_graph(echo_ctx *c) {
+  free_all(c->graph_allocs);
+  const GraphBuild &B = c->gb;
+  auto &o = c->graph_allocs;
+  int rc;
+  if ((rc = upload(c, o, &c->seg_lvl_off, B.seg_lvl_off)) || (rc = upload(c, o, &c->seg_node_off, B.seg_node_off)) ||
+      (rc = upload(c, o, &c->ov_chunks, B.ov_chunks)) ||
+      (rc = upload(c, o, &c->cq_off, B.cq_off)) || (rc = upload(c, o, &c->cq_ops, B.cq_ops)) ||
+      (rc = upload(c, o, &c->lq_off, B.lq_off)) || (rc = upload(c, o, &c->lq_ops, B.lq_ops)) ||
+      (rc = upload(c, o, &c->cand_off, B.cand_off)) || (rc = upload(c, o, &c->cand_ops, B.cand_ops)) ||
+      (rc = upload(c, o, &c->cand_flag, B.cand_flag)) || (rc = upload(c, o, &c->cand_cidx, B.cand_cidx)) ||
+      (rc = upload(c, o, &c->cidx, B.cidx)) || (rc = upload(c, o, &c->cand_node, B.cand_node)) ||
+      (rc = upload(c, o, &c->nq_off, B.nq_off)) ||
+      (rc = upload(c, o, &c->nq, B.nq)) || (rc = upload(c, o, &c->dp_off, B.dp_off)) ||
+      (rc = upload(c, o, &c->dp, B.dp)) || (rc = upload(c, o, &c->q_off, B.q_off)) ||
+      (rc = upload(c, o, &c->q_ops, B.q_ops_int)) || (rc = upload(c, o, &c->int2ext, B.int2ext)) ||
+      (rc = upload(c, o, &c->ext2int, B.ext2int)) || (rc = upload(c, o, &c->node_sig, B.node_sig)) ||
+      (rc = upload(c, o, &c->comm_node, B.comm_node)) || (rc = upload(c, o, &c->comm_sig, B.comm_sig)) ||
+      (rc = upload(c, o, &c->sig_count, B.sig_count)) || (rc = upload(c, o, &c->kcl, B.kcl)) ||
+      (rc = upload(c, o, &c->local, B.local)) ||
+      (rc = upload(c, o, &c->sigs, B.sigs))) {
+    free_all(c->graph_allocs);
+    return rc;
+  }
+  CK(cudaStreamSynchronize(c->stream), "graph upload");
+  return ECHO_OK;
+}
+
+// Makes the folded (want = true) or the full build of the graph the active one.
+int activate_fold(echo_ctx *c, bool want) {
+  if (!c->fold_ok || want == c->fold_active) return ECHO_OK;
+  std::swap(c->gb, c->gb_alt);
+  c->fold_active = want;
+  free_all(c->scen_allocs);
+  c->scen_vs = 0;
+  return upload_graph(c);
+}
+
 }  // namespace
 
 extern "C" {
@@ -1072,6 +1381,8 @@ int echo_destroy(echo_ctx *c) {
   cudaStreamSynchronize(c->stream);
   free_all(c->graph_allocs);
   free_all(c->scen_allocs);
+  free_all(c->fold_allocs);
+  free_all(c->raw_allocs);
   if (c->stage) cudaFree(c->stage);
   if (c->status) cudaFree(c->status);
   for (auto &r : c->recs) {
@@ -1094,41 +1405,47 @@ int echo_check_graph(const echo_graph_desc *g, int64_t *n_levels, int64_t *max_w
   return ECHO_OK;
 }
 
+int echo_check_replicas(const echo_graph_desc *g, int64_t *n_ops_folded) {
+  GraphBuild b, fb;
+  Fold F;
+  Err e;
+  bool folded = false;
+  int rc = build_graph(g, b, e);
+  if (!rc) rc = build_folded(g, fb, F, &folded, e);
+  if (rc) return rc;
+  if (n_ops_folded) *n_ops_folded = folded ? fb.V : b.V;
+  return ECHO_OK;
+}
+
 int echo_load_graph(echo_ctx *c, const echo_graph_desc *g) {
   int rc = check_ctx(c);
   if (rc) return rc;
-  GraphBuild b;
+  GraphBuild b, fb;
+  Fold F;
   Err e;
-  rc = build_graph(g, b, e);
-  if (rc) return set_err(c, rc, e.msg);
+  bool folded = false;
+  if ((rc = build_graph(g, b, e)) || (rc = build_folded(g, fb, F, &folded, e))) return set_err(c, rc, e.msg);
   CK(cudaStreamSynchronize(c->stream), "cudaStreamSynchronize");
   free_all(c->graph_allocs);
   free_all(c->scen_allocs);
+  free_all(c->fold_allocs);
   c->scen_vs = 0;
   c->state = 0;
-  c->gb = std::move(b);
-  const GraphBuild &B = c->gb;
-  auto &o = c->graph_allocs;
-  if ((rc = upload(c, o, &c->seg_lvl_off, B.seg_lvl_off)) || (rc = upload(c, o, &c->seg_node_off, B.seg_node_off)) ||
-      (rc = upload(c, o, &c->ov_chunks, B.ov_chunks)) ||
-      (rc = upload(c, o, &c->cq_off, B.cq_off)) || (rc = upload(c, o, &c->cq_ops, B.cq_ops)) ||
-      (rc = upload(c, o, &c->lq_off, B.lq_off)) || (rc = upload(c, o, &c->lq_ops, B.lq_ops)) ||
-      (rc = upload(c, o, &c->cand_off, B.cand_off)) || (rc = upload(c, o, &c->cand_ops, B.cand_ops)) ||
-      (rc = upload(c, o, &c->cand_flag, B.cand_flag)) || (rc = upload(c, o, &c->cand_cidx, B.cand_cidx)) ||
-      (rc = upload(c, o, &c->cidx, B.cidx)) || (rc = upload(c, o, &c->cand_node, B.cand_node)) ||
-      (rc = upload(c, o, &c->nq_off, B.nq_off)) ||
-      (rc = upload(c, o, &c->nq, B.nq)) || (rc = upload(c, o, &c->dp_off, B.dp_off)) ||
-      (rc = upload(c, o, &c->dp, B.dp)) || (rc = upload(c, o, &c->q_off, B.q_off)) ||
-      (rc = upload(c, o, &c->q_ops, B.q_ops_int)) || (rc = upload(c, o, &c->int2ext, B.int2ext)) ||
-      (rc = upload(c, o, &c->ext2int, B.ext2int)) || (rc = upload(c, o, &c->node_sig, B.node_sig)) ||
-      (rc = upload(c, o, &c->comm_node, B.comm_node)) || (rc = upload(c, o, &c->comm_sig, B.comm_sig)) ||
-      (rc = upload(c, o, &c->sig_count, B.sig_count)) || (rc = upload(c, o, &c->kcl, B.kcl)) ||
-      (rc = upload(c, o, &c->local, B.local)) ||
-      (rc = upload(c, o, &c->sigs, B.sigs))) {
-    free_all(c->graph_allocs);
-    return rc;
+  c->fold_ok = c->fold_active = folded;
+  c->n_fold_pairs = 0;
+  if (folded) {  // compose the folded graph until a scenario batch breaks the symmetry
+    c->gb = std::move(fb);
+    c->gb_alt = std::move(b);
+    c->n_fold_pairs = (int64_t)F.pairs.size() / 2;
+    if (F.pairs.empty()) F.pairs.assign(2, 0);
+    if ((rc = upload(c, c->fold_allocs, &c->fold_pairs, F.pairs)) ||
+        (rc = dalloc(c, c->fold_allocs, &c->fold_flag, 1)))
+      return rc;
+  } else {
+    c->gb = std::move(b);
+    c->gb_alt = GraphBuild{};
   }
-  CK(cudaStreamSynchronize(c->stream), "graph upload");
+  if ((rc = upload_graph(c))) return rc;
   c->state = 1;
   return ECHO_OK;
 }
@@ -1138,13 +1455,13 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   if (rc) return rc;
   if (c->state < 1) return set_err(c, ECHO_E_STATE, "load a graph first");
   if (!sc) return set_err(c, ECHO_E_INVALID_ARG, "scenario descriptor is NULL");
-  const GraphBuild &B = c->gb;
-  const int64_t V = B.V;
+  const GraphBuild &B = c->gb;  // (the active build: folded or full)
+  const int64_t Vx = B.V_ext;
   const int32_t S = sc->n_scen;
   if (S < 1) return set_err(c, ECHO_E_INVALID_ARG, "n_scen must be >= 1");
   if (sc->n_kclass < 1 || sc->n_kclass <= B.max_kclass)
     return set_err(c, ECHO_E_INVALID_ARG, "n_kclass must exceed every compute op's kclass");
-  if (V > 0 && !sc->dur) return set_err(c, ECHO_E_INVALID_ARG, "dur is NULL");
+  if (Vx > 0 && !sc->dur) return set_err(c, ECHO_E_INVALID_ARG, "dur is NULL");
   if (sc->dur_bits != 0 && sc->dur_bits != 32 && sc->dur_bits != 64)
     return set_err(c, ECHO_E_INVALID_ARG, "dur_bits must be 32 or 64");
   if (!sc->slowdown) return set_err(c, ECHO_E_INVALID_ARG, "slowdown is NULL");
@@ -1163,6 +1480,33 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
 
   CK(cudaStreamSynchronize(c->stream), "cudaStreamSynchronize");
   c->state = 1;
+  // the caller's durations, as given, on the device
+  const int bits = sc->dur_bits == 32 ? 32 : 64;
+  const size_t raw_bytes = (size_t)Vx * S * (bits / 8);
+  if (raw_bytes > c->raw_cap) {
+    free_all(c->raw_allocs);
+    c->raw = nullptr;
+    c->raw_cap = 0;
+    uint8_t *p = nullptr;
+    if ((rc = dalloc(c, c->raw_allocs, &p, raw_bytes))) return rc;
+    c->raw = p;
+    c->raw_cap = raw_bytes;
+  }
+  if (Vx > 0)
+    CK(cudaMemcpyAsync(c->raw, sc->dur, raw_bytes, cudaMemcpyHostToDevice, c->stream), "duration upload");
+  if (c->fold_ok) {
+    // the folded graph gives the full graph's times when every replica op's
+    // durations equal its representative's in every scenario
+    int32_t h_flag = 0;
+    CK(cudaMemsetAsync(c->fold_flag, 0, sizeof(int32_t), c->stream), "memset");
+    CK(timed(c, "replica_check", [&] {
+         return echo::launch_replica_check(c->raw, bits, c->fold_pairs, c->n_fold_pairs, S, c->fold_flag, c->stream);
+       }), "replica check launch");
+    CK(cudaMemcpyAsync(&h_flag, c->fold_flag, sizeof h_flag, cudaMemcpyDeviceToHost, c->stream), "flag readback");
+    CK(cudaStreamSynchronize(c->stream), "cudaStreamSynchronize");
+    if ((rc = activate_fold(c, h_flag == 0))) return rc;
+  }
+  const int64_t V = B.V;
   const int sigma = pick_sigma(S, c->sms);
   int slog2 = 0;
   while ((1 << slog2) < sigma) ++slog2;
@@ -1179,7 +1523,7 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     const size_t CS = (size_t)std::max<int64_t>(B.n_cand, 1) * (size_t)nblk * sigma;  // compact matrices
     if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sfx, (size_t)C * S)) || (rc = dalloc(c, o, &c->sf, (size_t)C * S)) ||
         (rc = dalloc(c, o, &c->sums, (size_t)S)) || (rc = dalloc(c, o, &c->comm_sum, (size_t)S)) ||
-        (rc = dalloc(c, o, &c->raw, (size_t)V * S)) || (rc = dalloc(c, o, &c->dur, VS)) ||
+        (rc = dalloc(c, o, &c->dur, VS)) ||
         (rc = dalloc(c, o, &c->f[0], VS)) || (rc = dalloc(c, o, &c->f[1], VS)) ||
         (rc = dalloc(c, o, &c->cd[0], CS)) || (rc = dalloc(c, o, &c->ov, VS)) ||
         (rc = dalloc(c, o, &c->mk, (size_t)S)) || (rc = dalloc(c, o, &c->cc_ns, (size_t)G * S)) ||
@@ -1258,9 +1602,6 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   CK(cudaMemsetAsync(c->sums, 0, S * sizeof(double), c->stream), "memset");
   CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
   if (V > 0) {
-    const int bits = sc->dur_bits == 32 ? 32 : 64;
-    CK(cudaMemcpyAsync(c->raw, sc->dur, (size_t)V * S * (bits / 8), cudaMemcpyHostToDevice, c->stream),
-       "duration upload");
     CK(timed(c, "permute_rows", [&] {
          return echo::launch_permute_rows(c->raw, bits, c->int2ext, c->local, V, S, c->lay, c->dur, c->sums,
                                           c->status, c->stream);
@@ -1440,7 +1781,7 @@ static int composition_status(echo_ctx *c) {
 
 static int read_range_check(echo_ctx *c, int64_t op0, int64_t op1, int need_state) {
   if (c->state < need_state) return set_err(c, ECHO_E_STATE, "nothing to read yet");
-  if (op0 < 0 || op1 < op0 || op1 > c->gb.V) return set_err(c, ECHO_E_INVALID_ARG, "op range out of bounds");
+  if (op0 < 0 || op1 < op0 || op1 > c->gb.V_ext) return set_err(c, ECHO_E_INVALID_ARG, "op range out of bounds");
   return ECHO_OK;
 }
 
@@ -1597,7 +1938,9 @@ int echo_graph_info_get(echo_ctx *c, echo_graph_info *info) {
   if (!c || !info) return ECHO_E_INVALID_ARG;
   if (c->state < 1) return set_err(c, ECHO_E_STATE, "load a graph first");
   const GraphBuild &B = c->gb;
-  info->n_ops = B.V;
+  info->n_ops = B.V_ext;
+  info->n_ops_composed = B.V;
+  info->replicas_folded = c->fold_active ? 1 : 0;
   info->n_edges = B.E;
   info->n_levels = B.L;
   info->max_width = B.max_width;

@@ -163,6 +163,10 @@ cudaError_t launch_cc_scatter(const int32_t *comm_node, const int32_t *comm_sig,
 cudaError_t launch_cc_query(int64_t n, const uint8_t *type, const uint8_t *algo, const int64_t *nbytes,
                             const int32_t *N, const int32_t *M, const double *lg, ScenParams p,
                             const ChunkTable &tbl, double *out, cudaStream_t st);
+// sets *flag when row pairs[2p] of the [V][S] matrix `raw` (int32 or int64) differs
+// from row pairs[2p+1] in some scenario
+cudaError_t launch_replica_check(const void *raw, int bits, const int32_t *pairs, int64_t n_pairs, int32_t S,
+                                 int32_t *flag, cudaStream_t st);
 cudaError_t launch_permute_rows(const void *raw, int bits, const int32_t *int2ext, const uint8_t *local,
                                 int64_t V, int32_t S, MatLayout lay, int64_t *dur, double *sums, int32_t *status,
                                 cudaStream_t st);

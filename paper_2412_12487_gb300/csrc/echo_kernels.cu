@@ -510,6 +510,34 @@ cudaError_t launch_permute_rows(const void *raw, int bits, const int32_t *int2ex
   return cudaGetLastError();
 }
 
+template <typename T>
+__global__ void replica_check_kernel(const T *__restrict__ raw, const int32_t *__restrict__ pairs, int64_t n_pairs,
+                                     int32_t S, int32_t *flag) {
+  const int64_t total = n_pairs * S;
+  bool diff = false;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t p = idx / S, s = idx - p * S;
+    diff |= raw[(int64_t)pairs[2 * p] * S + s] != raw[(int64_t)pairs[2 * p + 1] * S + s];
+  }
+  if (__any_sync(0xffffffffu, diff) && (threadIdx.x & 31) == 0) *flag = 1;
+}
+
+cudaError_t launch_replica_check(const void *raw, int bits, const int32_t *pairs, int64_t n_pairs, int32_t S,
+                                 int32_t *flag, cudaStream_t st) {
+  if (n_pairs == 0 || S == 0) return cudaSuccess;
+  const int64_t total = n_pairs * S;
+  const int threads = 256;
+  const int64_t blocks = std::min<int64_t>((total + threads - 1) / threads, 152 * 16);
+  if (bits == 32)
+    replica_check_kernel<int32_t><<<(unsigned)blocks, threads, 0, st>>>(static_cast<const int32_t *>(raw), pairs,
+                                                                         n_pairs, S, flag);
+  else
+    replica_check_kernel<int64_t><<<(unsigned)blocks, threads, 0, st>>>(static_cast<const int64_t *>(raw), pairs,
+                                                                         n_pairs, S, flag);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
   if (a.S == 0 || a.n_chunks == 0) return cudaSuccess;
   if (a.n_cq < 0 || a.n_cq > kMaxStreams) return cudaErrorInvalidValue;

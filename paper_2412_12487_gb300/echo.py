@@ -20,7 +20,7 @@ STATUS_NAMES = {0: "ECHO_OK", 1: "ECHO_E_INVALID_ARG", 2: "ECHO_E_BAD_GRAPH", 3:
                 8: "ECHO_E_OVERFLOW", 9: "ECHO_E_UNSUPPORTED"}
 
 # every function the header declares (checked by the tests)
-EXPORTS = ["echo_create", "echo_destroy", "echo_check_graph", "echo_load_graph", "echo_load_scenarios",
+EXPORTS = ["echo_create", "echo_destroy", "echo_check_graph", "echo_check_replicas", "echo_load_graph", "echo_load_scenarios",
            "echo_estimate_collectives", "echo_compose", "echo_read_times", "echo_read_makespan",
            "echo_read_cc", "echo_read_overlap", "echo_cc_query", "echo_cc_query_noalloc",
            "echo_graph_info_get", "echo_set_cc_model",
@@ -45,7 +45,8 @@ class GraphDesc(C.Structure):
                 ("kind", C.c_void_p), ("kclass", C.c_void_p), ("group", C.c_void_p),
                 ("cc_type", C.c_void_p), ("cc_algo", C.c_void_p), ("cc_bytes", C.c_void_p),
                 ("pred_off", C.c_void_p), ("pred_idx", C.c_void_p), ("q_off", C.c_void_p),
-                ("q_ops", C.c_void_p), ("grp_off", C.c_void_p), ("grp_rank", C.c_void_p)]
+                ("q_ops", C.c_void_p), ("grp_off", C.c_void_p), ("grp_rank", C.c_void_p),
+                ("replica_of", C.c_void_p)]
 
 
 class ScenDesc(C.Structure):
@@ -72,8 +73,9 @@ class GraphInfo(C.Structure):
     _fields_ = [("n_ops", C.c_int64), ("n_edges", C.c_int64), ("n_levels", C.c_int64),
                 ("max_width", C.c_int64), ("n_queue_entries", C.c_int64), ("n_comm_ops", C.c_int64),
                 ("n_signatures", C.c_int64), ("n_segments", C.c_int64), ("n_segment_levels", C.c_int64),
-                ("n_overlap_candidates", C.c_int64),
-                ("n_ranks", C.c_int32), ("n_streams", C.c_int32), ("sigma", C.c_int32)]
+                ("n_overlap_candidates", C.c_int64), ("n_ops_composed", C.c_int64),
+                ("n_ranks", C.c_int32), ("n_streams", C.c_int32), ("sigma", C.c_int32),
+                ("replicas_folded", C.c_int32)]
 
 
 class KernelStat(C.Structure):
@@ -102,6 +104,7 @@ def load_library(path: Optional[str] = None):
         "echo_create": ([C.POINTER(vp), C.c_int, vp], C.c_int),
         "echo_destroy": ([vp], C.c_int),
         "echo_check_graph": ([C.POINTER(GraphDesc), C.POINTER(i64), C.POINTER(i64)], C.c_int),
+        "echo_check_replicas": ([C.POINTER(GraphDesc), C.POINTER(i64)], C.c_int),
         "echo_load_graph": ([vp, C.POINTER(GraphDesc)], C.c_int),
         "echo_load_scenarios": ([vp, C.POINTER(ScenDesc)], C.c_int),
         "echo_estimate_collectives": ([vp], C.c_int),
@@ -153,7 +156,8 @@ def _graph_desc(g, keep: list) -> GraphDesc:
                      a(g.kind, np.uint8), a(g.kclass, np.uint8), a(g.group, np.int32),
                      a(g.cc_type, np.uint8), a(g.cc_algo, np.uint8), a(g.cc_bytes, np.int64),
                      a(g.pred_off, np.int64), a(g.pred_idx, np.int32), a(g.q_off, np.int64),
-                     a(g.q_ops, np.int32), a(g.grp_off, np.int64), a(g.grp_rank, np.int32))
+                     a(g.q_ops, np.int32), a(g.grp_off, np.int64), a(g.grp_rank, np.int32),
+                     a(g.replica_of, np.int32) if getattr(g, "replica_of", None) is not None else None)
 
 
 def check_graph(g) -> Tuple[int, int]:
@@ -166,6 +170,19 @@ def check_graph(g) -> Tuple[int, int]:
     if rc:
         raise EchoError(rc, lib.echo_strerror(rc).decode())
     return int(L.value), int(W.value)
+
+
+def check_replicas(g) -> int:
+    """Host-only check of ``g.replica_of``: the number of ops the folded graph
+    composes (``g.n_ops`` when nothing is folded)."""
+    lib = load_library()
+    keep: list = []
+    d = _graph_desc(g, keep)
+    n = C.c_int64(0)
+    rc = lib.echo_check_replicas(C.byref(d), C.byref(n))
+    if rc:
+        raise EchoError(rc, lib.echo_strerror(rc).decode())
+    return int(n.value)
 
 
 class Echo:

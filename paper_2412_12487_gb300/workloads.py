@@ -82,6 +82,7 @@ class Graph:
     work: np.ndarray      # FLOP(-equivalent) per op, input-recipe only
     noise: np.ndarray     # lognormal factor per op, input-recipe only
     name: str = ""
+    replica_of: Optional[np.ndarray] = None  # int32 [n_ranks]: rank -> its representative
 
     @property
     def n_ops(self) -> int:
@@ -140,6 +141,9 @@ class GPTConfig:
     fixed_scenario: bool = False     # one fixed H800-like scenario instead of random draws
     graph_seed: int = 0
     scen_seed: int = 1000
+    # DP replicas that run identical kernels (each replica op takes its replica-0
+    # original's noise draw); the graph then carries replica_of for folding
+    identical_replicas: bool = False
 
 
 # The five workloads (GPT shapes of Table 7; 3D-parallel layouts as in Sec. 8).
@@ -577,9 +581,21 @@ def build_gpt_graph(c: GPTConfig) -> Graph:
 
     rng = np.random.Generator(np.random.PCG64(c.graph_seed))
     noise = np.exp(rng.normal(0.0, 0.1, size=V))
+    replica_of = None
+    if c.identical_replicas and DP > 1:
+        # rank (dp, p, t) mirrors rank (0, p, t): the op at each timeline position of a
+        # replica takes the noise of the op at the same position of replica 0
+        replica_of = (np.arange(R) % (PP * TP)).astype(np.int32)
+        orig = np.arange(V)
+        for q in range(nq):
+            r, k = divmod(q, N_STREAMS)
+            qa = int(replica_of[r]) * N_STREAMS + k
+            if qa != q:
+                orig[q_ops[q_off[q]:q_off[q + 1]]] = q_ops[q_off[qa]:q_off[qa + 1]]
+        noise = noise[orig]
     g = Graph(R, N_STREAMS, c.gpus_per_node, kind, kclass, group, cc_type, cc_algo, cc_bytes,
               pred_off, pred_idx, q_off, q_ops, grp_off, grp_rank.astype(np.int32), work, noise,
-              name=c.name)
+              name=c.name, replica_of=replica_of)
     return g
 
 
