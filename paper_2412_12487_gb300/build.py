@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libecho.so")
 BUILD_DIR = os.path.join(PKG, "_build")
-SOURCES = ["echo_kernels.cu", "echo_compose.cu", "echo_host.cpp"]
+SOURCES = ["echo_kernels.cu", "echo_compose.cu", "echo_dataflow.cu", "echo_host.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

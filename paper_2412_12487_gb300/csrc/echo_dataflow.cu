@@ -1,0 +1,235 @@
+// echo_dataflow.cu -- the dataflow composer: the max-plus pass of Sec. 4.2 with one
+// warp per (rank, group of 32 scenarios) instead of one block per scenario block.
+//
+// The levelled kernels synchronize a whole scenario block at every segment level,
+// so a graph with many levels and few scenarios leaves most SMs idle and pays one
+// synchronization per level.  Here every warp walks its rank's ops in the internal
+// (topological) order on its own, with the latest finish of each of the rank's
+// timelines in shared memory, and waits only where a value comes from another
+// warp:
+//   - a collective or P2P op (Sec. 5.2: it starts when its last member has
+//     launched it): each member warp publishes its partial launch time (the
+//     latest finish among the op's inputs on its rank) and reads the others'.
+//     Groups of more than 8 members gather at one member, which publishes the
+//     finish;
+//   - a data input produced on another rank: its producer publishes its finish.
+// A published value is one 64-bit word per scenario: the time (below 2^56) with
+// the launch's 8-bit tag in the top byte, written by one relaxed store and polled
+// by relaxed loads, so no flag, fence or reset is needed between launches.  Every
+// warp is resident (cooperative launch) and waits only for ops earlier in the
+// topological order, so the earliest unfinished op can always proceed.  Every
+// wait is bounded: a warp that gives up sets the abort flag and the timeout
+// status, and every other warp leaves at its next wait.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdint>
+
+#include "echo_internal.h"
+
+namespace echo {
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr uint64_t kValueMask = (1ull << 56) - 1;
+
+__device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t *p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_relaxed_u64(uint64_t *p, uint64_t v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ int32_t ld_relaxed_s32(const int32_t *p) {
+  int32_t v;
+  asm volatile("ld.relaxed.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Waits until every lane sees the tag in the words p[i << 5] for i < n but
+// `skip` (n <= 8: one round's loads are in flight together), and folds their
+// values into t.  False when this wait or another warp's gave up.
+__device__ bool df_gather(const uint64_t *p, uint32_t n, uint32_t skip, uint64_t tag, int64_t &t,
+                          const DataflowArgs &a) {
+  const long long t0 = clock64();
+  unsigned ns = 32;
+  uint64_t x[8];
+  for (uint32_t round = 0;; ++round) {
+    bool ok = true;
+#pragma unroll
+    for (uint32_t i = 0; i < 8; ++i) {
+      x[i] = i < n && i != skip ? ld_relaxed_u64(p + ((int64_t)i << 5)) : tag;
+      ok &= (x[i] & ~kValueMask) == tag;
+    }
+    if (__all_sync(kFull, ok)) break;
+    const bool give_up = ((round & 15) == 15 && ld_relaxed_s32(a.abort_flag) != 0) ||
+                         clock64() - t0 > a.wait_limit_cycles;
+    if (__any_sync(kFull, give_up)) {
+      if ((threadIdx.x & 31) == 0) {
+        atomicExch(a.abort_flag, 1);
+        atomicCAS(a.status, (int32_t)kDevOk, (int32_t)kDevTimeout);
+      }
+      return false;
+    }
+    if (round >= 32) {  // spin first: most waits end within a few L2 round trips
+      __nanosleep(ns);
+      if (ns < 256) ns <<= 1;
+    }
+  }
+#pragma unroll
+  for (uint32_t i = 0; i < 8; ++i) t = max(t, (int64_t)(x[i] & kValueMask));
+  return true;
+}
+
+template <bool CAND>
+__global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_kernel(DataflowArgs a) {
+  extern __shared__ int64_t df_last[];  // [warps][n_streams][32]: latest finish of each timeline
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  const int64_t wid = (int64_t)blockIdx.x * (kDfThreads / 32) + wib;
+  if (wid >= (int64_t)a.R * a.G) return;  // uniform over the warp
+  const int32_t r = (int32_t)(wid % a.R), g = (int32_t)(wid / a.R);
+  const int32_t s = g * 32 + lane;
+  int64_t *last = df_last + (int64_t)wib * a.n_streams * 32 + lane;
+  for (int k = 0; k < a.n_streams; ++k) last[k * 32] = 0;
+  // rows of 32 scenarios: element (i, s) of an [n][S] matrix at ((g * n + i) << 5) + lane
+  const int64_t *dur = a.dur + (((int64_t)g * a.V) << 5) + lane;
+  const int64_t *cdu = CAND ? a.cdur + (((int64_t)g * a.n_cand) << 5) + lane : nullptr;
+  int64_t *f = a.f + (((int64_t)g * a.V) << 5) + lane;
+  uint64_t *part = a.part + (((int64_t)g * a.n_slots) << 5) + lane;
+  uint64_t *xval = a.xval + (((int64_t)g * a.n_exports) << 5) + lane;
+  const uint64_t tag = (uint64_t)(a.epoch & 0xFF) << 56;
+  const int64_t e0 = a.off[r], e1 = a.off[r + 1];
+  int64_t mx = 0;
+  // batches of 8 entries of 8 words: lane l holds words 2(l % 4) and 2(l % 4) + 1
+  // of entry l / 4.  Records are loaded three batches ahead of their use, the
+  // durations one batch ahead.
+  auto rec = [&](int64_t b) -> uint2 {
+    return b + lane / 4 < e1 ? __ldg(reinterpret_cast<const uint2 *>(a.rec) + 4 * b + lane) : make_uint2(0, 0);
+  };
+  auto durs = [&](int64_t b, uint2 w, int64_t(&d)[kDfBatch]) {
+#pragma unroll
+    for (int j = 0; j < kDfBatch; ++j) {
+      const uint32_t v = __shfl_sync(kFull, w.x, 4 * j), ci = __shfl_sync(kFull, w.y, 4 * j);
+      d[j] = 0;
+      if (b + j < e1) d[j] = (CAND && ci != ~0u) ? cdu[(int64_t)ci << 5] : dur[(int64_t)v << 5];
+    }
+  };
+  uint2 w0 = rec(e0), w1 = rec(e0 + kDfBatch), w2 = rec(e0 + 2 * kDfBatch);
+  int64_t d0[kDfBatch];
+  durs(e0, w0, d0);
+  int64_t cur = 0;  // finish of the previous op of the program
+  for (int64_t b = e0; b < e1; b += kDfBatch) {
+    const uint2 w3 = rec(b + 3 * kDfBatch);
+    int64_t d1[kDfBatch];
+    durs(b + kDfBatch, w1, d1);
+    const int n_here = e1 - b < kDfBatch ? (int)(e1 - b) : kDfBatch;
+    // a full batch of common ops (inputs: the previous op at most) runs branch-free
+    bool plain = n_here == kDfBatch;
+#pragma unroll
+    for (int j = 0; j < kDfBatch; ++j) plain &= (__shfl_sync(kFull, w0.x, 4 * j + 1) & kDfSlowMask) == 0;
+    if (plain) {
+#pragma unroll
+      for (int j = 0; j < kDfBatch; ++j) {
+        const uint32_t v = __shfl_sync(kFull, w0.x, 4 * j), hdr = __shfl_sync(kFull, w0.x, 4 * j + 1);
+        cur = ((hdr & kDfPrev) ? cur : 0) + d0[j];
+        f[(int64_t)v << 5] = cur;
+        last[(hdr & 15) * 32] = cur;
+        mx = max(mx, cur);
+      }
+    } else {
+#pragma unroll
+    for (int j = 0; j < kDfBatch; ++j) {
+      if (j >= n_here) break;
+      const uint32_t v = __shfl_sync(kFull, w0.x, 4 * j);
+      const uint32_t hdr = __shfl_sync(kFull, w0.x, 4 * j + 1);
+      int64_t t = (hdr & kDfPrev) ? cur : 0;
+      if ((hdr & kDfSlowMask) == 0) {  // the common op: its inputs are the previous op at most
+        cur = t + d0[j];
+        f[(int64_t)v << 5] = cur;
+        last[(hdr & 15) * 32] = cur;
+        mx = max(mx, cur);
+        continue;
+      }
+      // the latest finish among the op's inputs on this rank: the previous op, the
+      // timelines' latest ops (mask), then the other inputs
+      const uint32_t oo = __shfl_sync(kFull, w0.y, 4 * j + 1);
+      for (uint32_t m = hdr >> 16; m; m &= m - 1) t = max(t, last[(__ffs(m) - 1) * 32]);
+      const uint32_t n_extra = (hdr >> 8) & 0xFF;
+      for (uint32_t i = 0; i < n_extra; ++i) {
+        const uint32_t x = __ldg(&a.opnd[oo + i]), p = x & kDfPayload;
+        if ((x >> 30) == kDfInLocal) {
+          t = max(t, f[(int64_t)p << 5]);
+        } else if (!df_gather(xval + ((int64_t)p << 5), 1, ~0u, tag, t, a)) {  // another warp's
+          return;
+        }
+      }
+      int64_t fv = t + d0[j];
+      if (hdr & kDfComm) {
+        const uint32_t slot = __shfl_sync(kFull, w0.x, 4 * j + 2), nmme = __shfl_sync(kFull, w0.y, 4 * j + 2);
+        const uint32_t nm = nmme & 0xFFFF, me = nmme >> 16;
+        if (nm > 1) {
+          if (a.skip_slot != (int64_t)slot + me) st_relaxed_u64(part + ((int64_t)(slot + me) << 5), tag | (uint64_t)t);
+          if (!(hdr & kDfTwoHop) || me == 0) {
+            for (uint32_t m0 = 0; m0 < nm; m0 += 8)  // the other members, 8 at a time
+              if (!df_gather(part + ((int64_t)(slot + m0) << 5), min(nm - m0, 8u), me - m0, tag, t, a)) return;
+            fv = t + d0[j];
+          } else {  // the first member gathers and publishes the finish
+            int64_t u = 0;
+            if (!df_gather(xval + ((int64_t)__shfl_sync(kFull, w0.x, 4 * j + 3) << 5), 1, ~0u, tag, u, a)) return;
+            fv = u;
+          }
+        }
+      }
+      f[(int64_t)v << 5] = fv;  // (every member of a comm op stores the same finish)
+      if (hdr & kDfExport)
+        st_relaxed_u64(xval + ((int64_t)__shfl_sync(kFull, w0.x, 4 * j + 3) << 5), tag | (uint64_t)fv);
+      last[(hdr & 15) * 32] = fv;
+      cur = fv;
+      mx = max(mx, fv);
+    }
+    }
+    w0 = w1;
+    w1 = w2;
+    w2 = w3;
+#pragma unroll
+    for (int j = 0; j < kDfBatch; ++j) d0[j] = d1[j];
+  }
+  if (s < a.S) atomicMax(reinterpret_cast<unsigned long long *>(a.makespan + s), (unsigned long long)mx);
+}
+
+}  // namespace
+
+size_t dataflow_smem_bytes(int32_t n_streams) { return (size_t)(kDfThreads / 32) * n_streams * 32 * sizeof(int64_t); }
+
+bool dataflow_fits(int64_t n_warps, int32_t n_streams, int device) {
+  int sms = 0, coop = 0, per_sm0 = 0, per_sm1 = 0;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+  cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, device);
+  const size_t smem = dataflow_smem_bytes(n_streams);
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm0, compose_dataflow_kernel<false>, kDfThreads, smem) !=
+          cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm1, compose_dataflow_kernel<true>, kDfThreads, smem) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  const int64_t blocks = (n_warps + kDfThreads / 32 - 1) / (kDfThreads / 32);
+  return coop && blocks <= (int64_t)std::min(per_sm0, per_sm1) * sms;
+}
+
+cudaError_t launch_compose_dataflow(const DataflowArgs &a, cudaStream_t st) {
+  const int64_t warps = (int64_t)a.R * a.G;
+  if (warps == 0) return cudaSuccess;
+  const dim3 grid((unsigned)((warps + kDfThreads / 32 - 1) / (kDfThreads / 32))), block(kDfThreads);
+  DataflowArgs args = a;
+  void *params[] = {&args};
+  const size_t smem = dataflow_smem_bytes(a.n_streams);
+  if (a.cdur)
+    return cudaLaunchCooperativeKernel((const void *)compose_dataflow_kernel<true>, grid, block, params, smem, st);
+  return cudaLaunchCooperativeKernel((const void *)compose_dataflow_kernel<false>, grid, block, params, smem, st);
+}
+
+}  // namespace echo

@@ -80,6 +80,11 @@ struct GraphBuild {
   std::vector<int64_t> hin_off;       // [n_seg+1] inputs of each segment's head
   std::vector<int32_t> hin;           // (internal ids, each the tail of an earlier segment)
   int32_t max_kclass = -1;
+  // programs of the dataflow composer (one per rank; see echo_internal.h)
+  bool df_ok = false;
+  std::vector<int64_t> df_off;
+  std::vector<uint32_t> df_rec, df_opnd;
+  int64_t df_slots = 0, df_exports = 0;
   bool stageable = true;              // every head has < 2^16 inputs
 };
 
@@ -188,6 +193,132 @@ void overlap_candidates(GraphBuild &b) {
   for (size_t k = 0; k < b.cand_ops.size(); ++k) b.cand_cidx[k] = b.n_cand ? b.cidx[b.cand_ops[k]] : 0;
   if (b.cand_ops.empty()) b.cand_ops.push_back(0);
   if (b.cand_cidx.empty()) b.cand_cidx.push_back(0);
+}
+
+
+// The dataflow composer's programs: every rank's ops in internal order with their
+// inputs on the rank (the latest op of one of its timelines: shared memory; an
+// earlier op of the rank: its stored finish), the inputs produced by other warps
+// (export flags) and, for comm ops, the partial slots of their members.  A comm
+// op's data producers run on its members, each member taking its own; one that
+// runs on no member is taken by the first member.
+void build_dataflow(GraphBuild &b) {
+  const int64_t V = b.V;
+  const int32_t R = b.R, NS = b.NS;
+  b.df_ok = false;
+  b.df_off.assign(R + 1, 0);
+  b.df_rec.clear();
+  b.df_opnd.clear();
+  if (V >= (int64_t)(echo::kDfPayload + 1u)) return;
+  // ranks of each op, ascending
+  std::vector<int64_t> ro_off(V + 1, 0);
+  for (int64_t q = 0; q < (int64_t)R * NS; ++q)
+    for (int64_t i = b.q_off[q]; i < b.q_off[q + 1]; ++i) ro_off[b.q_ops_int[i] + 1]++;
+  for (int64_t v = 0; v < V; ++v) ro_off[v + 1] += ro_off[v];
+  std::vector<int32_t> ro(std::max<int64_t>(ro_off[V], 1));
+  {
+    std::vector<int64_t> fill(ro_off.begin(), ro_off.end() - 1);
+    for (int64_t q = 0; q < (int64_t)R * NS; ++q)
+      for (int64_t i = b.q_off[q]; i < b.q_off[q + 1]; ++i) ro[fill[b.q_ops_int[i]]++] = (int32_t)(q / NS);
+  }
+  auto runs_on = [&](int32_t u, int32_t r) {
+    return std::binary_search(ro.data() + ro_off[u], ro.data() + ro_off[u + 1], r);
+  };
+  auto members = [&](int32_t v) { return ro_off[v + 1] - ro_off[v]; };
+  // partial slots, and the producers of each comm op that run on none of its members
+  std::vector<int64_t> slot(V, 0);
+  std::vector<uint8_t> uncovered(std::max<int64_t>(b.dp_off[V], 1), 0);
+  b.df_slots = 0;
+  for (int64_t v = 0; v < V; ++v) {
+    if (!b.is_comm[v]) continue;
+    if (members((int32_t)v) > 1) {
+      slot[v] = b.df_slots;
+      b.df_slots += members((int32_t)v);
+    }
+    for (int64_t e = b.dp_off[v]; e < b.dp_off[v + 1]; ++e) {
+      const int32_t u = b.dp[e];
+      bool cov = false;
+      for (int64_t k = ro_off[u]; k < ro_off[u + 1] && !cov; ++k) cov = runs_on((int32_t)v, ro[k]);
+      uncovered[e] = !cov;
+    }
+  }
+  // exports: ops another warp waits for
+  std::vector<int64_t> exp_id(V, -1);
+  b.df_exports = 0;
+  auto export_op = [&](int32_t u) {
+    if (exp_id[u] < 0) exp_id[u] = b.df_exports++;
+  };
+  for (int64_t v = 0; v < V; ++v) {
+    if (b.is_comm[v] && members((int32_t)v) > (int64_t)echo::kDfDirectMembers) export_op((int32_t)v);
+    for (int64_t e = b.dp_off[v]; e < b.dp_off[v + 1]; ++e) {
+      const int32_t u = b.dp[e];
+      if (b.is_comm[v] ? uncovered[e] != 0 : !runs_on(u, ro[ro_off[v]])) export_op(u);
+    }
+  }
+  if (b.df_exports >= (int64_t)(echo::kDfPayload + 1u)) return;
+  // the programs
+  std::vector<std::pair<int32_t, int32_t>> ops;  // (node, timeline) of the rank
+  std::vector<int8_t> tl(V, -1);
+  std::vector<int32_t> last(NS);
+  std::vector<uint32_t> extra;
+  for (int32_t r = 0; r < R; ++r) {
+    ops.clear();
+    for (int32_t k = 0; k < NS; ++k)
+      for (int64_t i = b.q_off[(int64_t)r * NS + k]; i < b.q_off[(int64_t)r * NS + k + 1]; ++i) {
+        ops.emplace_back(b.q_ops_int[i], k);
+        tl[b.q_ops_int[i]] = (int8_t)k;
+      }
+    std::sort(ops.begin(), ops.end());
+    std::fill(last.begin(), last.end(), -1);
+    int32_t prev = -1;  // the op before it in the program
+    for (auto [v, k] : ops) {
+      extra.clear();
+      uint32_t regs = last[k] >= 0 ? 1u << k : 0u;  // the op before it on its timeline
+      const bool comm = b.is_comm[v];
+      const int64_t nm = members(v);
+      const int64_t me = comm ? std::lower_bound(ro.data() + ro_off[v], ro.data() + ro_off[v + 1], r) - (ro.data() + ro_off[v]) : 0;
+      for (int64_t e = b.dp_off[v]; e < b.dp_off[v + 1]; ++e) {
+        const int32_t u = b.dp[e];
+        if (tl[u] >= 0) {  // runs on this rank
+          if (last[tl[u]] == u)
+            regs |= 1u << tl[u];
+          else
+            extra.push_back((echo::kDfInLocal << 30) | (uint32_t)u);
+        } else if (comm ? (uncovered[e] && me == 0) : true) {
+          extra.push_back((echo::kDfInRemote << 30) | (uint32_t)exp_id[u]);
+        }
+      }
+      // the previous op of the program, when an input, comes from a register
+      bool use_prev = false;
+      if (prev >= 0 && ((regs >> tl[prev]) & 1) && last[tl[prev]] == prev) {
+        use_prev = true;
+        regs &= ~(1u << tl[prev]);
+      }
+      const bool two_hop = comm && nm > (int64_t)echo::kDfDirectMembers;
+      const bool publish = exp_id[v] >= 0 && (!comm || me == 0);
+      if (extra.size() > 0xFF || nm > 0xFFFF || b.df_opnd.size() + extra.size() >= (size_t)UINT32_MAX) return;
+      const uint32_t hdr = (uint32_t)k | (comm ? echo::kDfComm : 0u) | (publish ? echo::kDfExport : 0u) |
+                           (two_hop ? echo::kDfTwoHop : 0u) | (use_prev ? echo::kDfPrev : 0u) |
+                           ((uint32_t)extra.size() << 8) | (regs << 16);
+      b.df_rec.push_back((uint32_t)v);
+      b.df_rec.push_back(b.cidx[v] >= 0 ? (uint32_t)b.cidx[v] : ~0u);
+      b.df_rec.push_back(hdr);
+      b.df_rec.push_back((uint32_t)b.df_opnd.size());
+      b.df_rec.push_back(comm ? (uint32_t)slot[v] : 0u);
+      b.df_rec.push_back(comm ? (uint32_t)nm | ((uint32_t)me << 16) : 0u);
+      b.df_rec.push_back(publish || two_hop ? (uint32_t)exp_id[v] : 0u);
+      b.df_rec.push_back(0u);
+      b.df_opnd.insert(b.df_opnd.end(), extra.begin(), extra.end());
+      last[k] = v;
+      prev = v;
+    }
+    for (auto [v, k] : ops) tl[v] = -1;
+    b.df_off[r + 1] = (int64_t)b.df_rec.size() / 8;
+  }
+  if (b.df_slots >= (int64_t)UINT32_MAX) return;
+  if (b.df_rec.empty()) b.df_rec.assign(8, 0);
+  if (b.df_opnd.empty()) b.df_opnd.push_back(0);
+  b.df_ok = true;
 }
 
 // `shape`, when given, replaces the (N, M, K) of every group computed from its
@@ -644,6 +775,7 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e, const std::vect
           return fail(e, ECHO_E_BAD_GRAPH, "internal: segment %lld reads level %d from level %d", (long long)t,
                       lvl[b.seg_int[b.hin[q]]], lvl[t]);
   }
+  build_dataflow(b);
   return ECHO_OK;
 }
 
@@ -1110,7 +1242,15 @@ struct echo_ctx {
   const int64_t *final_cd = nullptr;  // candidates' durations of the last composition (null: the original)
   bool have_ov = false;
   echo::OverlapArgs last_ov{};  // inputs of the last validator pass (to recompute its decisions)
-  int kernel_choice = 0;            // 0 automatic, 1 direct, 2 staged, 3 pipelined (tuning and tests)
+  int kernel_choice = 0;            // 0 automatic, 1 direct, 2 staged, 3 pipelined, 4 dataflow (tuning and tests)
+  // dataflow composer
+  bool use_df = false;
+  int64_t *df_off = nullptr;
+  uint32_t *df_rec = nullptr, *df_opnd = nullptr;
+  uint64_t *df_part = nullptr, *df_xval = nullptr;
+  size_t df_part_elems = 0, df_xval_elems = 0;
+  uint32_t df_epoch = 0;
+  int32_t *df_abort = nullptr;
   int cc_model = ECHO_CC_MODEL_WHITEBOX;
   long long wait_limit_cycles = 0;  // bound of every device-side wait
   int32_t skip_level = -1;          // failure injection for tests
@@ -1284,7 +1424,9 @@ int upload_graph(echo_ctx *c) {
       (rc = upload(c, o, &c->comm_node, B.comm_node)) || (rc = upload(c, o, &c->comm_sig, B.comm_sig)) ||
       (rc = upload(c, o, &c->sig_count, B.sig_count)) || (rc = upload(c, o, &c->kcl, B.kcl)) ||
       (rc = upload(c, o, &c->local, B.local)) ||
-      (rc = upload(c, o, &c->sigs, B.sigs))) {
+      (rc = upload(c, o, &c->sigs, B.sigs)) ||
+      (B.df_ok && ((rc = upload(c, o, &c->df_off, B.df_off)) || (rc = upload(c, o, &c->df_rec, B.df_rec)) ||
+                   (rc = upload(c, o, &c->df_opnd, B.df_opnd))))) {
     free_all(c->graph_allocs);
     return rc;
   }
@@ -1362,7 +1504,7 @@ int echo_create(echo_ctx **out, int device, void *cuda_stream) {
   c->status = static_cast<int32_t *>(st);
   if (const char *e = std::getenv("ECHO_COMPOSE_KERNEL")) {  // tuning and tests: force a compose kernel
     const std::string k(e);
-    c->kernel_choice = k == "direct" ? 1 : k == "staged" ? 2 : k == "pipelined" ? 3 : 0;
+    c->kernel_choice = k == "direct" ? 1 : k == "staged" ? 2 : k == "pipelined" ? 3 : k == "dataflow" ? 4 : 0;
   }
   // device waits give up after 2 s (tests shorten this and inject a level that never arrives)
   int clock_khz = 0;
@@ -1507,13 +1649,17 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     if ((rc = activate_fold(c, h_flag == 0))) return rc;
   }
   const int64_t V = B.V;
-  const int sigma = pick_sigma(S, c->sms);
+  // the dataflow composer works on rows of 32 scenarios
+  const int32_t n_groups = (S + 31) / 32;
+  const bool use_df = c->kernel_choice == 4 && B.df_ok &&
+                      echo::dataflow_fits((int64_t)B.R * n_groups, B.NS, c->device);
+  const int sigma = use_df ? 32 : pick_sigma(S, c->sms);
   int slog2 = 0;
   while ((1 << slog2) < sigma) ++slog2;
   // [op][scenario] matrices are stored in scenario blocks of sigma (the last padded)
   const size_t VS = (size_t)V * (size_t)((S + sigma - 1) / sigma) * sigma;
   const int32_t G = (int32_t)B.sigs.size();
-  if (c->scen_vs != VS || c->S != S || c->C != C || c->sigma != sigma) {
+  if (c->scen_vs != VS || c->S != S || c->C != C || c->sigma != sigma || c->use_df != use_df) {
     free_all(c->scen_allocs);
     c->scen_vs = 0;
     auto &o = c->scen_allocs;
@@ -1533,6 +1679,19 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
       return rc;
     }
     if (in_smem) c->gfrontier = nullptr;
+    c->use_df = use_df;
+    if (use_df) {
+      c->df_part_elems = (size_t)std::max<int64_t>(B.df_slots, 1) * n_groups * 32;
+      c->df_xval_elems = (size_t)std::max<int64_t>(B.df_exports, 1) * n_groups * 32;
+      if ((rc = dalloc(c, o, &c->df_part, c->df_part_elems)) || (rc = dalloc(c, o, &c->df_xval, c->df_xval_elems)) ||
+          (rc = dalloc(c, o, &c->df_abort, 1))) {
+        free_all(c->scen_allocs);
+        return rc;
+      }
+      // zeroed words carry tag 0, which no launch uses
+      CK(cudaMemsetAsync(c->df_part, 0, c->df_part_elems * sizeof(uint64_t), c->stream), "memset");
+      CK(cudaMemsetAsync(c->df_xval, 0, c->df_xval_elems * sizeof(uint64_t), c->stream), "memset");
+    }
     // padding lanes of the duration matrices stay zero
     CK(cudaMemsetAsync(c->dur, 0, VS * sizeof(int64_t), c->stream), "memset");
     CK(cudaMemsetAsync(c->cd[0], 0, CS * sizeof(int64_t), c->stream), "memset");
@@ -1549,11 +1708,12 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     if (const char *e = std::getenv("ECHO_BLOCKS_PER_SM")) bps = std::max(1, std::atoi(e));
     const size_t cap = std::min((size_t)std::max(optin - 1024, 0), (size_t)(per_sm / bps) - 1024);
     // the widest steps whose rings fit
-    for (int64_t step_cap = kStepNodes;; step_cap /= 2) {
+    for (int64_t step_cap = kStepNodes; !use_df; step_cap /= 2) {
       c->steps = make_steps(B, step_cap);
       c->plan = plan_staged(B, c->steps, sigma, cap);
       if (c->plan.ok || step_cap <= 2 * echo::kMaxSegment) break;
     }
+    if (use_df) c->plan = echo::StagedPlan{};
     const Steps &st = c->steps;
     c->plan.threads = threads;
     if (c->plan.ok) {
@@ -1645,6 +1805,9 @@ int echo_estimate_collectives(echo_ctx *c) {
     double bound = c->h_sums[s] * c->h_maxsf[s] + comm[s] + (double)B.V + 1.0;
     if (!(bound < 2305843009213693952.0))
       return set_err(c, ECHO_E_OVERFLOW, "scenario " + std::to_string(s) + ": total duration could overflow int64");
+    if (c->use_df && !(bound < (double)echo::kDfMaxTime))  // it tags times in their top byte
+      return set_err(c, ECHO_E_OVERFLOW, "scenario " + std::to_string(s) + ": times could reach 2^56 ns, "
+                                         "beyond the dataflow composer");
   }
   c->state = 3;
   return ECHO_OK;
@@ -1665,7 +1828,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   const GraphBuild &B = c->gb;
   // the pipelined kernel reads the validator's durations of the candidates from a
   // ring of its own; the others compose from a full matrix built for them
-  const bool ring = c->plan.ok && c->plan.pipelined && (c->kernel_choice == 0 || c->kernel_choice == 3);
+  const bool ring = c->use_df || (c->plan.ok && c->plan.pipelined && (c->kernel_choice == 0 || c->kernel_choice == 3));
   if (refine > 1 && !c->cd[1]) {
     if ((rc = dalloc(c, c->scen_allocs, &c->cd[1], c->cd_elems))) return rc;
     CK(cudaMemsetAsync(c->cd[1], 0, c->cd_elems * sizeof(int64_t), c->stream), "memset");
@@ -1677,6 +1840,37 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   // one composition with durations `d` (and, for the pipelined kernel, the
   // candidates' durations `cdur`) into `f`
   auto compose_pass = [&](const int64_t *d, const int64_t *cdur, int64_t *f) -> cudaError_t {
+    if (c->use_df) {
+      echo::DataflowArgs a{};
+      a.S = c->S;
+      a.G = (c->S + 31) / 32;
+      a.R = B.R;
+      a.n_streams = B.NS;
+      a.V = B.V;
+      a.n_cand = B.n_cand;
+      a.n_slots = std::max<int64_t>(B.df_slots, 1);
+      a.n_exports = std::max<int64_t>(B.df_exports, 1);
+      a.off = c->df_off;
+      a.rec = c->df_rec;
+      a.opnd = c->df_opnd;
+      a.dur = d;
+      a.cdur = cdur;
+      a.f = f;
+      a.part = c->df_part;
+      a.xval = c->df_xval;
+      if ((++c->df_epoch & 0xFF) == 0) ++c->df_epoch;  // (tag 0 marks a word never written)
+      a.epoch = c->df_epoch;
+      a.abort_flag = c->df_abort;
+      a.makespan = c->mk;
+      a.status = c->status;
+      a.wait_limit_cycles = c->wait_limit_cycles;
+      a.skip_slot = c->skip_level;
+      cudaError_t err;
+      if ((err = cudaMemsetAsync(c->mk, 0, (size_t)c->S * sizeof(int64_t), c->stream)) != cudaSuccess ||
+          (err = cudaMemsetAsync(c->df_abort, 0, sizeof(int32_t), c->stream)) != cudaSuccess)
+        return err;
+      return timed(c, "compose", [&] { return echo::launch_compose_dataflow(a, c->stream); });
+    }
     if (c->plan.ok && c->kernel_choice != 1) {
       echo::StagedArgs a{};
       a.S = c->S;
@@ -1775,7 +1969,14 @@ static int composition_status(echo_ctx *c) {
   int32_t st = 0;
   int rc = sync_status(c, &st);
   if (rc) return rc;
-  if (st == echo::kDevTimeout) return set_err(c, ECHO_E_TIMEOUT, "a device-side wait of the composer gave up");
+  if (st == echo::kDevTimeout) {
+    if (c->use_df) {  // words a warp never wrote must not carry a later launch's tag
+      cudaMemsetAsync(c->df_part, 0, c->df_part_elems * sizeof(uint64_t), c->stream);
+      cudaMemsetAsync(c->df_xval, 0, c->df_xval_elems * sizeof(uint64_t), c->stream);
+      cudaStreamSynchronize(c->stream);
+    }
+    return set_err(c, ECHO_E_TIMEOUT, "a device-side wait of the composer gave up");
+  }
   return ECHO_OK;
 }
 

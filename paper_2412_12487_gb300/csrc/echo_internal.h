@@ -154,6 +154,52 @@ struct OverlapArgs {
   uint8_t *ov;             // (out, [V][S] rows of the candidates; may be null)
 };
 
+// Dataflow composer (echo_dataflow.cu): one warp per (rank, group of 32
+// scenarios), matrices in rows of 32 scenarios.  A rank's program lists its ops in
+// internal order, 8 words each: node, level-order candidate index (~0u: none),
+// header, offset of its other inputs in `opnd`, first partial slot (comm ops),
+// member count | own member index << 16 (comm ops), export id (an op whose finish
+// other warps read, or a two-hop join's), 0.  Header: bits 0-3 the op's timeline
+// on the rank, kDf* flags (kDfPrev: the op before it in the program is an input),
+// bits 8-15 the number of other inputs, bits 16-31 the rank's timelines whose
+// latest op is another input.  Other inputs: top 2 bits the
+// kind, an earlier op of the rank (node id) or another warp's op (export id).
+// Published values are times below 2^56 tagged with the launch's epoch in the
+// top byte.
+constexpr int kDfThreads = 32;     // one warp per block
+constexpr int kDfMinBlocks = 21;  // warps per SM to keep resident (80 registers a thread)
+constexpr int kDfBatch = 8;
+constexpr uint32_t kDfPayload = 0x3FFFFFFFu;
+enum : uint32_t { kDfInLocal = 1, kDfInRemote = 2 };
+enum : uint32_t { kDfComm = 1u << 4, kDfPrev = 1u << 5, kDfExport = 1u << 6, kDfTwoHop = 1u << 7 };
+// anything beyond "the previous op of the program is the only input"
+constexpr uint32_t kDfSlowMask = 0xFFFFFF00u | kDfComm | kDfExport | kDfTwoHop;
+constexpr uint32_t kDfDirectMembers = 8;  // larger groups gather at their first member
+constexpr int64_t kDfMaxTime = 1ll << 56;
+
+struct DataflowArgs {
+  int32_t S, G, R, n_streams;  // scenarios, groups of 32 scenarios, ranks, timelines per rank
+  int64_t V, n_cand, n_slots, n_exports;  // rows of dur / f, of cdur, of part, of xval
+  const int64_t *off;          // [R+1] program entries of each rank
+  const uint32_t *rec;         // [entries][8]
+  const uint32_t *opnd;
+  const int64_t *dur;          // durations (comm rows: the CC durations)
+  const int64_t *cdur;         // candidates' durations (compact), or null: dur
+  int64_t *f;                  // finish times
+  uint64_t *part;              // [n_slots][S] tagged partial launch times of comm ops
+  uint64_t *xval;              // [n_exports][S] tagged finishes read by other warps
+  uint32_t epoch;              // this launch's tag (low byte never 0: a zeroed word is never current)
+  int32_t *abort_flag;         // set by a warp whose wait gave up (zeroed before the launch)
+  int64_t *makespan;           // [S] (zeroed before the launch)
+  int32_t *status;
+  long long wait_limit_cycles;
+  int64_t skip_slot;           // failure injection for tests: this partial is never published (-1: none)
+};
+cudaError_t launch_compose_dataflow(const DataflowArgs &a, cudaStream_t st);
+size_t dataflow_smem_bytes(int32_t n_streams);
+// whether every warp of R * G warps can be resident at once (cooperative launch)
+bool dataflow_fits(int64_t n_warps, int32_t n_streams, int device);
+
 // kernels.cu
 cudaError_t launch_cc_estimate(const CcSig *sig, int32_t G, ScenParams p, int32_t S,
                                const ChunkTable &tbl, const int32_t *sig_count, double *cc_ns,

@@ -424,6 +424,58 @@ def test_every_compose_variant_bit_exact(sigma, kernel, monkeypatch):
         e.close()
 
 
+def test_dataflow_compose_bit_exact(monkeypatch):
+    # the dataflow composer (a warp per rank and 32 scenarios, flag-synchronized
+    # joins): GPT-1.3B with full and partial scenario groups and every validator
+    # variant, and random graphs with data edges across ranks (export flags) and
+    # groups of more than 8 members (two-hop joins)
+    monkeypatch.setenv("ECHO_COMPOSE_KERNEL", "dataflow")
+    c = W.config("gpt1.3b")
+    g = W.build_gpt_graph(c)
+    e = Echo(0)
+    try:
+        for S, refine, model, civ in ((32, 0, 0, 0), (37, 1, 0, 0), (64, 2, 1, 1), (5, 1, 0, 1)):
+            sc = W.make_scenarios(g, c, n_scen=S)
+            got = run_gpu(g, sc, refine, ctx=e, overlap_model=model, comm_interval=civ)
+            assert got["info"]["sigma"] == 32
+            want = oracle.compose(g, sc, refine_passes=refine, overlap_model=model, comm_interval=civ,
+                                  threads=THREADS)
+            assert_same(got, want, g, refine)
+        rng = np.random.default_rng(404)
+        for case in range(24):
+            g = SG.random_graph(rng, int(rng.integers(1, 150)), max_ranks=14 if case % 2 else 5,
+                                max_streams=5, p_edge=0.04)
+            sc = SG.random_scenarios(rng, g, int(rng.choice([1, 31, 32, 33, 70])), max_dur=30)
+            got = run_gpu(g, sc, 2, ctx=e)
+            assert_same(got, oracle.compose(g, sc, refine_passes=2), g, 2)
+    finally:
+        e.close()
+
+
+def test_dataflow_bounded_wait_reports_timeout(monkeypatch):
+    # failure detection without a GPU fault: one member never publishes its partial
+    # launch time of a collective, the other members' bounded waits give up after
+    # 20 ms, every warp leaves, and the host reports the timeout
+    c = W.config("gpt1.3b")
+    g = W.build_gpt_graph(c)
+    sc = W.make_scenarios(g, c, n_scen=64)
+    monkeypatch.setenv("ECHO_COMPOSE_KERNEL", "dataflow")
+    monkeypatch.setenv("ECHO_TEST_SKIP_LEVEL", "5")
+    monkeypatch.setenv("ECHO_TEST_WAIT_LIMIT_MS", "20")
+    with Echo(0) as e:
+        e.load_graph(g)
+        e.load_scenarios(sc)
+        e.estimate_collectives()
+        e.compose(refine_passes=0)
+        with pytest.raises(EchoError) as ei:
+            e.read_makespan()
+        assert ei.value.code == 7  # ECHO_E_TIMEOUT
+    monkeypatch.delenv("ECHO_TEST_SKIP_LEVEL")
+    monkeypatch.delenv("ECHO_TEST_WAIT_LIMIT_MS")
+    got = run_gpu(g, sc, 1)
+    assert_same(got, oracle.compose(g, sc, refine_passes=1, threads=THREADS), g, 1)
+
+
 def test_bounded_wait_reports_timeout(monkeypatch):
     # failure detection without a GPU fault: the producer of the pipelined kernel
     # never fills one segment level, every consumer's bounded wait gives up after
