@@ -276,7 +276,10 @@ typedef struct {
   int64_t n_overlap_candidates; /* compute ops the validator tests (the others can never
                                    overlap a comm op of their rank, whatever the durations) */
   int64_t n_ops_composed;    /* ops of the graph being composed                       */
-  int32_t n_ranks, n_streams, sigma; /* sigma: scenarios per thread block of the composer */
+  int32_t n_ranks, n_streams, sigma; /* sigma: scenarios per thread block of the composer;
+                                        32: the dataflow composer (a warp per rank and 32
+                                        scenarios), chosen for graphs with many levels and
+                                        few scenarios */
   int32_t replicas_folded;
 } echo_graph_info;
 int echo_graph_info_get(echo_ctx *ctx, echo_graph_info *info);

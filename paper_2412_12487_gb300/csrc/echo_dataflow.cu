@@ -13,9 +13,10 @@
 //     Groups of more than 8 members gather at one member, which publishes the
 //     finish;
 //   - a data input produced on another rank: its producer publishes its finish.
-// A published value is one 64-bit word per scenario: the time (below 2^56) with
-// the launch's 8-bit tag in the top byte, written by one relaxed store and polled
-// by relaxed loads, so no flag, fence or reset is needed between launches.  Every
+// A published value is one 64-bit word per scenario: the time (below 2^61, which
+// the host guarantees) with the launch's tag (1-7) in the top 3 bits, written by
+// one relaxed store and polled by relaxed loads, so neither flags nor fences are
+// needed; the host zeroes the words whenever the tags start over.  Every
 // warp is resident (cooperative launch) and waits only for ops earlier in the
 // topological order, so the earliest unfinished op can always proceed.  Every
 // wait is bounded: a warp that gives up sets the abort flag and the timeout
@@ -31,7 +32,7 @@ namespace echo {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr uint64_t kValueMask = (1ull << 56) - 1;
+constexpr uint64_t kValueMask = (1ull << 61) - 1;
 
 __device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t *p) {
   uint64_t v;
@@ -100,7 +101,7 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
   int64_t *f = a.f + (((int64_t)g * a.V) << 5) + lane;
   uint64_t *part = a.part + (((int64_t)g * a.n_slots) << 5) + lane;
   uint64_t *xval = a.xval + (((int64_t)g * a.n_exports) << 5) + lane;
-  const uint64_t tag = (uint64_t)(a.epoch & 0xFF) << 56;
+  const uint64_t tag = (uint64_t)a.epoch << 61;
   const int64_t e0 = a.off[r], e1 = a.off[r + 1];
   int64_t mx = 0;
   // batches of 8 entries of 8 words: lane l holds words 2(l % 4) and 2(l % 4) + 1

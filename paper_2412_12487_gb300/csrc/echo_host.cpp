@@ -1649,10 +1649,19 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     if ((rc = activate_fold(c, h_flag == 0))) return rc;
   }
   const int64_t V = B.V;
-  // the dataflow composer works on rows of 32 scenarios
+  // The dataflow composer (rows of 32 scenarios, a warp per rank) is serial in
+  // the length of the longest rank program, the levelled ones in their number
+  // of steps; measured on GB300 a program entry costs about 0.25-0.55 us and a
+  // step about 1.2-1.8 us, so it is chosen when the longest program is shorter
+  // than 2.5 steps per entry (and every warp can be resident).
   const int32_t n_groups = (S + 31) / 32;
-  const bool use_df = c->kernel_choice == 4 && B.df_ok &&
-                      echo::dataflow_fits((int64_t)B.R * n_groups, B.NS, c->device);
+  bool use_df = false;
+  if (B.df_ok && (c->kernel_choice == 0 || c->kernel_choice == 4) &&
+      echo::dataflow_fits((int64_t)B.R * n_groups, B.NS, c->device)) {
+    int64_t longest = 0;
+    for (int32_t r = 0; r < B.R; ++r) longest = std::max(longest, B.df_off[r + 1] - B.df_off[r]);
+    use_df = c->kernel_choice == 4 || 2 * longest < 5 * make_steps(B, kStepNodes).L;
+  }
   const int sigma = use_df ? 32 : pick_sigma(S, c->sms);
   int slog2 = 0;
   while ((1 << slog2) < sigma) ++slog2;
@@ -1805,9 +1814,6 @@ int echo_estimate_collectives(echo_ctx *c) {
     double bound = c->h_sums[s] * c->h_maxsf[s] + comm[s] + (double)B.V + 1.0;
     if (!(bound < 2305843009213693952.0))
       return set_err(c, ECHO_E_OVERFLOW, "scenario " + std::to_string(s) + ": total duration could overflow int64");
-    if (c->use_df && !(bound < (double)echo::kDfMaxTime))  // it tags times in their top byte
-      return set_err(c, ECHO_E_OVERFLOW, "scenario " + std::to_string(s) + ": times could reach 2^56 ns, "
-                                         "beyond the dataflow composer");
   }
   c->state = 3;
   return ECHO_OK;
@@ -1858,14 +1864,21 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       a.f = f;
       a.part = c->df_part;
       a.xval = c->df_xval;
-      if ((++c->df_epoch & 0xFF) == 0) ++c->df_epoch;  // (tag 0 marks a word never written)
+      // tags run 1..7; before they start over, every word is zeroed so that none
+      // written (or left unwritten by an aborted launch) carries a current tag
+      cudaError_t err;
+      if (++c->df_epoch > 7) {
+        c->df_epoch = 1;
+        if ((err = cudaMemsetAsync(c->df_part, 0, c->df_part_elems * sizeof(uint64_t), c->stream)) != cudaSuccess ||
+            (err = cudaMemsetAsync(c->df_xval, 0, c->df_xval_elems * sizeof(uint64_t), c->stream)) != cudaSuccess)
+          return err;
+      }
       a.epoch = c->df_epoch;
       a.abort_flag = c->df_abort;
       a.makespan = c->mk;
       a.status = c->status;
       a.wait_limit_cycles = c->wait_limit_cycles;
       a.skip_slot = c->skip_level;
-      cudaError_t err;
       if ((err = cudaMemsetAsync(c->mk, 0, (size_t)c->S * sizeof(int64_t), c->stream)) != cudaSuccess ||
           (err = cudaMemsetAsync(c->df_abort, 0, sizeof(int32_t), c->stream)) != cudaSuccess)
         return err;

@@ -164,8 +164,8 @@ struct OverlapArgs {
 // bits 8-15 the number of other inputs, bits 16-31 the rank's timelines whose
 // latest op is another input.  Other inputs: top 2 bits the
 // kind, an earlier op of the rank (node id) or another warp's op (export id).
-// Published values are times below 2^56 tagged with the launch's epoch in the
-// top byte.
+// Published values are times (below 2^61) tagged with the launch's epoch (1-7)
+// in the top 3 bits.
 constexpr int kDfThreads = 32;     // one warp per block
 constexpr int kDfMinBlocks = 21;  // warps per SM to keep resident (80 registers a thread)
 constexpr int kDfBatch = 8;
@@ -175,7 +175,6 @@ enum : uint32_t { kDfComm = 1u << 4, kDfPrev = 1u << 5, kDfExport = 1u << 6, kDf
 // anything beyond "the previous op of the program is the only input"
 constexpr uint32_t kDfSlowMask = 0xFFFFFF00u | kDfComm | kDfExport | kDfTwoHop;
 constexpr uint32_t kDfDirectMembers = 8;  // larger groups gather at their first member
-constexpr int64_t kDfMaxTime = 1ll << 56;
 
 struct DataflowArgs {
   int32_t S, G, R, n_streams;  // scenarios, groups of 32 scenarios, ranks, timelines per rank
@@ -188,7 +187,7 @@ struct DataflowArgs {
   int64_t *f;                  // finish times
   uint64_t *part;              // [n_slots][S] tagged partial launch times of comm ops
   uint64_t *xval;              // [n_exports][S] tagged finishes read by other warps
-  uint32_t epoch;              // this launch's tag (low byte never 0: a zeroed word is never current)
+  uint32_t epoch;              // this launch's tag, 1-7 (0 marks a word never written)
   int32_t *abort_flag;         // set by a warp whose wait gave up (zeroed before the launch)
   int64_t *makespan;           // [S] (zeroed before the launch)
   int32_t *status;
