@@ -85,15 +85,24 @@ __device__ bool df_gather(const uint64_t *p, uint32_t n, uint32_t skip, uint64_t
   return true;
 }
 
+__device__ __forceinline__ void cp_async_8(void *smem, const void *gmem) {
+  const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(sa), "l"(gmem) : "memory");
+}
+
 template <bool CAND>
 __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_kernel(DataflowArgs a) {
-  extern __shared__ int64_t df_last[];  // [warps][n_streams][32]: latest finish of each timeline
+  // per warp: the duration ring [kDfDepth + 1][kDfBatch][32], then [n_streams][32]
+  // latest finishes of the rank's timelines
+  extern __shared__ int64_t df_smem[];
+  int64_t *dring = df_smem + (int64_t)(threadIdx.x >> 5) * ((kDfDepth + 1) * kDfBatch * 32 + a.n_streams * 32);
+  int64_t *df_last = dring + (kDfDepth + 1) * kDfBatch * 32;
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const int64_t wid = (int64_t)blockIdx.x * (kDfThreads / 32) + wib;
   if (wid >= (int64_t)a.R * a.G) return;  // uniform over the warp
   const int32_t r = (int32_t)(wid % a.R), g = (int32_t)(wid / a.R);
   const int32_t s = g * 32 + lane;
-  int64_t *last = df_last + (int64_t)wib * a.n_streams * 32 + lane;
+  int64_t *last = df_last + lane;
   for (int k = 0; k < a.n_streams; ++k) last[k * 32] = 0;
   // rows of 32 scenarios: element (i, s) of an [n][S] matrix at ((g * n + i) << 5) + lane
   const int64_t *dur = a.dur + (((int64_t)g * a.V) << 5) + lane;
@@ -105,27 +114,32 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
   const int64_t e0 = a.off[r], e1 = a.off[r + 1];
   int64_t mx = 0;
   // batches of 8 entries of 8 words: lane l holds words 2(l % 4) and 2(l % 4) + 1
-  // of entry l / 4.  Records are loaded three batches ahead of their use, the
-  // durations one batch ahead.
+  // of entry l / 4.  Records are loaded kDfDepth + 1 batches ahead of their use;
+  // each lane copies its own duration elements kDfDepth batches ahead into the
+  // ring (cp.async, one commit group per batch), and reads only its own.
   auto rec = [&](int64_t b) -> uint2 {
     return b + lane / 4 < e1 ? __ldg(reinterpret_cast<const uint2 *>(a.rec) + 4 * b + lane) : make_uint2(0, 0);
   };
-  auto durs = [&](int64_t b, uint2 w, int64_t(&d)[kDfBatch]) {
+  auto durs = [&](int64_t b, uint2 w) {  // copies batch b's durations into its ring slot
+    int64_t *slot = dring + ((b - e0) / kDfBatch % (kDfDepth + 1)) * (kDfBatch * 32) + lane;
 #pragma unroll
     for (int j = 0; j < kDfBatch; ++j) {
       const uint32_t v = __shfl_sync(kFull, w.x, 4 * j), ci = __shfl_sync(kFull, w.y, 4 * j);
-      d[j] = 0;
-      if (b + j < e1) d[j] = (CAND && ci != ~0u) ? cdu[(int64_t)ci << 5] : dur[(int64_t)v << 5];
+      if (b + j < e1) cp_async_8(slot + j * 32, (CAND && ci != ~0u) ? cdu + ((int64_t)ci << 5) : dur + ((int64_t)v << 5));
     }
+    asm volatile("cp.async.commit_group;" ::: "memory");
   };
-  uint2 w0 = rec(e0), w1 = rec(e0 + kDfBatch), w2 = rec(e0 + 2 * kDfBatch);
-  int64_t d0[kDfBatch];
-  durs(e0, w0, d0);
+  static_assert(kDfDepth == 3, "the record registers below hold kDfDepth + 1 batches");
+  uint2 w0 = rec(e0), w1 = rec(e0 + kDfBatch), w2 = rec(e0 + 2 * kDfBatch), w3 = rec(e0 + 3 * kDfBatch);
+  durs(e0, w0);
+  durs(e0 + kDfBatch, w1);
+  durs(e0 + 2 * kDfBatch, w2);
   int64_t cur = 0;  // finish of the previous op of the program
   for (int64_t b = e0; b < e1; b += kDfBatch) {
-    const uint2 w3 = rec(b + 3 * kDfBatch);
-    int64_t d1[kDfBatch];
-    durs(b + kDfBatch, w1, d1);
+    const uint2 w4 = rec(b + 4 * kDfBatch);
+    durs(b + 3 * kDfBatch, w3);
+    asm volatile("cp.async.wait_group 3;" ::: "memory");  // this batch's group is complete
+    const int64_t *d0 = dring + ((b - e0) / kDfBatch % (kDfDepth + 1)) * (kDfBatch * 32) + lane;
     const int n_here = e1 - b < kDfBatch ? (int)(e1 - b) : kDfBatch;
     // a full batch of common ops (inputs: the previous op at most) runs branch-free
     bool plain = n_here == kDfBatch;
@@ -135,7 +149,7 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
 #pragma unroll
       for (int j = 0; j < kDfBatch; ++j) {
         const uint32_t v = __shfl_sync(kFull, w0.x, 4 * j), hdr = __shfl_sync(kFull, w0.x, 4 * j + 1);
-        cur = ((hdr & kDfPrev) ? cur : 0) + d0[j];
+        cur = ((hdr & kDfPrev) ? cur : 0) + d0[j * 32];
         f[(int64_t)v << 5] = cur;
         last[(hdr & 15) * 32] = cur;
         mx = max(mx, cur);
@@ -148,7 +162,7 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
       const uint32_t hdr = __shfl_sync(kFull, w0.x, 4 * j + 1);
       int64_t t = (hdr & kDfPrev) ? cur : 0;
       if ((hdr & kDfSlowMask) == 0) {  // the common op: its inputs are the previous op at most
-        cur = t + d0[j];
+        cur = t + d0[j * 32];
         f[(int64_t)v << 5] = cur;
         last[(hdr & 15) * 32] = cur;
         mx = max(mx, cur);
@@ -164,10 +178,11 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
         if ((x >> 30) == kDfInLocal) {
           t = max(t, f[(int64_t)p << 5]);
         } else if (!df_gather(xval + ((int64_t)p << 5), 1, ~0u, tag, t, a)) {  // another warp's
+          asm volatile("cp.async.wait_all;" ::: "memory");  // (its own copies land before it leaves)
           return;
         }
       }
-      int64_t fv = t + d0[j];
+      int64_t fv = t + d0[j * 32];
       if (hdr & kDfComm) {
         const uint32_t slot = __shfl_sync(kFull, w0.x, 4 * j + 2), nmme = __shfl_sync(kFull, w0.y, 4 * j + 2);
         const uint32_t nm = nmme & 0xFFFF, me = nmme >> 16;
@@ -175,11 +190,17 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
           if (a.skip_slot != (int64_t)slot + me) st_relaxed_u64(part + ((int64_t)(slot + me) << 5), tag | (uint64_t)t);
           if (!(hdr & kDfTwoHop) || me == 0) {
             for (uint32_t m0 = 0; m0 < nm; m0 += 8)  // the other members, 8 at a time
-              if (!df_gather(part + ((int64_t)(slot + m0) << 5), min(nm - m0, 8u), me - m0, tag, t, a)) return;
-            fv = t + d0[j];
+              if (!df_gather(part + ((int64_t)(slot + m0) << 5), min(nm - m0, 8u), me - m0, tag, t, a)) {
+                asm volatile("cp.async.wait_all;" ::: "memory");
+                return;
+              }
+            fv = t + d0[j * 32];
           } else {  // the first member gathers and publishes the finish
             int64_t u = 0;
-            if (!df_gather(xval + ((int64_t)__shfl_sync(kFull, w0.x, 4 * j + 3) << 5), 1, ~0u, tag, u, a)) return;
+            if (!df_gather(xval + ((int64_t)__shfl_sync(kFull, w0.x, 4 * j + 3) << 5), 1, ~0u, tag, u, a)) {
+              asm volatile("cp.async.wait_all;" ::: "memory");
+              return;
+            }
             fv = u;
           }
         }
@@ -195,15 +216,17 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
     w0 = w1;
     w1 = w2;
     w2 = w3;
-#pragma unroll
-    for (int j = 0; j < kDfBatch; ++j) d0[j] = d1[j];
+    w3 = w4;
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
   if (s < a.S) atomicMax(reinterpret_cast<unsigned long long *>(a.makespan + s), (unsigned long long)mx);
 }
 
 }  // namespace
 
-size_t dataflow_smem_bytes(int32_t n_streams) { return (size_t)(kDfThreads / 32) * n_streams * 32 * sizeof(int64_t); }
+size_t dataflow_smem_bytes(int32_t n_streams) {
+  return (size_t)(kDfThreads / 32) * ((kDfDepth + 1) * kDfBatch * 32 + n_streams * 32) * sizeof(int64_t);
+}
 
 bool dataflow_fits(int64_t n_warps, int32_t n_streams, int device) {
   int sms = 0, coop = 0, per_sm0 = 0, per_sm1 = 0;

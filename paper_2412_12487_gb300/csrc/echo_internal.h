@@ -169,6 +169,7 @@ struct OverlapArgs {
 constexpr int kDfThreads = 32;     // one warp per block
 constexpr int kDfMinBlocks = 21;  // warps per SM to keep resident (80 registers a thread)
 constexpr int kDfBatch = 8;
+constexpr int kDfDepth = 3;       // batches of durations in flight ahead of the one in use
 constexpr uint32_t kDfPayload = 0x3FFFFFFFu;
 enum : uint32_t { kDfInLocal = 1, kDfInRemote = 2 };
 enum : uint32_t { kDfComm = 1u << 4, kDfPrev = 1u << 5, kDfExport = 1u << 6, kDfTwoHop = 1u << 7 };
