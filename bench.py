@@ -155,12 +155,12 @@ def pinned_host_array(shape, dtype=np.int64):
         return torch.from_numpy(np.empty(0, dtype)).new_empty(shape).pin_memory()
 
 
-def build_inputs(rank, world, n_scen=None, pinned=True):
+def build_inputs(rank, world, n_scen=None, pinned=True, workload=WORKLOAD):
     """The graph and this rank's slice of a batch of n_scen * world scenarios."""
     import torch
     from paper_2412_12487_gb300 import sharding as SH
     from paper_2412_12487_gb300 import workloads as W
-    c = W.config(WORKLOAD)
+    c = W.config(workload)
     c = W.GPTConfig(**{**c.__dict__, "n_scen": n_scen or c.n_scen})
     t0 = time.time()
     g = W.build_gpt_graph(c)
@@ -191,7 +191,7 @@ def run_echo(args):
     torch.cuda.set_device(local)
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    c, g, sc, dur_t = build_inputs(rank, world, args.scenarios)
+    c, g, sc, dur_t = build_inputs(rank, world, args.scenarios, workload=args.workload)
     V, S = g.n_ops, sc.n_scen
     # a stream of its own: the events below and every library launch share it
     stream = torch.cuda.Stream(local)
@@ -286,7 +286,9 @@ def run_echo(args):
     b_pass = algorithmic_bytes_per_pass(g, info, S)
     per_launch_ms = comp_ms / max(comp_launches, 1)
     achieved = b_pass / (per_launch_ms / 1e3) / 1e9 if comp_launches else None
-    traffic = profiled_traffic(V * S)
+    composer = "dataflow" if info["sigma"] == 32 else "levelled"
+    # the committed capture is of the levelled composer on this workload
+    traffic = profiled_traffic(V * S) if args.workload == WORKLOAD and composer == "levelled" else None
     out = None
     if rank == 0:
         cpu = cpu_baseline(g, c, args) if world == 1 and args.cpu_sample > 0 else None
@@ -297,7 +299,7 @@ def run_echo(args):
             "vs_baseline": None, "dtype": "int64", "data": "synthetic",
             "config": {"workload": f"{c.name} x {S} scenarios per GPU", "ops": V, "edges": g.n_edges,
                        "levels": info["n_levels"], "scenarios_per_gpu": S, "refine_passes": 1,
-                       "sigma": info["sigma"],
+                       "sigma": info["sigma"], "composer": composer,
                        "updates_per_step": units,
                        "l2": f"no flush: the {V * S * 8 / 1e9:.1f} GB duration matrix and the "
                              f"finish matrices each exceed the 129 MB L2"},
@@ -346,7 +348,7 @@ def run_reference(args):
         return None
     import oracle
     from paper_2412_12487_gb300 import workloads as W
-    c = W.config(WORKLOAD)
+    c = W.config(args.workload)
     g = W.build_gpt_graph(c)
     base = W.scenario_params(c)
     oracle.build()
@@ -380,6 +382,8 @@ def main():
     ap.add_argument("--impl", default="echo", choices=["echo", "reference"])
     ap.add_argument("--cpu-sample", type=int, default=8,
                     help="scenarios of the CPU-oracle baseline sample (0 = skip)")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    help="workload name (default: the GPT-175B step); others for profiling and comparison")
     ap.add_argument("--scenarios", type=int, default=None,
                     help="scenarios per GPU (default: the workload's 1024); smaller values "
                          "make small cases for profiling")
