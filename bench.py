@@ -329,7 +329,7 @@ def cpu_baseline(g, c, args, n_sample=None):
     same workload (the first scenarios of the batch)."""
     import oracle
     from paper_2412_12487_gb300 import workloads as W
-    n_sample = n_sample or args.cpu_sample
+    n_sample = min(n_sample or args.cpu_sample, c.n_scen)
     sub = W.select_scenarios(W.scenario_params(c), g, list(range(n_sample)))
     t0 = time.time()
     oracle.compose(g, sub, refine_passes=1, threads=1, want_cc=False, want_overlap=False)
@@ -338,6 +338,56 @@ def cpu_baseline(g, c, args, n_sample=None):
             "sample": f"{n_sample} of the {c.n_scen} scenarios of {c.name} ({g.n_ops} ops), "
                       f"CC estimate + 2 compositions + overlap, {dt:.1f} s single-threaded",
             "seconds": dt, "host_cores_available": os.cpu_count()}
+
+
+CCQ_WORKLOAD = "cc-queries"
+
+
+def run_cc_queries(args):
+    """The standalone CC-estimator sweep (1M queries of Sec. 5.3's closed forms):
+    queries/s of the estimator kernel (device time) and through the C ABI call
+    (host arrays in, host results out), with the oracle's rate on a sample."""
+    import torch
+    import oracle
+    from paper_2412_12487_gb300 import Echo
+    from paper_2412_12487_gb300 import workloads as W
+    n = args.scenarios or 1_000_000
+    q = W.make_cc_queries(n)
+    stream = torch.cuda.Stream(0)
+    torch.cuda.set_stream(stream)
+    with Echo(0, stream) as e:
+        for _ in range(args.warmup):
+            e.cc_query(q)
+        e.set_profiling(True)
+        e.read_profile()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            out = e.cc_query(q)
+        torch.cuda.synchronize()
+        call_ms = (time.perf_counter() - t0) / args.steps * 1e3
+        prof = e.read_profile()
+    k_n, k_ms = prof.get("cc_query", (0, 0.0))
+    kern_ms = k_ms / max(k_n, 1)
+    oracle.build()
+    m = min(n, 20000)
+    t0 = time.perf_counter()
+    ref = np.array([oracle.cc_ns(int(q.cc_type[i]), int(q.cc_algo[i]), int(q.nbytes[i]), int(q.n_ranks[i]),
+                                 int(q.n_nodes[i]), -(-int(q.n_ranks[i]) // int(q.n_nodes[i])),
+                                 float(np.log2(q.n_nodes[i])), float(q.alpha_ns[i]), float(q.bw_intra[i]),
+                                 float(q.lat_intra[i]), float(q.bw_inter[i]), float(q.lat_inter[i]),
+                                 float(q.delta[i])) for i in range(m)])
+    cpu_s = time.perf_counter() - t0
+    rel = float(np.max(np.abs(out[:m] - ref) / np.maximum(np.abs(ref), 1e-300)))
+    return {"metric": "CC-estimator queries/s", "value": n / (kern_ms / 1e3), "unit": "queries/s",
+            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": kern_ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": f"{n} CC-estimator queries (Sec. 5.3)"},
+            "e2e": {"value": n / (call_ms / 1e3), "unit": "queries/s", "ms_per_step": call_ms,
+                    "h2d_bytes_per_step": n * (1 + 1 + 8 + 4 + 4 + 6 * 8), "d2h_bytes_per_step": n * 8},
+            "max_rel_diff_vs_oracle_sample": rel,
+            "cpu_baseline": {"value": m / cpu_s, "unit": "queries/s", "cores": 1, "kind": "oracle",
+                             "sample": f"first {m} queries, one at a time through the oracle's C function"}}
 
 
 def run_reference(args):
@@ -393,6 +443,10 @@ def main():
         args.warmup = 3
     if args.impl == "reference":
         out = run_reference(args)
+    elif args.workload == CCQ_WORKLOAD:
+        import __graft_entry__
+        __graft_entry__.build()
+        out = run_cc_queries(args)
     else:
         import __graft_entry__
         __graft_entry__.build()

@@ -232,9 +232,9 @@ __global__ void permute_rows_kernel(const T *__restrict__ raw, const int32_t *__
 constexpr int kOverlapThreads = 128;
 constexpr int kOverlapBatch = 8;  // divides 32 (the shuffled op list's width)
 // LAUNCH: a comm op's interval on the rank opens at the rank's launch of it
-// (a.lq_off), else at its start
-template <int NCMAX, bool LAUNCH>
-__global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a) {
+// (a.lq_off), else at its start.  PROP: the proportional slowdown model (a.model 1)
+template <int NCMAX, bool LAUNCH, bool PROP>
+__global__ void __launch_bounds__(kOverlapThreads, 8) overlap_kernel(OverlapArgs a) {  // 64 registers: occupancy hides its row-load latency
   const int32_t S = a.S;
   const int32_t s = blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t c = blockIdx.y + (int64_t)gridDim.y * blockIdx.z;
@@ -345,7 +345,7 @@ __global__ void __launch_bounds__(kOverlapThreads) overlap_kernel(OverlapArgs a)
         if (cn) {
           const int64_t d0 = cu ? du[v << sh] : dv;  // the original duration
           int64_t dn = d0;
-          if (hit && a.model == 1) {
+          if (PROP && hit) {
             // proportional model: the length of [sv, fv) covered by the union of the
             // comm intervals, swept in start order across the timelines.  Later
             // candidates start no earlier than fv, so a cursor moves past every
@@ -545,25 +545,26 @@ cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
   int64_t gy = a.n_chunks < 65535 ? a.n_chunks : 65535;
   int64_t gz = (a.n_chunks + gy - 1) / gy;
   dim3 grid((a.S + tx - 1) / tx, (unsigned)gy, (unsigned)gz);
-  auto go = [&](auto launch) {
-    constexpr bool L = decltype(launch)::value;
+  auto go = [&](auto launch, auto prop) {
+    constexpr bool L = decltype(launch)::value, P = decltype(prop)::value;
     if (a.n_cq <= 1)
-      overlap_kernel<1, L><<<grid, tx, 0, st>>>(a);
+      overlap_kernel<1, L, P><<<grid, tx, 0, st>>>(a);
     else if (a.n_cq <= 2)
-      overlap_kernel<2, L><<<grid, tx, 0, st>>>(a);
+      overlap_kernel<2, L, P><<<grid, tx, 0, st>>>(a);
     else if (a.n_cq <= 3)
-      overlap_kernel<3, L><<<grid, tx, 0, st>>>(a);
+      overlap_kernel<3, L, P><<<grid, tx, 0, st>>>(a);
     else if (a.n_cq <= 4)
-      overlap_kernel<4, L><<<grid, tx, 0, st>>>(a);
+      overlap_kernel<4, L, P><<<grid, tx, 0, st>>>(a);
     else if (a.n_cq <= 8)
-      overlap_kernel<8, L><<<grid, tx, 0, st>>>(a);
+      overlap_kernel<8, L, P><<<grid, tx, 0, st>>>(a);
     else
-      overlap_kernel<kMaxStreams, L><<<grid, tx, 0, st>>>(a);
+      overlap_kernel<kMaxStreams, L, P><<<grid, tx, 0, st>>>(a);
   };
+  const bool prop = a.model == 1 && a.cd_next;
   if (a.lq_off)
-    go(std::true_type{});
+    prop ? go(std::true_type{}, std::true_type{}) : go(std::true_type{}, std::false_type{});
   else
-    go(std::false_type{});
+    prop ? go(std::false_type{}, std::true_type{}) : go(std::false_type{}, std::false_type{});
   return cudaGetLastError();
 }
 
