@@ -41,6 +41,9 @@ KIND_COMPUTE, KIND_MEMCPY, KIND_COLL, KIND_P2P = 0, 1, 2, 3
 CC_ALLREDUCE, CC_ALLGATHER, CC_REDUCESCATTER, CC_SENDRECV = 0, 1, 2, 3
 ALGO_RING, ALGO_TREE, ALGO_AUTO = 0, 1, 2
 STREAM_COMPUTE, STREAM_TP, STREAM_PP, STREAM_DP, STREAM_MEMCPY = 0, 1, 2, 3, 4
+# interleaved schedules: activation receives (STREAM_PP holds the sends), gradient
+# sends and gradient receives on timelines of their own
+STREAM_PP_RECV, STREAM_PP_GRAD, STREAM_PP_GRAD_RECV = 5, 6, 7
 N_STREAMS = 5
 
 # kernel classes (the kernel types the slowdown statistics of Sec. 2.3 distinguish)
@@ -144,6 +147,8 @@ class GPTConfig:
     # DP replicas that run identical kernels (each replica op takes its replica-0
     # original's noise draw); the graph then carries replica_of for folding
     identical_replicas: bool = False
+    # model chunks per rank: 1 = 1F1B, v > 1 = interleaved 1F1B over PP * v virtual stages
+    virtual_stages: int = 1
 
 
 # The five workloads (GPT shapes of Table 7; 3D-parallel layouts as in Sec. 8).
@@ -154,15 +159,16 @@ CONFIGS: Dict[str, GPTConfig] = {
                          scen_seed=1002),
     "gpt175b": GPTConfig("gpt-175b-tp8pp6dp2-m16", 96, 12288, 96, 2048, 8, 6, 2, 16, 1024,
                          scen_seed=1003),
-    "gpt175b-1024": GPTConfig("gpt-175b-tp8pp16dp8-m64", 96, 12288, 96, 2048, 8, 16, 8, 64, 64,
-                              scen_seed=1004),
+    "gpt175b-1024": GPTConfig("gpt-175b-tp8pp16dp8-m64-v2", 96, 12288, 96, 2048, 8, 16, 8, 64, 64,
+                              scen_seed=1004, virtual_stages=2),
 }
 
 
 # ---------------------------------------------------------------------------------------
 # per-stage program (template shared by every rank of a pipeline stage)
 # ---------------------------------------------------------------------------------------
-_E_COMP, _E_MEMCPY, _E_TP, _E_P2P, _E_DP, _E_WORLD = range(6)
+_E_COMP, _E_MEMCPY, _E_TP, _E_P2P, _E_DP, _E_WORLD, _E_P2P_RECV, _E_P2P_GRAD, _E_P2P_GRAD_RECV = range(9)
+_E_P2P_ALL = (_E_P2P, _E_P2P_RECV, _E_P2P_GRAD, _E_P2P_GRAD_RECV)
 
 
 class _StageProgram:
@@ -405,6 +411,148 @@ def _stage_program(c: GPTConfig, p: int) -> _StageProgram:
     return prog
 
 
+def _stage_program_interleaved(c: GPTConfig, p: int) -> _StageProgram:
+    """Issue order of one rank of pipeline stage ``p`` under interleaved 1F1B: the
+    rank holds v model chunks, chunk ch being virtual stage s = ch * PP + p of
+    PP * v, each with layers / (PP * v) layers.  Virtual microbatch k runs
+    microbatch (k // (PP * v)) * PP + k % PP on chunk (k // PP) % v (backwards
+    take the chunks in reverse); a rank runs (PP - p - 1) * 2 + (v - 1) * PP
+    forwards before its first backward (all of them when m == PP), then
+    alternates.
+
+    Every transfer between consecutive virtual stages is its own 2-member P2P
+    node, keyed by ('fa' | 'g', lower physical stage, lower virtual stage,
+    microbatch).  Sends and receives of activations and of gradients each take a
+    timeline of their own (the schedule's batched asynchronous send/recv calls do
+    not wait for one another), so every such timeline carries one link's transfers
+    of one kind, which both ends issue in the same (forward or backward) order."""
+    PP, m, tp, dp, v = c.pp, c.microbatches, c.tp, c.dp, c.virtual_stages
+    if c.layers % (PP * v):
+        raise ValueError("layers must divide evenly across the virtual pipeline stages")
+    if m % PP:
+        raise ValueError("interleaved 1F1B needs microbatches divisible by the pipeline stages")
+    nl = c.layers // (PP * v)
+    b, h = c.seq, c.hidden
+    act_bytes = b * h * 2
+    prog = _StageProgram()
+    fwd = _fwd_kernels(c)
+    bwd = _bwd_kernels(c)
+    M = MEM_FLOP_PER_BYTE
+    n_virtual = PP * v
+    dp_entries: List[int] = []
+    bucket = [0.0]
+    act_out: Dict[Tuple[int, int], int] = {}
+
+    def tp_ar(dep):
+        return prog.comm(_E_TP, act_bytes, CC_ALLREDUCE, ALGO_AUTO, None, deps=[dep])
+
+    def flush_bucket(dep):
+        if dp > 1 and bucket[0] > 0:
+            e = prog.comm(_E_DP, int(bucket[0]) * 2, CC_ALLREDUCE, ALGO_AUTO, len(dp_entries), deps=[dep])
+            dp_entries.append(e)
+        bucket[0] = 0.0
+
+    def add_grad(params, dep, last_mb):
+        if last_mb and dp > 1:
+            bucket[0] += params
+            if bucket[0] >= DP_BUCKET_ELEMS:
+                flush_bucket(dep)
+
+    def xfer(kind, s, mb, send, deps=()):
+        et = {("fa", True): _E_P2P, ("fa", False): _E_P2P_RECV,
+              ("g", True): _E_P2P_GRAD, ("g", False): _E_P2P_GRAD_RECV}[(kind, send)]
+        return prog.comm(et, act_bytes, CC_SENDRECV, ALGO_RING, (kind, s % PP, s, mb), deps=deps)
+
+    def F(mb, ch):
+        s = ch * PP + p
+        dep = xfer("fa", s - 1, mb, False) if s > 0 else None
+        if s == 0:
+            mc = prog.memcpy(b * 8)
+            dep = prog.comp(KC_EMB, 4 * b * h * M, deps=[mc])
+        pend = [dep]
+        prev = dep
+        for _ in range(nl):
+            for name, kc, work in fwd:
+                if name == "AR":
+                    if tp > 1:
+                        pend = [tp_ar(prev)]
+                    continue
+                prev = prog.comp(kc, work, deps=pend)
+                pend = []
+        if s == n_virtual - 1:
+            x = prog.comp(KC_NORM, 4 * b * h * M, deps=pend)
+            x = prog.comp(KC_GEMM, 2 * b * h * VOCAB / tp)
+            x = prog.comp(KC_LOSS, 4 * b * VOCAB / tp * M)
+            prog.memcpy(4, deps=[x])
+            prev = x
+        else:
+            xfer("fa", s, mb, True, deps=[prev])
+        act_out[(mb, ch)] = prev
+
+    def B(mb, ch):
+        s = ch * PP + p
+        last_mb = mb == m - 1
+        pend = [xfer("g", s, mb, False)] if s < n_virtual - 1 else []
+        if s == n_virtual - 1:
+            prog.comp(KC_LOSS, 4 * b * VOCAB / tp * M, deps=pend)
+            pend = []
+            prog.comp(KC_GEMM, 2 * b * h * VOCAB / tp)
+            g = prog.comp(KC_GEMM, 2 * b * h * VOCAB / tp)
+            add_grad(h * VOCAB / tp, g, last_mb)
+            prog.comp(KC_NORM, 6 * b * h * M)
+        prev = None
+        for _ in range(nl):
+            for name, kc, work, params in bwd:
+                if name == "AR":
+                    if tp > 1:
+                        pend = [tp_ar(prev)]
+                    continue
+                prev = prog.comp(kc, work, deps=pend)
+                pend = []
+                if params:
+                    add_grad(params, prev, last_mb)
+        if s == 0:
+            g = prog.comp(KC_EMB, 4 * b * h * M, deps=pend)
+            add_grad(VOCAB * h / tp, g, last_mb)
+            prev = g
+        else:
+            xfer("g", s - 1, mb, True, deps=[prev])
+        if last_mb:
+            flush_bucket(prev)
+
+    total = m * v
+
+    def mb_of(k):
+        return (k // n_virtual) * PP + k % PP
+
+    def chunk_of(k, forward):
+        ch = (k % n_virtual) // PP
+        return ch if forward else v - 1 - ch
+
+    warm = total if m == PP else min((PP - p - 1) * 2 + (v - 1) * PP, total)
+    kf = kb = 0
+    for _ in range(warm):
+        F(mb_of(kf), chunk_of(kf, True))
+        kf += 1
+    for _ in range(total - warm):
+        F(mb_of(kf), chunk_of(kf, True))
+        kf += 1
+        B(mb_of(kb), chunk_of(kb, False))
+        kb += 1
+    while kb < total:
+        B(mb_of(kb), chunk_of(kb, False))
+        kb += 1
+    gn = prog.comp(KC_ELEM, 4.0e5 * 20000.0, deps=dp_entries)
+    n_params = nl * v * 12 * h * h / tp
+    pend = [gn]
+    if c.tp * c.pp * c.dp > 1:
+        pend = [prog.comm(_E_WORLD, 4, CC_ALLREDUCE, ALGO_AUTO, None, deps=[gn])]
+    for _ in range(3):
+        prog.comp(KC_OPT, n_params * 16 / 3 * M, deps=pend)
+        pend = []
+    return prog
+
+
 def _rank(c: GPTConfig, dp: int, p: int, t: int) -> int:
     return (dp * c.pp + p) * c.tp + t
 
@@ -413,14 +561,16 @@ def build_gpt_graph(c: GPTConfig) -> Graph:
     """Build the merged multi-rank execution graph of one training step."""
     TP, PP, DP = c.tp, c.pp, c.dp
     R = TP * PP * DP
-    progs = [_stage_program(c, p) for p in range(PP)]
+    inter = c.virtual_stages > 1
+    NS = N_STREAMS + 3 if inter else N_STREAMS
+    progs = [(_stage_program_interleaved if inter else _stage_program)(c, p) for p in range(PP)]
 
     # P2P keys: every key must be issued by exactly the two adjacent stages
     p2p_keys: Dict[object, int] = {}
     p2p_seen: Dict[object, int] = {}
     for p, pr in enumerate(progs):
         for et, key in zip(pr.etype, pr.key):
-            if et == _E_P2P:
+            if et in _E_P2P_ALL:
                 if key not in p2p_keys:
                     p2p_keys[key] = len(p2p_keys)
                 p2p_seen[key] = p2p_seen.get(key, 0) + 1
@@ -456,7 +606,8 @@ def build_gpt_graph(c: GPTConfig) -> Graph:
     g_tp = 0
     n_tpg = DP * PP if TP > 1 else 0
     g_p2p = g_tp + n_tpg
-    n_p2pg = (PP - 1) * DP * TP
+    n_links = PP if inter else PP - 1  # interleaved: also the last stage -> the first
+    n_p2pg = n_links * DP * TP
     g_dp = g_p2p + n_p2pg
     n_dpg = PP * TP if DP > 1 else 0
     g_world = g_dp + n_dpg
@@ -466,10 +617,10 @@ def build_gpt_graph(c: GPTConfig) -> Graph:
         for p in range(PP):
             if TP > 1:
                 members.append(np.array([_rank(c, d, p, t) for t in range(TP)], np.int32))
-    for bb in range(PP - 1):
+    for bb in range(n_links):
         for d in range(DP):
             for t in range(TP):
-                members.append(np.array([_rank(c, d, bb, t), _rank(c, d, bb + 1, t)], np.int32))
+                members.append(np.array(sorted([_rank(c, d, bb, t), _rank(c, d, (bb + 1) % PP, t)]), np.int32))
     if DP > 1:
         for p in range(PP):
             for t in range(TP):
@@ -509,9 +660,8 @@ def build_gpt_graph(c: GPTConfig) -> Graph:
         ti = np.cumsum(tpm) - 1
         base[tpm] = tp_base[p] + ti[tpm] * DP
         mdp[tpm] = 1
-        p2m = et == _E_P2P
-        kidx = np.array([p2p_keys[k] if e == _E_P2P else 0 for e, k in zip(pr.etype, pr.key)],
-                        np.int64)
+        p2m = np.isin(et, _E_P2P_ALL)
+        kidx = np.array([p2p_keys[k] if e in _E_P2P_ALL else 0 for e, k in zip(pr.etype, pr.key)], np.int64)
         base[p2m] = p2p_base + kidx[p2m] * DP * TP
         mdp[p2m] = TP
         mtp[p2m] = 1
@@ -531,7 +681,7 @@ def build_gpt_graph(c: GPTConfig) -> Graph:
         alg = np.asarray(pr.algo, np.uint8)
         ekind = np.where(et == _E_COMP, KIND_COMPUTE,
                          np.where(et == _E_MEMCPY, KIND_MEMCPY,
-                                  np.where(et == _E_P2P, KIND_P2P, KIND_COLL))).astype(np.uint8)
+                                  np.where(p2m, KIND_P2P, KIND_COLL))).astype(np.uint8)
         flat = ids.reshape(-1)
         kind[flat] = np.tile(ekind, DP * TP)
         kclass[flat] = np.tile(kcl, DP * TP)
@@ -550,13 +700,16 @@ def build_gpt_graph(c: GPTConfig) -> Graph:
         group[ids[:, comm_mask].reshape(-1)] = grp[:, comm_mask].reshape(-1)
 
         # program order per stream
-        for stream, mask in ((STREAM_COMPUTE, et == _E_COMP), (STREAM_TP, tpm),
-                             (STREAM_PP, p2m), (STREAM_DP, dpm | wm),
-                             (STREAM_MEMCPY, et == _E_MEMCPY)):
+        lanes = ((STREAM_COMPUTE, et == _E_COMP), (STREAM_TP, tpm), (STREAM_PP, et == _E_P2P),
+                 (STREAM_DP, dpm | wm), (STREAM_MEMCPY, et == _E_MEMCPY))
+        if inter:
+            lanes += ((STREAM_PP_RECV, et == _E_P2P_RECV), (STREAM_PP_GRAD, et == _E_P2P_GRAD),
+                      (STREAM_PP_GRAD_RECV, et == _E_P2P_GRAD_RECV))
+        for stream, mask in lanes:
             sel = ids[:, mask]
             for j in range(DP * TP):
                 r = _rank(c, int(dpv[j]), p, int(tpv[j]))
-                queues[r * N_STREAMS + stream] = sel[j]
+                queues[r * NS + stream] = sel[j]
         # data edges
         if pr.src:
             s_e = np.asarray(pr.src, np.int64)
@@ -564,7 +717,7 @@ def build_gpt_graph(c: GPTConfig) -> Graph:
             srcs.append(ids[:, s_e].reshape(-1))
             dsts.append(ids[:, d_e].reshape(-1))
 
-    nq = R * N_STREAMS
+    nq = R * NS
     q_lens = [len(queues.get(q, ())) for q in range(nq)]
     q_off = np.zeros(nq + 1, np.int64)
     q_off[1:] = np.cumsum(q_lens)
@@ -588,12 +741,12 @@ def build_gpt_graph(c: GPTConfig) -> Graph:
         replica_of = (np.arange(R) % (PP * TP)).astype(np.int32)
         orig = np.arange(V)
         for q in range(nq):
-            r, k = divmod(q, N_STREAMS)
-            qa = int(replica_of[r]) * N_STREAMS + k
+            r, k = divmod(q, NS)
+            qa = int(replica_of[r]) * NS + k
             if qa != q:
                 orig[q_ops[q_off[q]:q_off[q + 1]]] = q_ops[q_off[qa]:q_off[qa + 1]]
         noise = noise[orig]
-    g = Graph(R, N_STREAMS, c.gpus_per_node, kind, kclass, group, cc_type, cc_algo, cc_bytes,
+    g = Graph(R, NS, c.gpus_per_node, kind, kclass, group, cc_type, cc_algo, cc_bytes,
               pred_off, pred_idx, q_off, q_ops, grp_off, grp_rank.astype(np.int32), work, noise,
               name=c.name, replica_of=replica_of)
     return g
