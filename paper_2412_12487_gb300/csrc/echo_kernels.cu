@@ -233,8 +233,13 @@ constexpr int kOverlapThreads = 128;
 constexpr int kOverlapBatch = 8;  // divides 32 (the shuffled op list's width)
 // LAUNCH: a comm op's interval on the rank opens at the rank's launch of it
 // (a.lq_off), else at its start.  PROP: the proportional slowdown model (a.model 1)
+// Blocks per SM the register budget allows.  Occupancy hides the row-load latency
+// (at 3 comm timelines, 64 registers beat 108 by 12%); wide cursor sets keep their
+// registers instead of spilling.
+constexpr int overlap_min_blocks(int ncmax) { return ncmax <= 3 ? 8 : ncmax <= 4 ? 6 : 1; }
+
 template <int NCMAX, bool LAUNCH, bool PROP>
-__global__ void __launch_bounds__(kOverlapThreads, 8) overlap_kernel(OverlapArgs a) {  // 64 registers: occupancy hides its row-load latency
+__global__ void __launch_bounds__(kOverlapThreads, overlap_min_blocks(NCMAX)) overlap_kernel(OverlapArgs a) {
   const int32_t S = a.S;
   const int32_t s = blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t c = blockIdx.y + (int64_t)gridDim.y * blockIdx.z;
@@ -304,6 +309,7 @@ __global__ void __launch_bounds__(kOverlapThreads, 8) overlap_kernel(OverlapArgs
       }
     }
   }
+
   // groups of kOverlapBatch ops: their finish times and durations are loaded together
   for (int64_t i0 = c0; i0 < c1; i0 += kOverlapBatch) {
     if (i0 > c0 && ((i0 - c0) & 31) == 0) {
@@ -555,6 +561,8 @@ cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
       overlap_kernel<3, L, P><<<grid, tx, 0, st>>>(a);
     else if (a.n_cq <= 4)
       overlap_kernel<4, L, P><<<grid, tx, 0, st>>>(a);
+    else if (a.n_cq <= 6)
+      overlap_kernel<6, L, P><<<grid, tx, 0, st>>>(a);
     else if (a.n_cq <= 8)
       overlap_kernel<8, L, P><<<grid, tx, 0, st>>>(a);
     else
