@@ -231,13 +231,13 @@ __global__ void permute_rows_kernel(const T *__restrict__ raw, const int32_t *__
 // ---------------------------------------------------------------------------------
 constexpr int kOverlapThreads = 128;
 constexpr int kOverlapBatch = 8;  // divides 32 (the shuffled op list's width)
-// LAUNCH: a comm op's interval on the rank opens at the rank's launch of it
-// (a.lq_off), else at its start.  PROP: the proportional slowdown model (a.model 1)
 // Blocks per SM the register budget allows.  Occupancy hides the row-load latency
 // (at 3 comm timelines, 64 registers beat 108 by 12%); wide cursor sets keep their
 // registers instead of spilling.
 constexpr int overlap_min_blocks(int ncmax) { return ncmax <= 3 ? 8 : ncmax <= 4 ? 6 : 1; }
 
+// LAUNCH: a comm op's interval on the rank opens at the rank's launch of it
+// (a.lq_off), else at its start.  PROP: the proportional slowdown model (a.model 1)
 template <int NCMAX, bool LAUNCH, bool PROP>
 __global__ void __launch_bounds__(kOverlapThreads, overlap_min_blocks(NCMAX)) overlap_kernel(OverlapArgs a) {
   const int32_t S = a.S;
@@ -309,7 +309,6 @@ __global__ void __launch_bounds__(kOverlapThreads, overlap_min_blocks(NCMAX)) ov
       }
     }
   }
-
   // groups of kOverlapBatch ops: their finish times and durations are loaded together
   for (int64_t i0 = c0; i0 < c1; i0 += kOverlapBatch) {
     if (i0 > c0 && ((i0 - c0) & 31) == 0) {
