@@ -210,16 +210,21 @@ void build_dataflow(GraphBuild &b) {
   b.df_rec.clear();
   b.df_opnd.clear();
   if (V >= (int64_t)(echo::kDfPayload + 1u)) return;
-  // ranks of each op, ascending
+  // ranks of each op, ascending, with the op's timeline on each
   std::vector<int64_t> ro_off(V + 1, 0);
   for (int64_t q = 0; q < (int64_t)R * NS; ++q)
     for (int64_t i = b.q_off[q]; i < b.q_off[q + 1]; ++i) ro_off[b.q_ops_int[i] + 1]++;
   for (int64_t v = 0; v < V; ++v) ro_off[v + 1] += ro_off[v];
   std::vector<int32_t> ro(std::max<int64_t>(ro_off[V], 1));
+  std::vector<int8_t> rt(ro.size());
   {
     std::vector<int64_t> fill(ro_off.begin(), ro_off.end() - 1);
     for (int64_t q = 0; q < (int64_t)R * NS; ++q)
-      for (int64_t i = b.q_off[q]; i < b.q_off[q + 1]; ++i) ro[fill[b.q_ops_int[i]]++] = (int32_t)(q / NS);
+      for (int64_t i = b.q_off[q]; i < b.q_off[q + 1]; ++i) {
+        const int64_t at = fill[b.q_ops_int[i]]++;
+        ro[at] = (int32_t)(q / NS);
+        rt[at] = (int8_t)(q % NS);
+      }
   }
   auto runs_on = [&](int32_t u, int32_t r) {
     return std::binary_search(ro.data() + ro_off[u], ro.data() + ro_off[u + 1], r);
@@ -256,32 +261,35 @@ void build_dataflow(GraphBuild &b) {
     }
   }
   if (b.df_exports >= (int64_t)(echo::kDfPayload + 1u)) return;
-  // the programs
-  std::vector<std::pair<int32_t, int32_t>> ops;  // (node, timeline) of the rank
-  std::vector<int8_t> tl(V, -1);
-  std::vector<int32_t> last(NS);
+  // the programs, written in one pass over the ops in internal order (each rank's
+  // entries land in its own range, in that order); per rank only the latest op of
+  // each timeline and the previous op are kept
+  for (int32_t r = 0; r < R; ++r) b.df_off[r + 1] = b.df_off[r] + (b.q_off[(int64_t)(r + 1) * NS] - b.q_off[(int64_t)r * NS]);
+  b.df_rec.assign((size_t)b.df_off[R] * 8, 0u);
+  std::vector<int64_t> cnt(R, 0);
+  std::vector<int32_t> last((size_t)R * NS, -1), prev(R, -1);
+  std::vector<int8_t> prev_tl(R, 0);
   std::vector<uint32_t> extra;
-  for (int32_t r = 0; r < R; ++r) {
-    ops.clear();
-    for (int32_t k = 0; k < NS; ++k)
-      for (int64_t i = b.q_off[(int64_t)r * NS + k]; i < b.q_off[(int64_t)r * NS + k + 1]; ++i) {
-        ops.emplace_back(b.q_ops_int[i], k);
-        tl[b.q_ops_int[i]] = (int8_t)k;
-      }
-    std::sort(ops.begin(), ops.end());
-    std::fill(last.begin(), last.end(), -1);
-    int32_t prev = -1;  // the op before it in the program
-    for (auto [v, k] : ops) {
+  auto timeline_on = [&](int32_t u, int32_t r) -> int {  // u's timeline on rank r, -1 if none
+    const int32_t *lo = ro.data() + ro_off[u], *hi = ro.data() + ro_off[u + 1];
+    const int32_t *p = std::lower_bound(lo, hi, r);
+    return p != hi && *p == r ? rt[p - ro.data()] : -1;
+  };
+  for (int64_t v = 0; v < V; ++v) {
+    const bool comm = b.is_comm[v];
+    const int64_t nm = members((int32_t)v);
+    for (int64_t j = ro_off[v]; j < ro_off[v + 1]; ++j) {
+      const int32_t r = ro[j], k = rt[j];
+      const int64_t me = j - ro_off[v];
+      int32_t *lr = last.data() + (size_t)r * NS;
       extra.clear();
-      uint32_t regs = last[k] >= 0 ? 1u << k : 0u;  // the op before it on its timeline
-      const bool comm = b.is_comm[v];
-      const int64_t nm = members(v);
-      const int64_t me = comm ? std::lower_bound(ro.data() + ro_off[v], ro.data() + ro_off[v + 1], r) - (ro.data() + ro_off[v]) : 0;
+      uint32_t regs = lr[k] >= 0 ? 1u << k : 0u;  // the op before it on its timeline
       for (int64_t e = b.dp_off[v]; e < b.dp_off[v + 1]; ++e) {
         const int32_t u = b.dp[e];
-        if (tl[u] >= 0) {  // runs on this rank
-          if (last[tl[u]] == u)
-            regs |= 1u << tl[u];
+        const int ku = timeline_on(u, r);
+        if (ku >= 0) {  // runs on this rank
+          if (lr[ku] == u)
+            regs |= 1u << ku;
           else
             extra.push_back((echo::kDfInLocal << 30) | (uint32_t)u);
         } else if (comm ? (uncovered[e] && me == 0) : true) {
@@ -290,9 +298,9 @@ void build_dataflow(GraphBuild &b) {
       }
       // the previous op of the program, when an input, comes from a register
       bool use_prev = false;
-      if (prev >= 0 && ((regs >> tl[prev]) & 1) && last[tl[prev]] == prev) {
+      if (prev[r] >= 0 && ((regs >> prev_tl[r]) & 1) && lr[prev_tl[r]] == prev[r]) {
         use_prev = true;
-        regs &= ~(1u << tl[prev]);
+        regs &= ~(1u << prev_tl[r]);
       }
       const bool two_hop = comm && nm > (int64_t)echo::kDfDirectMembers;
       const bool publish = exp_id[v] >= 0 && (!comm || me == 0);
@@ -300,20 +308,20 @@ void build_dataflow(GraphBuild &b) {
       const uint32_t hdr = (uint32_t)k | (comm ? echo::kDfComm : 0u) | (publish ? echo::kDfExport : 0u) |
                            (two_hop ? echo::kDfTwoHop : 0u) | (use_prev ? echo::kDfPrev : 0u) |
                            ((uint32_t)extra.size() << 8) | (regs << 16);
-      b.df_rec.push_back((uint32_t)v);
-      b.df_rec.push_back(b.cidx[v] >= 0 ? (uint32_t)b.cidx[v] : ~0u);
-      b.df_rec.push_back(hdr);
-      b.df_rec.push_back((uint32_t)b.df_opnd.size());
-      b.df_rec.push_back(comm ? (uint32_t)slot[v] : 0u);
-      b.df_rec.push_back(comm ? (uint32_t)nm | ((uint32_t)me << 16) : 0u);
-      b.df_rec.push_back(publish || two_hop ? (uint32_t)exp_id[v] : 0u);
-      b.df_rec.push_back(0u);
+      uint32_t *w = b.df_rec.data() + (size_t)(b.df_off[r] + cnt[r]++) * 8;
+      w[0] = (uint32_t)v;
+      w[1] = b.cidx[v] >= 0 ? (uint32_t)b.cidx[v] : ~0u;
+      w[2] = hdr;
+      w[3] = (uint32_t)b.df_opnd.size();
+      w[4] = comm ? (uint32_t)slot[v] : 0u;
+      w[5] = comm ? (uint32_t)nm | ((uint32_t)me << 16) : 0u;
+      w[6] = publish || two_hop ? (uint32_t)exp_id[v] : 0u;
+      w[7] = 0u;
       b.df_opnd.insert(b.df_opnd.end(), extra.begin(), extra.end());
-      last[k] = v;
-      prev = v;
+      lr[k] = (int32_t)v;
+      prev[r] = (int32_t)v;
+      prev_tl[r] = (int8_t)k;
     }
-    for (auto [v, k] : ops) tl[v] = -1;
-    b.df_off[r + 1] = (int64_t)b.df_rec.size() / 8;
   }
   if (b.df_slots >= (int64_t)UINT32_MAX) return;
   if (b.df_rec.empty()) b.df_rec.assign(8, 0);
