@@ -118,3 +118,17 @@ def test_hand_built_pair():
     assert E.check_replicas(_pair()) == 2  # a0 and the all-reduce
     _rejected(_pair(mirror_launch=False))  # rank 1 would launch at 0, rank 0 after a0
     _rejected(_pair(extra=True))           # timelines of different lengths
+
+
+def test_folding_interleaved_schedules():
+    # 8 timelines per rank and lone transfers between virtual stages: replicas of a
+    # DP group still mirror each other, and the oracle composes them symmetrically
+    c = W.GPTConfig("i-L8-pp2-m2-v2-dp2", 8, 512, 8, 256, 2, 2, 2, 2, 3, virtual_stages=2,
+                    identical_replicas=True)
+    g = W.build_gpt_graph(c)
+    assert g.n_streams == 8
+    orig = originals(g)
+    assert E.check_replicas(g) == len(np.unique(orig)) < g.n_ops
+    sc = W.make_scenarios(g, c)
+    r = oracle.compose(g, sc, refine_passes=1, comm_interval=1)
+    assert np.array_equal(r.finish, r.finish[orig]) and np.array_equal(r.overlapped, r.overlapped[orig])
