@@ -24,6 +24,7 @@ import re
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -55,7 +56,7 @@ class Clocks:
     def __init__(self, index=None):
         self.index = index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+        self.path = os.path.join(tempfile.gettempdir(), f"echo_bench_clocks_{os.getpid()}.csv")
 
     def start(self):
         try:
