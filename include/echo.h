@@ -51,7 +51,7 @@ typedef enum {
   ECHO_E_CUDA = 6,        /* a CUDA runtime call failed                                */
   ECHO_E_TIMEOUT = 7,     /* a bounded device-side wait gave up                        */
   ECHO_E_OVERFLOW = 8,    /* a finish time could exceed the int64 range                */
-  ECHO_E_UNSUPPORTED = 9  /* a size beyond what this build supports                    */
+  ECHO_E_UNSUPPORTED = 9  /* a size beyond what the library supports                   */
 } echo_status;
 
 /* op kinds (Sec. 4.2 timelines: computation, communication, memcpy) */
