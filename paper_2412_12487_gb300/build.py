@@ -1,7 +1,8 @@
 """Build ``libecho.so`` in-tree with nvcc for sm_103a (GB300).
 
-The three translation units compile in parallel and link into one shared library
-exporting the C ABI of ``include/echo.h``.
+The translation units compile in parallel and link into one shared library
+exporting the C ABI of ``include/echo.h``.  The overlap test compiles once per
+variant family (launch interval x proportional model), four objects in parallel.
 """
 from __future__ import annotations
 
@@ -17,7 +18,11 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libecho.so")
 BUILD_DIR = os.path.join(PKG, "_build")
-SOURCES = ["echo_kernels.cu", "echo_compose.cu", "echo_dataflow.cu", "echo_host.cpp"]
+# (source, extra nvcc flags, object)
+UNITS = [(f, [], f + ".o") for f in ("echo_kernels.cu", "echo_compose.cu", "echo_dataflow.cu", "echo_host.cpp")] + [
+    ("echo_overlap.cu", [f"-DECHO_OV_LAUNCH={l}", f"-DECHO_OV_PROP={p}"], f"echo_overlap_l{l}_p{p}.o")
+    for l in (0, 1) for p in (0, 1)]
+SOURCES = sorted({u[0] for u in UNITS})
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -48,9 +53,10 @@ def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) 
     os.makedirs(BUILD_DIR, exist_ok=True)
     exe = nvcc()
 
-    def compile_one(src):
-        obj = os.path.join(BUILD_DIR, src + ".o")
-        cmd = [exe] + _flags() + (["-Xptxas", "-v"] if ptxas_info and src.endswith(".cu") else []) + \
+    def compile_one(unit):
+        src, extra, obj_name = unit
+        obj = os.path.join(BUILD_DIR, obj_name)
+        cmd = [exe] + _flags() + extra + (["-Xptxas", "-v"] if ptxas_info and src.endswith(".cu") else []) + \
             ["-c", os.path.join(CSRC, src), "-o", obj]
         if src.endswith(".cpp"):
             cmd[1:1] = ["-x", "cu"]
@@ -61,8 +67,8 @@ def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) 
             sys.stderr.write(r.stdout + r.stderr)
         return obj
 
-    with ThreadPoolExecutor(len(SOURCES)) as ex:
-        objs = list(ex.map(compile_one, SOURCES))
+    with ThreadPoolExecutor(len(UNITS)) as ex:
+        objs = list(ex.map(compile_one, UNITS))
     tmp = LIB + f".{os.getpid()}.tmp"
     r = subprocess.run([exe] + ARCH + ["-shared", "-o", tmp] + objs, capture_output=True, text=True)
     if r.returncode != 0:

@@ -15,6 +15,7 @@ constexpr int kMetaChunk = 128;            // segment levels of metadata staged 
 constexpr int kMetaCap = 136;              // metadata entries per staging buffer (>= kMetaChunk + 1)
 constexpr uint32_t kFarRef = 0x80000000u;  // predecessor reference read from global memory
 constexpr int kOverlapChunk = 128;         // compute ops per overlap-test thread
+constexpr int kOverlapThreads = 128;       // threads per block of the overlap test
 constexpr int kMaxSegment = 64;            // longest serial chain composed as one segment
 constexpr int kPipeStages = 16;            // stages (mbarrier pairs) of the pipelined compose
 constexpr int kPipeConsumerWarps = 16;     // composing warps of the pipelined compose
@@ -199,6 +200,13 @@ cudaError_t launch_compose_dataflow(const DataflowArgs &a, cudaStream_t st);
 size_t dataflow_smem_bytes(int32_t n_streams);
 // whether every warp of R * G warps can be resident at once (cooperative launch)
 bool dataflow_fits(int64_t n_warps, int32_t n_streams, int device);
+
+// overlap.cu: the overlap test, one entry point per (launch interval, proportional
+// model) pair, each dispatching on the number of comm timelines
+cudaError_t launch_overlap_l0_p0(const OverlapArgs &a, dim3 grid, int tx, cudaStream_t st);
+cudaError_t launch_overlap_l0_p1(const OverlapArgs &a, dim3 grid, int tx, cudaStream_t st);
+cudaError_t launch_overlap_l1_p0(const OverlapArgs &a, dim3 grid, int tx, cudaStream_t st);
+cudaError_t launch_overlap_l1_p1(const OverlapArgs &a, dim3 grid, int tx, cudaStream_t st);
 
 // kernels.cu
 cudaError_t launch_cc_estimate(const CcSig *sig, int32_t G, ScenParams p, int32_t S,
