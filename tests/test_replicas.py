@@ -132,3 +132,72 @@ def test_folding_interleaved_schedules():
     sc = W.make_scenarios(g, c)
     r = oracle.compose(g, sc, refine_passes=1, comm_interval=1)
     assert np.array_equal(r.finish, r.finish[orig]) and np.array_equal(r.overlapped, r.overlapped[orig])
+
+
+def _replicate(rng, g0, sc0):
+    """Two replicas of random graph g0 (ranks r and r + H, H = R0 rounded up to whole
+    nodes, so that every copied group spans the same node layout).  Some collectives become
+    one op shared by both replicas (members of both copies, producers of both), the
+    rest are copied.  Returns the graph with replica_of, its scenarios, and for each
+    op of g0 its (replica 0, replica 1) ids."""
+    R0, NS, V0 = g0.n_ranks, g0.n_streams, g0.n_ops
+    H = -(-R0 // g0.gpus_per_node) * g0.gpus_per_node
+    comm = (g0.kind == W.KIND_COLL)
+    shared = comm & (rng.random(V0) < 0.5)
+    ids = np.zeros((V0, 2), np.int64)
+    ops = []
+    for v in range(V0):
+        base = {"kind": int(g0.kind[v]), "kclass": int(g0.kclass[v]), "cc_type": int(g0.cc_type[v]),
+                "cc_algo": int(g0.cc_algo[v]), "cc_bytes": int(g0.cc_bytes[v])}
+        for rep in ((0,) if shared[v] else (0, 1)):
+            ids[v, rep] = len(ops)
+            ops.append(dict(base, rep=rep, orig=v))
+        if shared[v]:
+            ids[v, 1] = ids[v, 0]
+    groups, gmap = [], {}
+    for o in ops:
+        v = o["orig"]
+        if g0.kind[v] in (W.KIND_COLL, W.KIND_P2P):
+            mem = g0.grp_rank[g0.grp_off[g0.group[v]]:g0.grp_off[g0.group[v] + 1]].tolist()
+            m = sorted(mem + [x + H for x in mem]) if shared[v] else sorted(x + H * o["rep"] for x in mem)
+            o["group"] = gmap.setdefault(tuple(m), len(groups))
+            if o["group"] == len(groups):
+                groups.append(m)
+        preds = g0.pred_idx[g0.pred_off[v]:g0.pred_off[v + 1]].tolist()
+        reps = (0, 1) if shared[v] else (o["rep"],)
+        o["preds"] = sorted({int(ids[u, rp]) for u in preds for rp in reps})
+    queues = {}
+    for q in range(R0 * NS):
+        r, k = divmod(q, NS)
+        lst = g0.q_ops[g0.q_off[q]:g0.q_off[q + 1]].tolist()
+        queues[(r, k)] = [int(ids[v, 0]) for v in lst]
+        queues[(r + H, k)] = [int(ids[v, 1]) for v in lst]
+    g = SG.graph_from_lists(2 * H, NS, ops, queues, groups, gpus_per_node=g0.gpus_per_node)
+    g.replica_of = np.concatenate([np.arange(H), np.arange(R0), np.arange(R0, H)]).astype(np.int32)
+    dur = np.zeros((len(ops), sc0.n_scen), np.int64)
+    for v in range(V0):
+        dur[ids[v, 0]] = sc0.dur[v]
+        dur[ids[v, 1]] = sc0.dur[v]
+    sc = W.Scenarios(dur=dur, alpha_ns=sc0.alpha_ns, bw_intra=sc0.bw_intra, lat_intra=sc0.lat_intra,
+                     bw_inter=sc0.bw_inter, lat_inter=sc0.lat_inter, delta=sc0.delta,
+                     slowdown=sc0.slowdown, peak_flop_per_ns=sc0.peak_flop_per_ns)
+    return g, sc, ids
+
+
+def test_folding_random_replicated_graphs():
+    # random graphs in two replicas, some collectives shared by both: the host check
+    # folds them back to the original op count, and the oracle's composition of the
+    # full graph gives every copy its original's times
+    rng = np.random.default_rng(808)
+    folded = 0
+    for case in range(60):
+        g0 = SG.random_graph(rng, int(rng.integers(2, 40)), max_ranks=3, max_streams=4, p_edge=0.1)
+        sc0 = SG.random_scenarios(rng, g0, 3, max_dur=40)
+        g, sc, ids = _replicate(rng, g0, sc0)
+        assert E.check_replicas(g) == g0.n_ops, case
+        folded += g.n_ops > g0.n_ops
+        for civ in (0, 1):
+            r = oracle.compose(g, sc, refine_passes=2, comm_interval=civ)
+            assert np.array_equal(r.finish[ids[:, 0]], r.finish[ids[:, 1]]), case
+            assert np.array_equal(r.overlapped[ids[:, 0]], r.overlapped[ids[:, 1]]), case
+    assert folded > 40
