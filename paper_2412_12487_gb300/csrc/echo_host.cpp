@@ -1449,7 +1449,12 @@ int activate_fold(echo_ctx *c, bool want) {
   c->fold_active = want;
   free_all(c->scen_allocs);
   c->scen_vs = 0;
-  return upload_graph(c);
+  const int rc = upload_graph(c);
+  if (rc) {  // no device graph any more: the graph must be loaded again
+    c->state = 0;
+    c->fold_ok = false;
+  }
+  return rc;
 }
 
 }  // namespace
