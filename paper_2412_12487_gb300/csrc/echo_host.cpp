@@ -330,9 +330,11 @@ void build_dataflow(GraphBuild &b) {
 }
 
 // `shape`, when given, replaces the (N, M, K) of every group computed from its
-// members (a folded graph keeps the shapes of the caller's groups).
+// members (a folded graph keeps the shapes of the caller's groups).  `programs`:
+// also build the dataflow composer's programs (not needed to validate a graph).
 using Shape = std::array<int32_t, 3>;
-int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e, const std::vector<Shape> *shape = nullptr) {
+int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e, const std::vector<Shape> *shape = nullptr,
+                bool programs = true) {
   if (!g) return fail(e, ECHO_E_INVALID_ARG, "graph descriptor is NULL");
   const int64_t V = g->n_ops;
   if (V < 0 || V >= INT32_MAX) return fail(e, ECHO_E_INVALID_ARG, "n_ops %lld out of range", (long long)V);
@@ -783,7 +785,7 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e, const std::vect
           return fail(e, ECHO_E_BAD_GRAPH, "internal: segment %lld reads level %d from level %d", (long long)t,
                       lvl[b.seg_int[b.hin[q]]], lvl[t]);
   }
-  build_dataflow(b);
+  if (programs) build_dataflow(b);
   return ECHO_OK;
 }
 
@@ -1024,13 +1026,13 @@ int build_fold(const echo_graph_desc *g, const int32_t *replica_of, Fold &F, Err
 // The folded graph of `g` when its replica_of marks replicas: `fb` composes it,
 // with int2ext / ext2int / V_ext in the caller's ids.  Returns ECHO_OK with
 // *folded = false when there is nothing to fold.
-int build_folded(const echo_graph_desc *g, GraphBuild &fb, Fold &F, bool *folded, Err &e) {
+int build_folded(const echo_graph_desc *g, GraphBuild &fb, Fold &F, bool *folded, Err &e, bool programs = true) {
   *folded = false;
   if (!g->replica_of) return ECHO_OK;
   int rc = build_fold(g, g->replica_of, F, e);
   if (rc || F.keep.empty()) return rc;
   Err e2;
-  rc = build_graph(&F.desc, fb, e2, &F.shape);
+  rc = build_graph(&F.desc, fb, e2, &F.shape, programs);
   if (rc) return fail(e, ECHO_E_BAD_GRAPH, "replica_of: the folded graph is not valid (%s)", e2.msg.c_str());
   for (auto &x : fb.int2ext) x = F.keep[x];
   std::vector<int32_t> e2i(g->n_ops);
@@ -1553,7 +1555,7 @@ int echo_destroy(echo_ctx *c) {
 int echo_check_graph(const echo_graph_desc *g, int64_t *n_levels, int64_t *max_width) {
   GraphBuild b;
   Err e;
-  int rc = build_graph(g, b, e);
+  int rc = build_graph(g, b, e, nullptr, false);
   if (rc) return rc;
   if (n_levels) *n_levels = b.L;
   if (max_width) *max_width = b.max_width;
@@ -1565,8 +1567,8 @@ int echo_check_replicas(const echo_graph_desc *g, int64_t *n_ops_folded) {
   Fold F;
   Err e;
   bool folded = false;
-  int rc = build_graph(g, b, e);
-  if (!rc) rc = build_folded(g, fb, F, &folded, e);
+  int rc = build_graph(g, b, e, nullptr, false);
+  if (!rc) rc = build_folded(g, fb, F, &folded, e, false);
   if (rc) return rc;
   if (n_ops_folded) *n_ops_folded = folded ? fb.V : b.V;
   return ECHO_OK;
