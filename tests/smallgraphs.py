@@ -176,11 +176,20 @@ def launch_preds(g: W.Graph):
     return out
 
 
-def brute_compose(g: W.Graph, sc: W.Scenarios, s: int, refine_passes: int, cc_fn, comm_interval: int = 0):
+def covered_length(pieces):
+    """Length of the union of half-open intervals, by coordinate compression."""
+    xs = sorted({x for p in pieces for x in p})
+    return sum(b - a for a, b in zip(xs, xs[1:]) if any(lo <= a and b <= hi for lo, hi in pieces))
+
+
+def brute_compose(g: W.Graph, sc: W.Scenarios, s: int, refine_passes: int, cc_fn, comm_interval: int = 0,
+                  overlap_model: int = 0):
     """Brute-force reference of one scenario: CC durations from ``cc_fn`` (pinned on
     its own), composition by path enumeration, overlap by checking every pair.  A
     comm op's interval on rank r starts at its start (comm_interval 0) or when r
-    has launched it (1: the latest finish among ``launch_preds``)."""
+    has launched it (1: the latest finish among ``launch_preds``).  An overlapped
+    kernel takes rint(d * f) (overlap_model 0) or rint(d + (f - 1) * covered
+    length) (1)."""
     V = g.n_ops
     d0 = np.zeros(V, np.int64)
     for v in range(V):
@@ -199,19 +208,26 @@ def brute_compose(g: W.Graph, sc: W.Scenarios, s: int, refine_passes: int, cc_fn
     ov = np.zeros(V, np.uint8)
     for _ in range(refine_passes):
         st = fin - d
+        covered = np.zeros(V, np.int64)
         for v in range(V):
             if g.kind[v] != W.KIND_COMPUTE:
                 continue
-            hit = 0
+            pieces = []
             for w in range(V):
                 for r in ranks[v] & ranks[w] if g.kind[w] in (W.KIND_COLL, W.KIND_P2P) else ():
                     lo = st[w] if comm_interval == 0 else max([0] + [int(fin[u]) for u in lp[(w, r)]])
-                    if max(st[v], lo) < min(fin[v], fin[w]):
-                        hit = 1
-            ov[v] = hit
+                    a, b = max(int(st[v]), int(lo)), min(int(fin[v]), int(fin[w]))
+                    if a < b:
+                        pieces.append((a, b))
+            ov[v] = 1 if pieces else 0
+            covered[v] = covered_length(pieces)
         d = d0.copy()
         for v in range(V):
             if g.kind[v] == W.KIND_COMPUTE and ov[v]:
-                d[v] = int(np.rint(float(d0[v]) * sc.slowdown[g.kclass[v], s]))
+                f = float(sc.slowdown[g.kclass[v], s])
+                if overlap_model == 1:
+                    d[v] = int(np.rint(float(d0[v]) + (f - 1.0) * float(covered[v])))
+                else:
+                    d[v] = int(np.rint(float(d0[v]) * f))
         fin = brute_finish(g, d)
     return fin - d, fin, ov

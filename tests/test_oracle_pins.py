@@ -358,6 +358,33 @@ def test_brute_force_launch_intervals(seed):
                 assert (r.overlapped[:, s] == ov).all(), (seed, case, passes)
 
 
+@pytest.mark.parametrize("seed", range(3))
+def test_brute_force_proportional_slowdown(seed):
+    # the proportional model against a pair-by-pair brute force whose covered
+    # length comes from coordinate compression, with either comm interval
+    # sparse graphs with several comm timelines, so that kernels often run under
+    # two concurrent comm ops (where the union differs from the sum)
+    rng = np.random.default_rng(3000 + seed)
+    for case in range(150):
+        g = SG.random_graph(rng, int(rng.integers(4, 26)), max_ranks=2, max_streams=5, p_edge=0.04,
+                            min_streams=3)
+        sc = SG.random_scenarios(rng, g, 2)
+        for passes, civ in ((1, 0), (2, 1), (1, 1)):
+            r = oracle.compose(g, sc, refine_passes=passes, overlap_model=1, comm_interval=civ)
+            for s in range(sc.n_scen):
+                st, fn, ov = SG.brute_compose(g, sc, s, passes, oracle.cc_ns, comm_interval=civ, overlap_model=1)
+                assert (r.finish[:, s] == fn).all(), (seed, case, passes, civ)
+                assert (r.overlapped[:, s] == ov).all(), (seed, case, passes, civ)
+
+
+def test_covered_length_helper():
+    # the brute force's own union length, by hand
+    assert SG.covered_length([]) == 0
+    assert SG.covered_length([(0, 10), (5, 15)]) == 15
+    assert SG.covered_length([(0, 2), (4, 6), (1, 5)]) == 6
+    assert SG.covered_length([(3, 4), (3, 4)]) == 1
+
+
 def test_auto_takes_the_faster_algorithm():
     rng = np.random.default_rng(13)
     for _ in range(300):
