@@ -183,6 +183,14 @@ int echo_destroy(echo_ctx *ctx);
  * the widest level (either pointer may be NULL). */
 int echo_check_graph(const echo_graph_desc *g, int64_t *n_levels, int64_t *max_width);
 
+/* Host-only overlap candidates (Sec. 3's validator tests only these): flags[v] = 1
+ * for every compute op v (caller ids) that can overlap a comm op of its rank in
+ * some scenario, judged from the issue order and data edges among the rank's own
+ * ops (an op that must finish before the comm op starts, or start after it ends,
+ * never overlaps it).  flags: [n_ops] host buffer, or NULL; *n_candidates their
+ * count, or NULL.  Errors as echo_check_graph. */
+int echo_overlap_candidates(const echo_graph_desc *g, uint8_t *flags, int64_t *n_candidates);
+
 /* Host-only check of a graph with replica_of: the validation echo_load_graph
  * performs, and the number of ops the folded graph composes (n_ops when
  * replica_of is NULL or marks no replica).  Errors as echo_load_graph. */

@@ -1574,6 +1574,17 @@ int echo_check_replicas(const echo_graph_desc *g, int64_t *n_ops_folded) {
   return ECHO_OK;
 }
 
+int echo_overlap_candidates(const echo_graph_desc *g, uint8_t *flags, int64_t *n_candidates) {
+  GraphBuild b;
+  Err e;
+  const int rc = build_graph(g, b, e, nullptr, false);
+  if (rc) return rc;
+  if (flags)
+    for (int64_t v = 0; v < b.V; ++v) flags[v] = b.cand_flag[b.ext2int[v]];
+  if (n_candidates) *n_candidates = b.n_cand;
+  return ECHO_OK;
+}
+
 int echo_load_graph(echo_ctx *c, const echo_graph_desc *g) {
   int rc = check_ctx(c);
   if (rc) return rc;

@@ -20,7 +20,7 @@ STATUS_NAMES = {0: "ECHO_OK", 1: "ECHO_E_INVALID_ARG", 2: "ECHO_E_BAD_GRAPH", 3:
                 8: "ECHO_E_OVERFLOW", 9: "ECHO_E_UNSUPPORTED"}
 
 # every function the header declares (checked by the tests)
-EXPORTS = ["echo_create", "echo_destroy", "echo_check_graph", "echo_check_replicas", "echo_load_graph", "echo_load_scenarios",
+EXPORTS = ["echo_create", "echo_destroy", "echo_check_graph", "echo_check_replicas", "echo_overlap_candidates", "echo_load_graph", "echo_load_scenarios",
            "echo_estimate_collectives", "echo_compose", "echo_read_times", "echo_read_makespan",
            "echo_read_cc", "echo_read_overlap", "echo_cc_query", "echo_cc_query_noalloc",
            "echo_graph_info_get", "echo_set_cc_model",
@@ -105,6 +105,7 @@ def load_library(path: Optional[str] = None):
         "echo_destroy": ([vp], C.c_int),
         "echo_check_graph": ([C.POINTER(GraphDesc), C.POINTER(i64), C.POINTER(i64)], C.c_int),
         "echo_check_replicas": ([C.POINTER(GraphDesc), C.POINTER(i64)], C.c_int),
+        "echo_overlap_candidates": ([C.POINTER(GraphDesc), vp, C.POINTER(i64)], C.c_int),
         "echo_load_graph": ([vp, C.POINTER(GraphDesc)], C.c_int),
         "echo_load_scenarios": ([vp, C.POINTER(ScenDesc)], C.c_int),
         "echo_estimate_collectives": ([vp], C.c_int),
@@ -183,6 +184,21 @@ def check_replicas(g) -> int:
     if rc:
         raise EchoError(rc, lib.echo_strerror(rc).decode())
     return int(n.value)
+
+
+def overlap_candidates(g) -> np.ndarray:
+    """Host-only: uint8 [n_ops], 1 for the compute ops the validator tests (those
+    that can overlap a comm op of their rank in some scenario)."""
+    lib = load_library()
+    keep: list = []
+    d = _graph_desc(g, keep)
+    out = np.zeros(int(g.kind.shape[0]), np.uint8)
+    n = C.c_int64(0)
+    rc = lib.echo_overlap_candidates(C.byref(d), _ptr(out) if out.size else None, C.byref(n))
+    if rc:
+        raise EchoError(rc, lib.echo_strerror(rc).decode())
+    assert int(out.sum()) == int(n.value)
+    return out
 
 
 class Echo:

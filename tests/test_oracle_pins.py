@@ -623,3 +623,30 @@ def test_empty_graph_and_no_scenarios():
     g = SG.graph_from_lists(1, 2, [], {}, [])
     r = oracle.compose(g, _scen_fixed(3, dur=np.zeros((0, 3), np.int64)))
     assert (r.makespan == 0).all()
+
+
+def test_overlap_candidates_cover_every_overlap():
+    # the library's static candidate set (host analysis) must contain every kernel
+    # that the oracle's validator ever slows, in any scenario and variant; and it is
+    # a real filter on the GPT workloads
+    from paper_2412_12487_gb300.echo import overlap_candidates
+    rng = np.random.default_rng(4040)
+    for case in range(120):
+        g = SG.random_graph(rng, int(rng.integers(2, 40)), max_ranks=4, max_streams=5,
+                            p_edge=float(rng.choice([0.03, 0.1, 0.25])))
+        cand = overlap_candidates(g).astype(bool)
+        assert not cand[g.kind != W.KIND_COMPUTE].any()
+        sc = SG.random_scenarios(rng, g, 6, max_dur=int(rng.choice([5, 40, 400])))
+        for civ in (0, 1):
+            for model in (0, 1):
+                r = oracle.compose(g, sc, refine_passes=2, overlap_model=model, comm_interval=civ)
+                slowed = r.overlapped.any(axis=1).astype(bool)
+                assert not (slowed & ~cand).any(), (case, civ, model, np.nonzero(slowed & ~cand)[0])
+    for name, lo, hi in (("tiny", 0.05, 0.6), ("gpt1.3b", 0.05, 0.3)):
+        c = W.config(name)
+        g = W.build_gpt_graph(c)
+        cand = overlap_candidates(g).astype(bool)
+        comp = g.kind == W.KIND_COMPUTE
+        assert lo < cand.sum() / comp.sum() < hi, (name, cand.sum() / comp.sum())
+        r = oracle.compose(g, W.make_scenarios(g, c, n_scen=4), refine_passes=1, comm_interval=1)
+        assert not (r.overlapped.any(axis=1).astype(bool) & ~cand).any()
