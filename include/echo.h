@@ -183,7 +183,9 @@ int echo_destroy(echo_ctx *ctx);
  * the widest level (either pointer may be NULL). */
 int echo_check_graph(const echo_graph_desc *g, int64_t *n_levels, int64_t *max_width);
 
-/* Host-only overlap candidates (Sec. 3's validator tests only these): flags[v] = 1
+/* Host-only overlap candidates: the compute ops that the validator pass (Sec. 3, 6)
+ * tests.  This pruning is a static analysis of this library, not a step of the
+ * paper, and never changes a result: flags[v] = 1
  * for every compute op v (caller ids) that can overlap a comm op of its rank in
  * some scenario, judged from the issue order and data edges among the rank's own
  * ops (an op that must finish before the comm op starts, or start after it ends,
@@ -269,9 +271,10 @@ int echo_cc_query(echo_ctx *ctx, const echo_cc_query_desc *q, double *out_ns);
  *     before any stream capture.
  *   - Every call shares the array and clears its status word: calls that overlap
  *     on the GPU race.
- *   - A query whose node count M exceeds 65536 gets NaN and the call returns
- *     ECHO_E_UNSUPPORTED; a malformed query (the checks of echo_cc_query) gets NaN
- *     and the call returns ECHO_E_INVALID_ARG; other queries are still estimated. */
+ *   - A query whose node count M exceeds 65536 gets NaN, and so does a malformed
+ *     query (the checks of echo_cc_query); other queries are still estimated.  The
+ *     call returns ECHO_E_INVALID_ARG if any query was malformed, else
+ *     ECHO_E_UNSUPPORTED if any node count was too large, whatever the mix. */
 int echo_cc_query_noalloc(const echo_cc_query_desc *q, double *out_ns, void *cuda_stream);
 
 /* Shape of the loaded graph (after echo_load_graph).  n_ops counts the caller's
@@ -289,6 +292,8 @@ typedef struct {
                                         scenarios), chosen for graphs with many levels and
                                         few scenarios */
   int32_t replicas_folded;
+  int64_t n_validator_comm_entries; /* (comm op, member rank) pairs the validator's cursors
+                                       visit: those that can overlap a compute op of the rank */
 } echo_graph_info;
 int echo_graph_info_get(echo_ctx *ctx, echo_graph_info *info);
 

@@ -70,7 +70,9 @@ struct GraphBuild {
   std::vector<int32_t> cidx;          // [V] level-order index of a candidate (by internal id), -1 otherwise
   std::vector<int32_t> cand_cidx;     // level-order index of each entry of cand_ops
   std::vector<int32_t> cand_node;     // internal id of each candidate, in level order
-  std::vector<int64_t> ov_chunks;     // (rank, first candidate index) of the overlap test's chunks
+  std::vector<uint8_t> cand_kcl;      // kernel class of each entry of cand_ops
+  std::vector<uint8_t> q_rel;         // [queue entries] 1 for a comm op that can overlap a compute op
+                                      // of the entry's rank in some scenario (see overlap_candidates)
   int32_t n_cq = 0;                   // comm timelines per rank in cq_off (max over ranks)
   std::vector<int64_t> cq_off;        // [R*n_cq+1] comm ops of each (rank, comm timeline)
   std::vector<int32_t> cq_ops;        // internal ids, in issue order
@@ -93,15 +95,17 @@ bool finite_nonneg(double x) { return std::isfinite(x) && x >= 0.0; }
 constexpr int64_t kStepNodes = 2048;     // nodes of one composition step (a level or a part of one)
 constexpr int64_t kStepSegments = 1024;  // segments of one composition step
 
-// Compute ops that can overlap a comm op of their rank in some scenario (the
-// validator of Sec. 3 tests only these).  A rank's compute timeline is a serial
-// chain, so for a comm op w on rank r the compute ops of r up to the latest one
-// that reaches w finish before w starts, and those from the earliest one that w
-// reaches on start after w ends: only positions in between, (anc(w), desc(w)),
-// can intersect w's interval, whatever the durations.  anc and desc follow the
-// edges among rank r's own ops (data edges and the order of r's timelines); paths
-// through other ranks are ignored, which only widens the ranges.  Needs the
-// internal numbering (a topological order), q_off/q_ops_int and dp.
+// Compute ops that can overlap a comm op of their rank in some scenario: the only
+// ones the validator pass (Sec. 3, 6) tests.  This pruning is a static analysis of
+// this library, not a step of the paper; it never changes a result.  A rank's
+// compute timeline is a serial chain, so for a comm op w on rank r the compute ops
+// of r up to the latest one that reaches w finish before w starts, and those from
+// the earliest one that w reaches on start after w ends: only positions in
+// between, (anc(w), desc(w)), can intersect w's interval, whatever the durations.
+// anc and desc follow the edges among rank r's own ops (data edges and the order
+// of r's timelines); paths through other ranks are ignored, which only widens the
+// ranges.  Needs the internal numbering (a topological order), q_off/q_ops_int
+// and dp.
 void overlap_candidates(GraphBuild &b) {
   const int64_t V = b.V;
   const int32_t R = b.R, NS = b.NS;
@@ -118,7 +122,8 @@ void overlap_candidates(GraphBuild &b) {
   b.cand_off.assign(R + 1, 0);
   b.cand_ops.clear();
   b.cand_flag.assign(V, 0);
-  b.ov_chunks.clear();
+  b.cand_kcl.clear();
+  b.q_rel.assign(std::max<int64_t>(b.q_off[(int64_t)R * NS], 1), 0);
   std::vector<int32_t> nodes, cpos, prv, nxt, anc, desc;
   std::vector<int64_t> cover;
   for (int32_t r = 0; r < R; ++r) {
@@ -161,19 +166,24 @@ void overlap_candidates(GraphBuild &b) {
         cover[anc[j] + 1]++;
         cover[desc[j]]--;
       }
-    const int64_t first = (int64_t)b.cand_ops.size();
+    // the comm ops the validator's cursors visit on this rank: only those whose
+    // range holds a compute position (a tensor-parallel all-reduce between its
+    // producer and its consumer never overlaps a compute op of the rank, so its
+    // interval can be skipped without changing any decision or covered length)
+    for (int32_t k = 1; k < NS; ++k)
+      for (int64_t i = b.q_off[(int64_t)r * NS + k]; i < b.q_off[(int64_t)r * NS + k + 1]; ++i) {
+        const int32_t w = b.q_ops_int[i];
+        b.q_rel[i] = b.is_comm[w] && anc[loc[w]] + 1 < desc[loc[w]];
+      }
     int64_t run = 0;
     for (int64_t p = 0; p < n; ++p) {
       run += cover[p];
       if (run > 0) {
         const int32_t v = b.q_ops_int[c0 + p];
         b.cand_ops.push_back(v);
+        b.cand_kcl.push_back(b.kcl[v]);
         b.cand_flag[v] = 1;
       }
-    }
-    for (int64_t p = first; p < (int64_t)b.cand_ops.size(); p += echo::kOverlapChunk) {
-      b.ov_chunks.push_back(r);
-      b.ov_chunks.push_back(p);
     }
     b.cand_off[r + 1] = (int64_t)b.cand_ops.size();
     for (int64_t j = 0; j < m; ++j) loc[nodes[j]] = -1;
@@ -192,6 +202,7 @@ void overlap_candidates(GraphBuild &b) {
   b.cand_cidx.resize(b.cand_ops.size());
   for (size_t k = 0; k < b.cand_ops.size(); ++k) b.cand_cidx[k] = b.n_cand ? b.cidx[b.cand_ops[k]] : 0;
   if (b.cand_ops.empty()) b.cand_ops.push_back(0);
+  if (b.cand_kcl.empty()) b.cand_kcl.push_back(0);
   if (b.cand_cidx.empty()) b.cand_cidx.push_back(0);
 }
 
@@ -705,13 +716,14 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e, const std::vect
     }
   }
   overlap_candidates(b);
-  // the comm ops of each rank's timelines that hold any, in issue order
+  // the comm ops that can overlap a compute op of their rank, on each of the
+  // rank's timelines that hold any, in issue order
   for (int32_t r = 0; r < R; ++r) {
     int32_t n = 0;
     for (int32_t k = 1; k < NS; ++k) {
       const int64_t q = (int64_t)r * NS + k;
       for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i)
-        if (b.is_comm[b.q_ops_int[i]]) {
+        if (b.q_rel[i]) {
           ++n;
           break;
         }
@@ -741,7 +753,7 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e, const std::vect
         const size_t before = b.cq_ops.size();
         for (int64_t i = g->q_off[q]; i < g->q_off[q + 1]; ++i) {
           const int32_t w = b.q_ops_int[i];
-          if (!b.is_comm[w]) continue;
+          if (!b.q_rel[i]) continue;
           b.cq_ops.push_back(w);
           std::fill(best.begin(), best.end(), -1);
           if (i > g->q_off[q]) best[k] = i - 1;
@@ -1215,7 +1227,8 @@ struct echo_ctx {
   size_t raw_cap = 0;
   // device graph
   int64_t *seg_lvl_off = nullptr, *seg_node_off = nullptr, *nq_off = nullptr, *dp_off = nullptr, *q_off = nullptr;
-  int64_t *ov_chunks = nullptr, *cq_off = nullptr;
+  int64_t *cq_off = nullptr;
+  uint8_t *cand_kcl = nullptr;
   int32_t *cq_ops = nullptr, *lq_off = nullptr, *lq_ops = nullptr;
   int64_t *cand_off = nullptr;
   int32_t *cand_ops = nullptr;
@@ -1231,9 +1244,7 @@ struct echo_ctx {
   echo::MatLayout lay{0, 0};
   ChunkTable tbl{};
   double *prm = nullptr, *sums = nullptr, *comm_sum = nullptr, *cc_ns = nullptr;
-  uint64_t *sfx = nullptr;  // packed slowdown factors [C][S]
   double *sf = nullptr;     // slowdown factors [C][S]
-  std::vector<uint64_t> h_sfx;
   void *raw = nullptr;
   int64_t *dur = nullptr, *f[2] = {nullptr, nullptr}, *mk = nullptr, *cc_dur = nullptr;
   int64_t *gfrontier = nullptr;
@@ -1420,7 +1431,7 @@ int upload_graph(echo_ctx *c) {
   auto &o = c->graph_allocs;
   int rc;
   if ((rc = upload(c, o, &c->seg_lvl_off, B.seg_lvl_off)) || (rc = upload(c, o, &c->seg_node_off, B.seg_node_off)) ||
-      (rc = upload(c, o, &c->ov_chunks, B.ov_chunks)) ||
+      (rc = upload(c, o, &c->cand_kcl, B.cand_kcl)) ||
       (rc = upload(c, o, &c->cq_off, B.cq_off)) || (rc = upload(c, o, &c->cq_ops, B.cq_ops)) ||
       (rc = upload(c, o, &c->lq_off, B.lq_off)) || (rc = upload(c, o, &c->lq_ops, B.lq_ops)) ||
       (rc = upload(c, o, &c->cand_off, B.cand_off)) || (rc = upload(c, o, &c->cand_ops, B.cand_ops)) ||
@@ -1702,7 +1713,7 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
     echo::compose_smem_bytes(B.R * B.NS, sigma, &in_smem);
     int64_t nblk = (S + sigma - 1) / sigma;
     const size_t CS = (size_t)std::max<int64_t>(B.n_cand, 1) * (size_t)nblk * sigma;  // compact matrices
-    if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sfx, (size_t)C * S)) || (rc = dalloc(c, o, &c->sf, (size_t)C * S)) ||
+    if ((rc = dalloc(c, o, &c->prm, (size_t)6 * S)) || (rc = dalloc(c, o, &c->sf, (size_t)C * S)) ||
         (rc = dalloc(c, o, &c->sums, (size_t)S)) || (rc = dalloc(c, o, &c->comm_sum, (size_t)S)) ||
         (rc = dalloc(c, o, &c->dur, VS)) ||
         (rc = dalloc(c, o, &c->f[0], VS)) || (rc = dalloc(c, o, &c->f[1], VS)) ||
@@ -1782,16 +1793,6 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   const double *src[6] = {sc->alpha_ns, sc->bw_intra, sc->lat_intra, sc->bw_inter, sc->lat_inter, sc->delta};
   for (int k = 0; k < 6; ++k)
     CK(cudaMemcpyAsync(c->prm + (size_t)k * S, src[k], S * sizeof(double), cudaMemcpyHostToDevice, c->stream), "parameter upload");
-  // slowdown factors as (significand << 11) | biased exponent (factors are finite and > 0)
-  c->h_sfx.resize((size_t)C * S);
-  for (size_t k = 0; k < c->h_sfx.size(); ++k) {
-    uint64_t b;
-    std::memcpy(&b, &sc->slowdown[k], sizeof b);
-    const uint64_t ex = (b >> 52) & 0x7FF, fr = b & ((1ull << 52) - 1);
-    c->h_sfx[k] = ex == 0 ? (fr << 11) | 1 : ((fr | (1ull << 52)) << 11) | ex;
-  }
-  CK(cudaMemcpyAsync(c->sfx, c->h_sfx.data(), c->h_sfx.size() * sizeof(uint64_t), cudaMemcpyHostToDevice, c->stream),
-     "slowdown upload");
   CK(cudaMemcpyAsync(c->sf, sc->slowdown, (size_t)C * S * sizeof(double), cudaMemcpyHostToDevice, c->stream),
      "slowdown upload");
   CK(cudaMemsetAsync(c->sums, 0, S * sizeof(double), c->stream), "memset");
@@ -1858,8 +1859,8 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   if (civ != ECHO_COMM_EXECUTION && civ != ECHO_COMM_LAUNCH)
     return set_err(c, ECHO_E_INVALID_ARG, "unknown comm interval");
   const GraphBuild &B = c->gb;
-  // the pipelined kernel reads the validator's durations of the candidates from a
-  // ring of its own; the others compose from a full matrix built for them
+  // the pipelined and dataflow kernels read the validator's durations of the
+  // candidates (compact rows); the others compose from a full matrix built for them
   const bool ring = c->use_df || (c->plan.ok && c->plan.pipelined && (c->kernel_choice == 0 || c->kernel_choice == 3));
   if (refine > 1 && !c->cd[1]) {
     if ((rc = dalloc(c, c->scen_allocs, &c->cd[1], c->cd_elems))) return rc;
@@ -1869,9 +1870,44 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     if ((rc = dalloc(c, c->scen_allocs, &c->deff, c->scen_vs))) return rc;
   }
   c->state = 3;
-  // one composition with durations `d` (and, for the pipelined kernel, the
-  // candidates' durations `cdur`) into `f`
-  auto compose_pass = [&](const int64_t *d, const int64_t *cdur, int64_t *f) -> cudaError_t {
+  // the inputs of a validator pass, kept to recompute its decisions on demand
+  // (echo_read_overlap runs the overlap test on them again)
+  auto overlap_args = [&](const int64_t *f_prev, const int64_t *cd_used, int64_t *cd_next) {
+    echo::OverlapArgs o{};
+    o.lay = c->lay;
+    o.lay_c = c->lay_c;
+    o.S = c->S;
+    o.n_streams = B.NS;
+    o.n_ranks = B.R;
+    {  // pieces of each rank's list: enough warps for about four waves (16 warps per
+       // SM), each piece at least 64 candidates long
+      const int64_t base = (int64_t)B.R * ((c->S + 31) / 32), want = 4 * 16 * (int64_t)c->sms;
+      const int64_t per_rank = B.n_cand / std::max<int32_t>(B.R, 1);
+      o.parts = (int32_t)std::max<int64_t>(1, std::min((want + base - 1) / base, per_rank / 64));
+    }
+    o.cand_kcl = c->cand_kcl;
+    o.cand_off = c->cand_off;
+    o.cand_ops = c->cand_ops;
+    o.cand_cidx = c->cand_cidx;
+    o.n_cq = B.n_cq;
+    o.cq_off = c->cq_off;
+    o.cq_ops = c->cq_ops;
+    o.lq_off = civ == ECHO_COMM_LAUNCH ? c->lq_off : nullptr;
+    o.lq_ops = c->lq_ops;
+    o.kcl = c->kcl;
+    o.f = f_prev;
+    o.dur = c->dur;
+    o.cd_used = cd_used;
+    o.sf = c->sf;
+    o.model = model;
+    o.cd_next = cd_next;
+    o.ov = nullptr;  // the decisions are recomputed on demand by echo_read_overlap
+    return o;
+  };
+  // one composition with durations `d` (and, for the pipelined and dataflow
+  // kernels, the candidates' durations `cdur`) into `f`
+  auto compose_pass = [&](const int64_t *d, const int64_t *cdur, int64_t *f, bool adjusted) -> cudaError_t {
+    const char *name = adjusted ? "compose_adjusted" : "compose";
     if (c->use_df) {
       echo::DataflowArgs a{};
       a.S = c->S;
@@ -1908,7 +1944,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       if ((err = cudaMemsetAsync(c->mk, 0, (size_t)c->S * sizeof(int64_t), c->stream)) != cudaSuccess ||
           (err = cudaMemsetAsync(c->df_abort, 0, sizeof(int32_t), c->stream)) != cudaSuccess)
         return err;
-      return timed(c, "compose", [&] { return echo::launch_compose_dataflow(a, c->stream); });
+      return timed(c, name, [&] { return echo::launch_compose_dataflow(a, c->stream); });
     }
     if (c->plan.ok && c->kernel_choice != 1) {
       echo::StagedArgs a{};
@@ -1932,8 +1968,8 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       a.skip_level = c->skip_level;
       const bool pipe = c->plan.pipelined && (c->kernel_choice == 0 || c->kernel_choice == 3);
       if (pipe)
-        return timed(c, "compose", [&] { return echo::launch_compose_pipelined(a, c->sigma, c->plan, c->stream); });
-      return timed(c, "compose", [&] { return echo::launch_compose_staged(a, c->sigma, c->plan, c->stream); });
+        return timed(c, name, [&] { return echo::launch_compose_pipelined(a, c->sigma, c->plan, c->stream); });
+      return timed(c, name, [&] { return echo::launch_compose_staged(a, c->sigma, c->plan, c->stream); });
     }
     echo::ComposeArgs a{};
     a.V = B.V;
@@ -1954,36 +1990,13 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     return timed(c, "compose_direct", [&] { return echo::launch_compose(a, c->sigma, c->stream); });
   };
   CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
-  CK(compose_pass(c->dur, nullptr, c->f[0]), "compose launch");
+  CK(compose_pass(c->dur, nullptr, c->f[0], false), "compose launch");
   const int64_t *cd_used = nullptr;
   for (int32_t p = 1; p <= refine; ++p) {
-    echo::OverlapArgs o{};
-    o.lay = c->lay;
-    o.lay_c = c->lay_c;
-    o.S = c->S;
-    o.n_streams = B.NS;
-    o.n_chunks = (int64_t)B.ov_chunks.size() / 2;
-    o.chunks = c->ov_chunks;
-    o.cand_off = c->cand_off;
-    o.cand_ops = c->cand_ops;
-    o.cand_cidx = c->cand_cidx;
-    o.n_cq = B.n_cq;
-    o.cq_off = c->cq_off;
-    o.cq_ops = c->cq_ops;
-    o.lq_off = civ == ECHO_COMM_LAUNCH ? c->lq_off : nullptr;
-    o.lq_ops = c->lq_ops;
-    o.kcl = c->kcl;
-    o.f = c->f[(p - 1) % 2];
-    o.dur = c->dur;
-    o.cd_used = cd_used;
-    o.sfx = c->sfx;
-    o.sf = c->sf;
-    o.model = model;
-    o.cd_next = c->cd[(p - 1) % 2];
-    o.ov = nullptr;  // the decisions are recomputed on demand by echo_read_overlap
+    echo::OverlapArgs o = overlap_args(c->f[(p - 1) % 2], cd_used, c->cd[(p - 1) % 2]);
     CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");
     if (ring) {
-      CK(compose_pass(c->dur, o.cd_next, c->f[p % 2]), "compose launch");
+      CK(compose_pass(c->dur, o.cd_next, c->f[p % 2], true), "compose launch");
     } else {
       CK(cudaMemcpyAsync(c->deff, c->dur, c->scen_vs * sizeof(int64_t), cudaMemcpyDeviceToDevice, c->stream),
          "duration copy");
@@ -1991,7 +2004,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
            return echo::launch_scatter_candidates(c->cand_node, B.n_cand, c->S, c->lay, c->lay_c, o.cd_next, c->deff,
                                                   c->stream);
          }), "scatter launch");
-      CK(compose_pass(c->deff, nullptr, c->f[p % 2]), "compose launch");
+      CK(compose_pass(c->deff, nullptr, c->f[p % 2], true), "compose launch");
     }
     cd_used = o.cd_next;
     c->last_ov = o;
@@ -2010,9 +2023,18 @@ static int composition_status(echo_ctx *c) {
   if (rc) return rc;
   if (st == echo::kDevTimeout) {
     if (c->use_df) {  // words a warp never wrote must not carry a later launch's tag
-      cudaMemsetAsync(c->df_part, 0, c->df_part_elems * sizeof(uint64_t), c->stream);
-      cudaMemsetAsync(c->df_xval, 0, c->df_xval_elems * sizeof(uint64_t), c->stream);
-      cudaStreamSynchronize(c->stream);
+      cudaError_t e = cudaMemsetAsync(c->df_part, 0, c->df_part_elems * sizeof(uint64_t), c->stream);
+      if (e == cudaSuccess) e = cudaMemsetAsync(c->df_xval, 0, c->df_xval_elems * sizeof(uint64_t), c->stream);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+      if (e != cudaSuccess) {
+        // the words may still hold stale tags: drop the scenario buffers, so that
+        // the next echo_load_scenarios allocates and zeroes fresh ones
+        (void)cudaGetLastError();
+        free_all(c->scen_allocs);
+        c->scen_vs = 0;
+        c->state = 1;
+        return cuda_fail(c, e, "clearing the dataflow words after a timeout");
+      }
     }
     return set_err(c, ECHO_E_TIMEOUT, "a device-side wait of the composer gave up");
   }
@@ -2190,6 +2212,7 @@ int echo_graph_info_get(echo_ctx *c, echo_graph_info *info) {
   info->n_segments = B.n_seg;
   info->n_segment_levels = B.Ls;
   info->n_overlap_candidates = B.cand_off.empty() ? 0 : B.cand_off.back();
+  info->n_validator_comm_entries = B.cq_off.empty() ? 0 : B.cq_off.back();
   info->n_ranks = B.R;
   info->n_streams = B.NS;
   info->sigma = c->sigma;

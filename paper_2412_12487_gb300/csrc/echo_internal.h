@@ -14,8 +14,9 @@ constexpr int kComposeThreads = 512;       // direct compose kernel
 constexpr int kMetaChunk = 128;            // segment levels of metadata staged at a time
 constexpr int kMetaCap = 136;              // metadata entries per staging buffer (>= kMetaChunk + 1)
 constexpr uint32_t kFarRef = 0x80000000u;  // predecessor reference read from global memory
-constexpr int kOverlapChunk = 128;         // compute ops per overlap-test thread
-constexpr int kOverlapThreads = 128;       // threads per block of the overlap test
+constexpr int kOvBatch = 8;                // candidates per batch of the overlap test
+constexpr int kOvDepth = 3;                // batches of candidate rows in flight per warp
+constexpr int kOvWarps = 4;                // warps per block of the overlap test
 constexpr int kMaxSegment = 64;            // longest serial chain composed as one segment
 constexpr int kPipeStages = 16;            // stages (mbarrier pairs) of the pipelined compose
 constexpr int kPipeConsumerWarps = 16;     // composing warps of the pipelined compose
@@ -136,10 +137,11 @@ struct OverlapArgs {
   MatLayout lay_c;         // [n_cand][S] compact matrices (rows in level order)
   int32_t S, n_streams;
   int32_t n_cq;            // comm timelines per rank (lists of a rank with fewer are empty)
-  int64_t n_chunks;
-  const int64_t *chunks;   // [n_chunks][2]: (rank, first candidate index)
+  int32_t n_ranks;
+  int32_t parts;           // pieces of each rank's candidate list (one warp per piece and 32 scenarios)
   const int64_t *cand_off; const int32_t *cand_ops;  // [R+1]: each rank's overlap candidates, in issue order
   const int32_t *cand_cidx;                          // level-order index of each entry of cand_ops
+  const uint8_t *cand_kcl;                           // kernel class of each entry of cand_ops
   const int64_t *cq_off; const int32_t *cq_ops;  // [R*n_cq+1]: comm ops of each (rank, comm timeline)
   // launch conditions of each entry of cq_ops on its rank (CSR); null: a comm op's
   // interval is its execution [start, finish), else [latest of them, finish)
@@ -148,8 +150,7 @@ struct OverlapArgs {
   const int64_t *f;        // finish times of the last pass
   const int64_t *dur;      // original durations
   const int64_t *cd_used;  // candidates' durations in the last pass (compact), or null: the original ones
-  const uint64_t *sfx;     // [C][S] slowdown factors, packed as (53-bit significand << 11) | (exponent + 1075)
-  const double *sf;        // [C][S] the same factors (proportional model)
+  const double *sf;        // [C][S] slowdown factors
   int32_t model;           // 0: d * factor; 1: d + (factor - 1) * overlapped length
   int64_t *cd_next;        // (out, compact; may be null) candidates' durations for the next pass
   uint8_t *ov;             // (out, [V][S] rows of the candidates; may be null)
@@ -200,6 +201,9 @@ cudaError_t launch_compose_dataflow(const DataflowArgs &a, cudaStream_t st);
 size_t dataflow_smem_bytes(int32_t n_streams);
 // whether every warp of R * G warps can be resident at once (cooperative launch)
 bool dataflow_fits(int64_t n_warps, int32_t n_streams, int device);
+
+// shared memory of an overlap-test block: each warp's ring of candidate rows
+inline size_t overlap_smem_bytes() { return (size_t)kOvWarps * kOvDepth * kOvBatch * 2 * 32 * sizeof(int64_t); }
 
 // overlap.cu: the overlap test, one entry point per (launch interval, proportional
 // model) pair, each dispatching on the number of comm timelines

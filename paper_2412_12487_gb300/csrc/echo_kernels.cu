@@ -335,12 +335,11 @@ cudaError_t launch_replica_check(const void *raw, int bits, const int32_t *pairs
 }
 
 cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
-  if (a.S == 0 || a.n_chunks == 0) return cudaSuccess;
-  if (a.n_cq < 0 || a.n_cq > kMaxStreams) return cudaErrorInvalidValue;
-  const int tx = a.S >= kOverlapThreads ? kOverlapThreads : ((a.S + 31) / 32) * 32;
-  int64_t gy = a.n_chunks < 65535 ? a.n_chunks : 65535;
-  int64_t gz = (a.n_chunks + gy - 1) / gy;
-  const dim3 grid((a.S + tx - 1) / tx, (unsigned)gy, (unsigned)gz);
+  const int64_t warps = (int64_t)a.n_ranks * ((a.S + 31) / 32) * a.parts;
+  if (a.S == 0 || warps == 0) return cudaSuccess;
+  if (a.n_cq < 0 || a.n_cq > kMaxStreams || a.parts < 1) return cudaErrorInvalidValue;
+  const dim3 grid((unsigned)((warps + kOvWarps - 1) / kOvWarps));
+  const int tx = kOvWarps * 32;
   // the variants are compiled in four translation units (echo_overlap.cu)
   const bool prop = a.model == 1 && a.cd_next;
   if (a.lq_off)
@@ -393,8 +392,8 @@ cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int
 // device memory the kernel touches is the file-scope array below, which every GPU
 // that loads this library holds until the process exits.
 //
-// Layout of the array: bytes [0, 4) hold a status word, cleared at the start of
-// every call; from byte 256 on, log2(m) for m = 0..kNoallocMaxNodes, computed on
+// Layout of the array: bytes [0, 4) hold a status word (one bit per kind of bad
+// query), cleared at the start of every call; from byte 256 on, log2(m) for m = 0..kNoallocMaxNodes, computed on
 // the host with the same libm log2 the allocating path uses, so both paths give
 // identical estimates.  Node counts above kNoallocMaxNodes are rejected.
 // ---------------------------------------------------------------------------------
@@ -404,6 +403,8 @@ constexpr int32_t kNoallocMaxNodes = 65536;
 constexpr size_t kNoallocLgOffset = 256;
 constexpr size_t kNoallocScratchBytes = kNoallocLgOffset + sizeof(double) * (kNoallocMaxNodes + 1);
 constexpr int kNoallocMaxDevices = 64;
+// status bits: a batch may hold both kinds of bad query, so each sets its own bit
+// and the host ranks them (a malformed query before an unsupported size)
 enum : int32_t { kNoallocOk = 0, kNoallocTooManyNodes = 1, kNoallocBadQuery = 2 };
 }  // namespace
 }  // namespace echo
@@ -457,12 +458,12 @@ __global__ void cc_query_noalloc_kernel(int64_t n, const uint8_t *__restrict__ t
                     isfinite(p.bwe[i]) && p.bwe[i] > 0.0;
     if (!ok) {
       out[i] = nan;
-      set_status(status, kNoallocBadQuery);
+      atomicOr(status, kNoallocBadQuery);
       continue;
     }
     if (m > kNoallocMaxNodes) {
       out[i] = nan;
-      set_status(status, kNoallocTooManyNodes);
+      atomicOr(status, kNoallocTooManyNodes);
       continue;
     }
     const int K = (n_r + m - 1) / m;
@@ -518,7 +519,7 @@ extern "C" int echo_cc_query_noalloc(const echo_cc_query_desc *q, double *out_ns
   if (cudaMemcpyAsync(&status, d.ptr, sizeof(int32_t), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
       cudaStreamSynchronize(st) != cudaSuccess)
     return ECHO_E_CUDA;
-  if (status == kNoallocTooManyNodes) return ECHO_E_UNSUPPORTED;
-  if (status == kNoallocBadQuery) return ECHO_E_INVALID_ARG;
+  if (status & kNoallocBadQuery) return ECHO_E_INVALID_ARG;
+  if (status & kNoallocTooManyNodes) return ECHO_E_UNSUPPORTED;
   return ECHO_OK;
 }

@@ -7,6 +7,7 @@
 #include <cstdint>
 
 #include "echo_internal.h"
+#include "echo_slowdown.cuh"
 
 #if !defined(ECHO_OV_LAUNCH) || !defined(ECHO_OV_PROP)
 #error "compile with -DECHO_OV_LAUNCH=0|1 -DECHO_OV_PROP=0|1"
@@ -15,51 +16,16 @@
 namespace echo {
 namespace {
 
-// rint(p * 2^e) with ties to even, for p < 2^63 and a result below 2^63.
-__device__ __forceinline__ int64_t rint_scaled(uint64_t p, int e) {
-  if (e >= 0) return (int64_t)(p << e);
-  const int k = -e;
-  if (k >= 64) return 0;  // p * 2^e < 2^63 * 2^-64 = 1/2
-  const uint64_t q = p >> k, rem = p & ((1ull << k) - 1), half = 1ull << (k - 1);
-  return (int64_t)(q + ((rem > half || (rem == half && (q & 1))) ? 1 : 0));
-}
+using dev::slowed;
 
-// Slowed duration rint(fl(fl(d) * f)) (Sec. 2.3: a kernel's time grows by its
-// slowdown factor), evaluated exactly in integers so that the fp64 pipe, which is
-// slow on this part, stays idle.  f = M * 2^E is passed packed as (M << 11) |
-// (E + 1075), M < 2^53 its significand.  Each rounding is IEEE 754
-// roundTiesToEven: d to 53 significant bits (the int64 -> double conversion), the
-// exact product d * M (< 2^106) to 53 significant bits (the double product), then
-// to an integer (rint).  Products below 2^-1022, where the double product would be
-// subnormal, round to 0 either way.
-__device__ __forceinline__ int64_t slowed(int64_t d, uint64_t packed) {
-  const uint64_t M = packed >> 11;
-  int e = (int)(packed & 0x7FF) - 1075;
-  uint64_t x = (uint64_t)d;
-  if (x >> 53) {
-    const int s = 11 - __clzll((long long)x);  // bit length - 53
-    const uint64_t q = x >> s, rem = x & ((1ull << s) - 1), half = 1ull << (s - 1);
-    x = q + ((rem > half || (rem == half && (q & 1))) ? 1 : 0);
-    e += s;
-  }
-  const uint64_t lo = x * M, hi = __umul64hi(x, M);
-  const int nb = hi ? 128 - __clzll((long long)hi) : 64 - __clzll((long long)lo);
-  uint64_t p = lo;
-  if (nb > 53) {  // nb <= 106, so 1 <= s <= 53 and every dropped bit is in lo
-    const int s = nb - 53;
-    p = (lo >> s) | (hi << (64 - s));
-    const uint64_t rem = lo & ((1ull << s) - 1), half = 1ull << (s - 1);
-    p += (rem > half || (rem == half && (p & 1))) ? 1 : 0;
-    e += s;
-  }
-  return rint_scaled(p, e);
-}
+// Blocks per SM the register budget allows (4 warps each); wide cursor sets keep
+// their registers instead of spilling.
+constexpr int overlap_min_blocks(int ncmax) { return ncmax <= 6 ? 4 : ncmax <= 8 ? 3 : 1; }
 
-constexpr int kOverlapBatch = 8;  // divides 32 (the shuffled op list's width)
-// Blocks per SM the register budget allows.  Occupancy hides the row-load latency
-// (at 3 comm timelines, 64 registers beat 108 by 12%); wide cursor sets keep their
-// registers instead of spilling.
-constexpr int overlap_min_blocks(int ncmax) { return ncmax <= 3 ? 8 : ncmax <= 4 ? 6 : 1; }
+__device__ __forceinline__ void cp_async8(void *dst, const void *src) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(d), "l"(src) : "memory");
+}
 
 // When rank r launched the comm op of cq entry e: the latest finish among its
 // launch conditions on r (out of line: the cursor loads are unrolled many times).
@@ -70,21 +36,46 @@ __device__ __noinline__ int64_t launch_time(const int32_t *__restrict__ lq_off, 
   return t;
 }
 
+// The validator's overlap test, as a walk over each rank's candidates.  Warp w
+// takes piece p of rank r's candidate list (in issue order) for 32 scenarios
+// (one per lane).  Every timeline of a rank runs its ops one after the other, so
+// on each comm timeline the intervals are sorted and the candidates' starts only
+// grow: the lane keeps, per comm timeline, a cursor at the first comm op of
+// positive length that finishes after the current candidate starts, with that
+// op's interval in registers.  The candidate overlaps this timeline iff that
+// interval starts before the candidate finishes (later comm ops start after the
+// cursor op ends).  A piece that starts mid-list places its cursors by binary
+// search; the first piece starts them at the list heads.  The cursor lists hold
+// only the comm ops that can overlap a compute op of the rank, so moves are rare,
+// and the smallest cursor end and start decide most candidates with two
+// comparisons.  The finish times and durations of the candidates come through a
+// ring of kOvDepth batches of 8 (cp.async), so each warp keeps several batches of
+// loads in flight.  An overlapped compute op of positive length gets
+// rint(d * slowdown) (or the proportional form, both in fp64: on this part the
+// multiply costs fewer issue slots than an exact integer form) for the next composition
+// (cd_next, compact); the decisions themselves are stored only when `ov` is given.
 // LAUNCH: a comm op's interval on the rank opens at the rank's launch of it
-// (a.lq_off), else at its start.  PROP: the proportional slowdown model (a.model 1)
+// (a.lq_off), else at its start.  PROP: the proportional slowdown model.
 template <int NCMAX, bool LAUNCH, bool PROP>
-__global__ void __launch_bounds__(kOverlapThreads, overlap_min_blocks(NCMAX)) overlap_kernel(OverlapArgs a) {
+__global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) overlap_kernel(OverlapArgs a) {
+  extern __shared__ int64_t ov_ring[];
   const int32_t S = a.S;
-  const int32_t s = blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t c = blockIdx.y + (int64_t)gridDim.y * blockIdx.z;
-  if (c >= a.n_chunks) return;  // uniform over the block
-  const bool act = s < S;       // inactive lanes still take part in the warp shuffles
-  const int32_t sl = act ? s : 0;
   const int lane = threadIdx.x & 31;
+  const int64_t wid = (int64_t)blockIdx.x * kOvWarps + (threadIdx.x >> 5);
+  const int64_t G = (S + 31) / 32;
+  if (wid >= (int64_t)a.n_ranks * G * a.parts) return;  // uniform over the warp
+  const int32_t part = (int32_t)(wid % a.parts);
+  const int32_t r = (int32_t)(wid / a.parts % a.n_ranks);
+  const int32_t s = (int32_t)(wid / a.parts / a.n_ranks) * 32 + lane;
+  const bool act = s < S;  // inactive lanes still take part in the shuffles and copies
+  const int32_t sl = act ? s : 0;
   const int nc = a.n_cq;
-  const int64_t r = a.chunks[2 * c];
-  const int64_t c0 = a.chunks[2 * c + 1];
-  const int64_t c1 = min(a.cand_off[r + 1], c0 + kOverlapChunk);
+  // this piece of the rank's list, cut at multiples of the batch
+  const int64_t r0 = a.cand_off[r], r1 = a.cand_off[r + 1];
+  const int64_t nb = (r1 - r0 + kOvBatch - 1) / kOvBatch;
+  const int64_t c0 = min(r1, r0 + nb * part / a.parts * kOvBatch);
+  const int64_t c1 = min(r1, r0 + nb * (part + 1) / a.parts * kOvBatch);
+  if (c0 >= c1) return;
   // element (i, s) of a matrix sits at base + (i << sh)
   const int sh = a.lay.slog2;
   const int64_t base = a.lay.at(0, sl);
@@ -94,9 +85,7 @@ __global__ void __launch_bounds__(kOverlapThreads, overlap_min_blocks(NCMAX)) ov
   // previous validator pass's (compact [candidate][scenario] rows)
   const int64_t *__restrict__ cu = a.cd_used ? a.cd_used + a.lay_c.at(0, sl) : nullptr;
   int64_t *__restrict__ cn = a.cd_next ? a.cd_next + a.lay_c.at(0, sl) : nullptr;
-  int32_t qreg = c0 + lane < c1 ? a.cand_ops[c0 + lane] : 0;   // ops c0 .. c0+31 of the chunk
-  int32_t creg = c0 + lane < c1 ? a.cand_cidx[c0 + lane] : 0;  // and their level-order indices
-  auto cand_d = [&](int64_t v, int64_t ci) { return cu ? cu[ci << sh] : du[v << sh]; };
+  int64_t *ring = ov_ring + (int64_t)(threadIdx.x >> 5) * (kOvDepth * kOvBatch * 2 * 32) + lane;
   // per comm timeline: position, end, and interval of the cursor op; the cursor op
   // always has positive length and finishes after the current op's start (or the
   // cursor is at the end, with an interval that never overlaps)
@@ -116,21 +105,26 @@ __global__ void __launch_bounds__(kOverlapThreads, overlap_min_blocks(NCMAX)) ov
     }
   };
   {
-    const int64_t v = __shfl_sync(0xffffffffu, qreg, 0), ci = __shfl_sync(0xffffffffu, creg, 0);
-    const int64_t sv = act ? f[v << sh] - cand_d(v, ci) : 0;
+    int64_t sv0 = 0;  // the piece's first candidate's start (only for a search)
+    if (part > 0) {
+      const int64_t v = a.cand_ops[c0], ci = a.cand_cidx[c0];
+      sv0 = f[v << sh] - (cu ? cu[ci << sh] : du[v << sh]);
+    }
 #pragma unroll
     for (int j = 0; j < NCMAX; ++j) {
       cur[j] = end[j] = 0;
       sw[j] = fw[j] = INT64_MAX;
-      if (j < nc && act) {
+      if (j < nc) {
         int32_t lo = (int32_t)a.cq_off[r * nc + j], hi = (int32_t)a.cq_off[r * nc + j + 1];
         end[j] = hi;
-        while (lo < hi) {  // first comm op finishing after sv (finishes are sorted)
-          const int32_t mid = (lo + hi) >> 1;
-          if (f[(int64_t)a.cq_ops[mid] << sh] > sv)
-            hi = mid;
-          else
-            lo = mid + 1;
+        if (part > 0) {
+          while (lo < hi) {  // first comm op finishing after sv0 (finishes are sorted)
+            const int32_t mid = (lo + hi) >> 1;
+            if (f[(int64_t)a.cq_ops[mid] << sh] > sv0)
+              hi = mid;
+            else
+              lo = mid + 1;
+          }
         }
         cur[j] = lo;
         load(j);
@@ -141,92 +135,142 @@ __global__ void __launch_bounds__(kOverlapThreads, overlap_min_blocks(NCMAX)) ov
       }
     }
   }
-  // groups of kOverlapBatch ops: their finish times and durations are loaded together
-  for (int64_t i0 = c0; i0 < c1; i0 += kOverlapBatch) {
-    if (i0 > c0 && ((i0 - c0) & 31) == 0) {
-      qreg = i0 + lane < c1 ? a.cand_ops[i0 + lane] : 0;
-      creg = i0 + lane < c1 ? a.cand_cidx[i0 + lane] : 0;
-    }
-    int64_t vb[kOverlapBatch], cb[kOverlapBatch], fb[kOverlapBatch], db[kOverlapBatch];
+  // The smallest cursor end and start over the timelines: while every cursor op
+  // ends after a candidate starts (fmin > sv), no cursor moves, and the candidate
+  // overlaps iff some cursor op starts before it ends (smin < fv).
+  int64_t fmin, smin;
+  auto bounds = [&]() {
+    fmin = smin = INT64_MAX;
 #pragma unroll
-    for (int u = 0; u < kOverlapBatch; ++u) {
-      vb[u] = __shfl_sync(0xffffffffu, qreg, (int)((i0 - c0 + u) & 31));
-      cb[u] = __shfl_sync(0xffffffffu, creg, (int)((i0 - c0 + u) & 31));
-      fb[u] = db[u] = 0;
-      if (act && i0 + u < c1) {
-        fb[u] = f[vb[u] << sh];
-        db[u] = cand_d(vb[u], cb[u]);
+    for (int j = 0; j < NCMAX; ++j)
+      if (j < nc) {
+        fmin = min(fmin, fw[j]);
+        smin = min(smin, sw[j]);
+      }
+  };
+  bounds();
+  // candidate ids of a batch: lanes 0..7 hold node, level-order index and class
+  auto ids = [&](int64_t i0, int32_t &q, int32_t &cx, int32_t &kc) {
+    const int64_t i = i0 + (lane & (kOvBatch - 1));
+    const bool in = i < c1;
+    q = in ? a.cand_ops[i] : 0;
+    cx = in ? a.cand_cidx[i] : 0;
+    kc = in ? a.cand_kcl[i] : 0;
+  };
+  // the batch's finish times and durations (those of the pass that produced f)
+  auto issue = [&](int64_t i0, int32_t q, int32_t cx) {
+    int64_t *slot = ring + ((i0 - c0) / kOvBatch % kOvDepth) * (kOvBatch * 2 * 32);
+#pragma unroll
+    for (int u = 0; u < kOvBatch; ++u) {
+      const int64_t v = __shfl_sync(0xffffffffu, q, u), ci = __shfl_sync(0xffffffffu, cx, u);
+      if (i0 + u < c1) {
+        cp_async8(slot + (2 * u) * 32, f + (v << sh));
+        cp_async8(slot + (2 * u + 1) * 32, cu ? cu + (ci << sh) : du + (v << sh));
       }
     }
-    if (!act) continue;
-#pragma unroll
-    for (int u = 0; u < kOverlapBatch; ++u) {
-      if (i0 + u < c1) {
-        const int64_t v = vb[u], fv = fb[u], dv = db[u];
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+  };
+  static_assert(kOvDepth == 3, "the id registers below hold kOvDepth batches");
+  int32_t q0, x0, k0, q1, x1, k1, q2, x2, k2, q3, x3, k3;
+  ids(c0, q0, x0, k0);
+  ids(c0 + kOvBatch, q1, x1, k1);
+  ids(c0 + 2 * kOvBatch, q2, x2, k2);
+  issue(c0, q0, x0);
+  issue(c0 + kOvBatch, q1, x1);
+  for (int64_t i0 = c0; i0 < c1; i0 += kOvBatch) {
+    ids(i0 + 3 * kOvBatch, q3, x3, k3);
+    issue(i0 + 2 * kOvBatch, q2, x2);
+    asm volatile("cp.async.wait_group 2;\n" ::: "memory");  // this batch's copies landed
+    int64_t *slot = ring + ((i0 - c0) / kOvBatch % kOvDepth) * (kOvBatch * 2 * 32);
+    const int n_here = c1 - i0 < kOvBatch ? (int)(c1 - i0) : kOvBatch;
+    // 1) the cursor walk, candidate after candidate: a bit per overlapped candidate
+    //    (and, proportional model, its covered length in place of its finish)
+    uint32_t hits = 0;
+    if (act) {
+#pragma unroll 1
+      for (int u = 0; u < n_here; ++u) {
+        const int64_t fv = slot[(2 * u) * 32], dv = slot[(2 * u + 1) * 32];
         const int64_t sv = fv - dv;
-        bool hit = false;
+        if (fmin <= sv) {
 #pragma unroll
-        for (int j = 0; j < NCMAX; ++j) {
-          if (j < nc) {
-            if (fw[j] <= sv) {  // the cursor op ended before this op starts: move on
+          for (int j = 0; j < NCMAX; ++j) {
+            if (j < nc && fw[j] <= sv) {  // the cursor op ended before this op starts: move on
               do {
                 ++cur[j];
                 load(j);
               } while (cur[j] < end[j] && (fw[j] <= sv || sw[j] >= fw[j]));
             }
-            hit |= sw[j] < fv;
           }
+          bounds();
         }
-        hit = hit && sv < fv;
-        if (a.ov) a.ov[base + (v << sh)] = hit;
-        if (cn) {
-          const int64_t d0 = cu ? du[v << sh] : dv;  // the original duration
-          int64_t dn = d0;
-          if (PROP && hit) {
-            // proportional model: the length of [sv, fv) covered by the union of the
-            // comm intervals, swept in start order across the timelines.  Later
-            // candidates start no earlier than fv, so a cursor moves past every
-            // interval that ends by fv; one reaching beyond fv stays.
-            int64_t len = 0, covered = sv;
-            uint32_t held = 0;  // timelines whose cursor interval reaches beyond fv
-            while (true) {
-              int jb = -1;
-              int64_t first = fv;
+        const bool hit = smin < fv && sv < fv;
+        hits |= (uint32_t)hit << u;
+        if (PROP && hit && cn) {
+          // proportional model: the length of [sv, fv) covered by the union of the
+          // comm intervals, swept in start order across the timelines.  Later
+          // candidates start no earlier than fv, so a cursor moves past every
+          // interval that ends by fv; one reaching beyond fv stays.
+          int64_t len = 0, covered = sv;
+          uint32_t held = 0;  // timelines whose cursor interval reaches beyond fv
+          while (true) {
+            int jb = -1;
+            int64_t first = fv;
 #pragma unroll
-              for (int j = 0; j < NCMAX; ++j)
-                if (j < nc && !((held >> j) & 1) && sw[j] < first) {
-                  first = sw[j];
-                  jb = j;
-                }
-              if (jb < 0) break;
+            for (int j = 0; j < NCMAX; ++j)
+              if (j < nc && !((held >> j) & 1) && sw[j] < first) {
+                first = sw[j];
+                jb = j;
+              }
+            if (jb < 0) break;
 #pragma unroll
-              for (int j = 0; j < NCMAX; ++j) {  // (j == jb, in registers)
-                if (j != jb) continue;
-                const int64_t lo = max(sw[j], covered), hi = min(fw[j], fv);
-                if (hi > lo) {
-                  len += hi - lo;
-                  covered = hi;
-                }
-                if (fw[j] > fv) {
-                  held |= 1u << j;
-                } else {
-                  do {
-                    ++cur[j];
-                    load(j);
-                  } while (cur[j] < end[j] && sw[j] >= fw[j]);
-                }
+            for (int j = 0; j < NCMAX; ++j) {  // (j == jb, in registers)
+              if (j != jb) continue;
+              const int64_t lo = max(sw[j], covered), hi = min(fw[j], fv);
+              if (hi > lo) {
+                len += hi - lo;
+                covered = hi;
+              }
+              if (fw[j] > fv) {
+                held |= 1u << j;
+              } else {
+                do {
+                  ++cur[j];
+                  load(j);
+                } while (cur[j] < end[j] && sw[j] >= fw[j]);
               }
             }
-            const double f = a.sf[(int64_t)a.kcl[v] * S + sl];
-            dn = __double2ll_rn(__dadd_rn((double)d0, __dmul_rn(__dsub_rn(f, 1.0), (double)len)));
-          } else if (hit) {
-            dn = slowed(d0, a.sfx[(int64_t)a.kcl[v] * S + sl]);
           }
-          cn[cb[u] << sh] = dn;
+          bounds();
+          slot[(2 * u) * 32] = len;
         }
       }
     }
+    // 2) the outputs, the batch's candidates independently of each other
+#pragma unroll
+    for (int u = 0; u < kOvBatch; ++u) {
+      const int64_t v = __shfl_sync(0xffffffffu, q0, u);
+      const int64_t kc = __shfl_sync(0xffffffffu, k0, u);
+      const int64_t ci = __shfl_sync(0xffffffffu, x0, u);
+      if (!act || u >= n_here) continue;
+      const bool hit = (hits >> u) & 1;
+      if (a.ov) a.ov[base + (v << sh)] = hit;
+      if (cn) {
+        const int64_t d0 = cu ? du[v << sh] : slot[(2 * u + 1) * 32];  // the original duration
+        int64_t dn = d0;
+        if (hit) {
+          if (PROP)
+            dn = dev::slowed_proportional(d0, a.sf[kc * S + sl], slot[(2 * u) * 32]);
+          else
+            dn = slowed(d0, a.sf[kc * S + sl]);
+        }
+        cn[ci << sh] = dn;
+      }
+    }
+    q0 = q1, x0 = x1, k0 = k1;
+    q1 = q2, x1 = x2, k1 = k2;
+    q2 = q3, x2 = x3, k2 = k3;
   }
+  asm volatile("cp.async.wait_all;\n" ::: "memory");
 }
 
 }  // namespace
@@ -236,18 +280,19 @@ __global__ void __launch_bounds__(kOverlapThreads, overlap_min_blocks(NCMAX)) ov
 
 cudaError_t ECHO_OV_NAME(ECHO_OV_LAUNCH, ECHO_OV_PROP)(const OverlapArgs &a, dim3 grid, int tx, cudaStream_t st) {
   constexpr bool L = ECHO_OV_LAUNCH != 0, P = ECHO_OV_PROP != 0;
+  const size_t smem = overlap_smem_bytes();
   // (the 3-cursor variant serves 1 and 2 comm timelines too: every cursor loop
   // stops at the actual count)
   if (a.n_cq <= 3)
-    overlap_kernel<3, L, P><<<grid, tx, 0, st>>>(a);
+    overlap_kernel<3, L, P><<<grid, tx, smem, st>>>(a);
   else if (a.n_cq <= 4)
-    overlap_kernel<4, L, P><<<grid, tx, 0, st>>>(a);
+    overlap_kernel<4, L, P><<<grid, tx, smem, st>>>(a);
   else if (a.n_cq <= 6)
-    overlap_kernel<6, L, P><<<grid, tx, 0, st>>>(a);
+    overlap_kernel<6, L, P><<<grid, tx, smem, st>>>(a);
   else if (a.n_cq <= 8)
-    overlap_kernel<8, L, P><<<grid, tx, 0, st>>>(a);
+    overlap_kernel<8, L, P><<<grid, tx, smem, st>>>(a);
   else
-    overlap_kernel<kMaxStreams, L, P><<<grid, tx, 0, st>>>(a);
+    overlap_kernel<kMaxStreams, L, P><<<grid, tx, smem, st>>>(a);
   return cudaGetLastError();
 }
 

@@ -75,7 +75,7 @@ class GraphInfo(C.Structure):
                 ("n_signatures", C.c_int64), ("n_segments", C.c_int64), ("n_segment_levels", C.c_int64),
                 ("n_overlap_candidates", C.c_int64), ("n_ops_composed", C.c_int64),
                 ("n_ranks", C.c_int32), ("n_streams", C.c_int32), ("sigma", C.c_int32),
-                ("replicas_folded", C.c_int32)]
+                ("replicas_folded", C.c_int32), ("n_validator_comm_entries", C.c_int64)]
 
 
 class KernelStat(C.Structure):

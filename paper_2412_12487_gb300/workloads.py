@@ -161,6 +161,10 @@ CONFIGS: Dict[str, GPTConfig] = {
                          scen_seed=1003),
     "gpt175b-1024": GPTConfig("gpt-175b-tp8pp16dp8-m64-v2", 96, 12288, 96, 2048, 8, 16, 8, 64, 64,
                               scen_seed=1004, virtual_stages=2),
+    # a smaller case of the 1024-rank workload's structure (same ranks, schedule and
+    # timelines; 32 layers, 16 micro-batches), for kernel profiles that must stay small
+    "gpt175b-1024-small": GPTConfig("gpt-175b-tp8pp16dp8-m16-v2-32L", 32, 12288, 96, 2048, 8, 16, 8, 16, 64,
+                                    scen_seed=1004, virtual_stages=2),
 }
 
 

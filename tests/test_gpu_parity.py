@@ -89,10 +89,10 @@ def test_validator_many_comm_timelines_long_compute_timelines(S):
 
 
 def test_slowdown_rounding_is_exact():
-    """The validator evaluates rint(d * factor) in integers: every scenario slows one
-    kernel that overlaps a collective from time 0, with edge-case durations (around
-    2^31, 2^52, 2^53, large) and factors (exact ties, 1 + 2^-52, 1/3, tiny, subnormal),
-    and the slowed duration must equal the fp64 product rounded to nearest even."""
+    """The validator's rint(d * factor): every scenario slows one kernel that overlaps
+    a collective from time 0, with edge-case durations (around 2^31, 2^52, 2^53,
+    large) and factors (exact ties, 1 + 2^-52, 1/3, tiny, subnormal), and the slowed
+    duration must equal numpy's fp64 product rounded to nearest even."""
     ops = [{"kind": W.KIND_COMPUTE, "kclass": 0}, {"kind": W.KIND_COMPUTE, "kclass": 0},
            {"kind": W.KIND_COLL, "group": 0, "cc_type": W.CC_ALLREDUCE, "cc_bytes": 1 << 20}]
     g = SG.graph_from_lists(2, 2, ops, {(0, 0): [0], (1, 0): [1], (0, 1): [2], (1, 1): [2]}, [[0, 1]])
@@ -448,6 +448,30 @@ def test_dataflow_compose_bit_exact(monkeypatch):
             sc = SG.random_scenarios(rng, g, int(rng.choice([1, 31, 32, 33, 70])), max_dur=30)
             got = run_gpu(g, sc, 2, ctx=e)
             assert_same(got, oracle.compose(g, sc, refine_passes=2), g, 2)
+    finally:
+        e.close()
+
+
+@pytest.mark.parametrize("streams", [(2, 4), (5, 7), (8, 16)])
+def test_dataflow_validator_variants_bit_exact(streams, monkeypatch):
+    """The dataflow composer with the validator between its compositions (cursor
+    sets 3-, 4-, 6-, 8- and 16-wide): random multi-rank graphs with 1 to 15 comm
+    timelines per rank and long compute timelines, both overlap models, both comm
+    intervals and 1 to 3 validator passes, against the oracle."""
+    monkeypatch.setenv("ECHO_COMPOSE_KERNEL", "dataflow")
+    lo, hi = streams
+    rng = np.random.default_rng(7100 + hi)
+    e = Echo(0)
+    try:
+        for case in range(10):
+            g = SG.random_graph(rng, int(rng.integers(100, 700)), max_ranks=4, max_streams=hi,
+                                min_streams=lo, p_edge=0.004 if case % 2 else 0.02)
+            sc = SG.random_scenarios(rng, g, int(rng.choice([7, 32, 45, 64])), max_dur=60)
+            refine, model, civ = [(1, 0, 0), (2, 1, 0), (3, 0, 1), (1, 1, 1), (2, 0, 0)][case % 5]
+            got = run_gpu(g, sc, refine, ctx=e, overlap_model=model, comm_interval=civ)
+            assert got["info"]["sigma"] == 32
+            want = oracle.compose(g, sc, refine_passes=refine, overlap_model=model, comm_interval=civ)
+            assert_same(got, want, g, refine)
     finally:
         e.close()
 

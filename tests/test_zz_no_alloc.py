@@ -78,3 +78,25 @@ def test_noalloc_rejects_node_counts_beyond_its_table():
     rc, got = _call(lib, q2, stream)
     assert rc == 0
     np.testing.assert_allclose(got, want, rtol=CC_RTOL, atol=0)
+
+
+def test_noalloc_mixed_bad_queries_report_the_malformed_one():
+    """A batch with both a malformed query and one whose node count exceeds the
+    table returns ECHO_E_INVALID_ARG every time (the malformed query ranks first),
+    with NaN for both and every other query estimated."""
+    import torch
+    lib = E.load_library()
+    stream = torch.cuda.current_stream()
+    q = W.make_cc_queries(5000, seed=15)
+    bad = [17, 4000]              # M > N: malformed
+    big = [3, 2500, 4999]         # M > 65536: beyond the table
+    for i in bad:
+        q.n_nodes[i] = q.n_ranks[i] + 1
+    for i in big:
+        q.n_ranks[i] = 300_000
+        q.n_nodes[i] = 100_000
+    for _ in range(5):
+        rc, got = _call(lib, q, stream)
+        assert rc == 1  # ECHO_E_INVALID_ARG
+        assert np.isnan(got[bad + big]).all()
+        assert np.isfinite(np.delete(got, bad + big)).all()
