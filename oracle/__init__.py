@@ -52,7 +52,7 @@ class _Scen(C.Structure):
                 ("lat_intra", C.c_void_p), ("bw_inter", C.c_void_p), ("lat_inter", C.c_void_p),
                 ("delta", C.c_void_p), ("slowdown", C.c_void_p),
                 ("chunk_max_bytes", C.c_void_p), ("chunk_bytes", C.c_void_p), ("cc_model", C.c_int32),
-                ("overlap_model", C.c_int32), ("comm_interval", C.c_int32)]
+                ("overlap_model", C.c_int32), ("comm_interval", C.c_int32), ("ar_algo_policy", C.c_int32)]
 
 
 def _load():
@@ -119,13 +119,17 @@ class OracleResult:
 
 def compose(g, sc, refine_passes: int = 1, tie_seed: int = 0, threads: int = 1,
             want_cc: bool = True, want_overlap: bool = True, cc_model: int = 0,
-            overlap_model: int = 0, comm_interval: int = 0) -> OracleResult:
+            overlap_model: int = 0, comm_interval: int = 0, ar_algo_policy: int = 0,
+            want_times: bool = True) -> OracleResult:
     """Compose every scenario of ``sc`` on graph ``g`` (workloads.Graph/Scenarios).
     cc_model 0 takes collective times from Eqs. 2-5, 1 from the alpha-beta model.
     overlap_model 0 slows an overlapped kernel to d * factor, 1 to
     d + (factor - 1) * (length of its overlap with the rank's communication).
     comm_interval 0 takes a comm op's execution interval [start, finish) on each
-    member rank, 1 the interval from the rank's own launch of it to its finish."""
+    member rank, 1 the interval from the rank's own launch of it to its finish.
+    ar_algo_policy 0 keeps every all-reduce's own algorithm; 1 ring, 2 tree, 3 the
+    faster of the two, for every all-reduce.  want_times False returns only the
+    makespans (start and finish are None), for large batches."""
     lib = _load()
     V, S = g.n_ops, sc.n_scen
     keep = []
@@ -147,9 +151,9 @@ def compose(g, sc, refine_passes: int = 1, tie_seed: int = 0, threads: int = 1,
                arr(sc.slowdown, np.float64),
                arr(sc.chunk_max_bytes, np.int64) if n_chunk else None,
                arr(sc.chunk_bytes, np.int64) if n_chunk else None, int(cc_model), int(overlap_model),
-               int(comm_interval))
-    start = np.zeros((V, S), np.int64)
-    finish = np.zeros((V, S), np.int64)
+               int(comm_interval), int(ar_algo_policy))
+    start = np.zeros((V, S), np.int64) if want_times else None
+    finish = np.zeros((V, S), np.int64) if want_times else None
     mk = np.zeros(S, np.int64)
     ccn = np.full((V, S), np.nan) if want_cc else None
     ov = np.zeros((V, S), np.uint8) if want_overlap else None
@@ -159,7 +163,7 @@ def compose(g, sc, refine_passes: int = 1, tie_seed: int = 0, threads: int = 1,
 
     def run(i):
         rcs[i] = lib.oracle_compose(C.byref(gs), C.byref(ss), int(bounds[i]), int(bounds[i + 1]),
-                                    refine_passes, tie_seed, start.ctypes.data, finish.ctypes.data,
+                                    refine_passes, tie_seed, _p(start), _p(finish),
                                     mk.ctypes.data, _p(ccn), _p(ov))
 
     if threads == 1:

@@ -32,7 +32,9 @@
  *   launch conditions on r, rather than when the last member has); the bare "(N-1)" inside Eqs. 3-4 is read as a per-step latency,
  *   so every ring step costs L + p/B; send/recv costs eta chunk transfers over the
  *   intra- or inter-node link; AUTO all-reduce takes the faster of ring and tree
- *   (ties to ring); N = 1 or 0 bytes costs 0; slowed duration = rint(d * factor).
+ *   (ties to ring); an all-reduce policy (ring, tree or auto for every all-reduce)
+ *   may replace the per-op algorithm; N = 1 or 0 bytes costs 0; slowed duration =
+ *   rint(d * factor).
  *
  * Parity pins: see tests/test_oracle_pins.py.  Every function here is pinned
  * (closed forms, Table 6, brute force, invariants); none is "parity unpinned".
@@ -279,6 +281,7 @@ int oracle_compose(const oracle_graph *g, const oracle_scen *sc, int32_t s0, int
   int64_t V = g->n_ops;
   int32_t S = sc->n_scen;
   if (V < 0 || S < 0 || s0 < 0 || s1 > S || s0 > s1 || refine_passes < 0) return ORACLE_E_INVALID;
+  if (sc->ar_algo_policy < 0 || sc->ar_algo_policy > 3) return ORACLE_E_INVALID;
   int64_t nq = (int64_t)g->n_streams * g->n_ranks;
   int rc = 0;
 
@@ -367,9 +370,11 @@ int oracle_compose(const oracle_graph *g, const oracle_scen *sc, int32_t s0, int
       uint8_t k = g->kind[v];
       if (k == K_COLL || k == K_P2P) {
         int32_t gi = g->group[v];
+        /* an all-reduce policy replaces every all-reduce's own algorithm */
+        const int algo = g->cc_type[v] == T_AR && sc->ar_algo_policy > 0 ? sc->ar_algo_policy - 1 : g->cc_algo[v];
         double T = sc->cc_model == 1
                        ? oracle_cc_ns_alpha_beta(g->cc_bytes[v], gN[gi], gM[gi], prm)
-                       : oracle_cc_ns(g->cc_type[v], g->cc_algo[v], g->cc_bytes[v], gN[gi], gM[gi], gK[gi],
+                       : oracle_cc_ns(g->cc_type[v], algo, g->cc_bytes[v], gN[gi], gM[gi], gK[gi],
                                       glg[gi], prm, sc->n_chunk, sc->chunk_max_bytes, sc->chunk_bytes);
         if (cc_ns) cc_ns[v * S + s] = T;
         d0[v] = llrint(T);

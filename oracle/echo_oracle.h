@@ -39,6 +39,9 @@ typedef struct {
                             0: its execution [start, finish);
                             1: [launch on r, finish), launch = when r's own launch
                                conditions of it hold */
+  int32_t ar_algo_policy; /* all-reduce algorithm (Sec. 5.1: NCCL runs ring or tree):
+                             0: each op's own cc_algo; 1: ring, 2: tree, 3: the
+                             faster of the two, for every all-reduce */
 } oracle_scen;
 
 int64_t oracle_chunk_bytes(int64_t nbytes, int n_chunk, const int64_t *max_bytes,

@@ -398,6 +398,41 @@ def test_auto_takes_the_faster_algorithm():
         assert _cc(W.CC_ALLREDUCE, W.ALGO_AUTO, S, N, M, K, p) == min(r, t)
 
 
+@pytest.mark.parametrize("seed", range(4))
+def test_allreduce_policy_equals_rewriting_every_allreduce(seed):
+    """Sec. 5.1: NCCL runs an all-reduce as a ring or a tree.  A policy that forces
+    ring, tree or the faster of the two must give exactly the composition of the
+    same graph with every all-reduce's own algorithm rewritten to it, must leave
+    every other collective's estimate alone, and AUTO must be the per-op minimum
+    of the forced ring and tree estimates.  The graphs mix the three per-op
+    algorithms, and the large messages make ring and tree differ."""
+    import dataclasses
+    rng = np.random.default_rng(8800 + seed)
+    differs = False
+    for _ in range(12):
+        g = SG.random_graph(rng, int(rng.integers(10, 60)), max_ranks=5, max_streams=4, p_edge=0.08)
+        g = dataclasses.replace(g, cc_bytes=np.where(g.cc_bytes > 0, g.cc_bytes * 4096, 0))
+        sc = SG.random_scenarios(rng, g, 5, max_dur=2000)
+        ar = (g.cc_type == W.CC_ALLREDUCE) & ((g.kind == W.KIND_COLL) | (g.kind == W.KIND_P2P))
+        comm = (g.kind == W.KIND_COLL) | (g.kind == W.KIND_P2P)
+        base = oracle.compose(g, sc, refine_passes=1)
+        got = {}
+        for policy, algo in ((1, W.ALGO_RING), (2, W.ALGO_TREE), (3, W.ALGO_AUTO)):
+            forced = oracle.compose(g, sc, refine_passes=1, ar_algo_policy=policy)
+            g2 = dataclasses.replace(g, cc_algo=np.where(ar, algo, g.cc_algo).astype(np.uint8))
+            rewritten = oracle.compose(g2, sc, refine_passes=1)
+            assert np.array_equal(forced.finish, rewritten.finish)
+            assert np.array_equal(forced.start, rewritten.start)
+            np.testing.assert_array_equal(forced.cc_ns[comm], rewritten.cc_ns[comm])
+            np.testing.assert_array_equal(forced.cc_ns[comm & ~ar], base.cc_ns[comm & ~ar])
+            got[policy] = forced
+        np.testing.assert_array_equal(got[3].cc_ns[ar], np.minimum(got[1].cc_ns[ar], got[2].cc_ns[ar]))
+        differs |= bool((got[1].cc_ns[ar] != got[2].cc_ns[ar]).any())
+    assert differs
+    with pytest.raises(RuntimeError):
+        oracle.compose(g, sc, ar_algo_policy=4)
+
+
 def test_monotone_in_size_and_inverse_bandwidth():
     rng = np.random.default_rng(17)
     for _ in range(300):
