@@ -39,7 +39,7 @@
 extern "C" {
 #endif
 
-#define ECHO_ABI_VERSION 1
+#define ECHO_ABI_VERSION 2
 
 typedef enum {
   ECHO_OK = 0,
@@ -167,9 +167,17 @@ typedef struct {
    * before it on r's timeline and its data producers that run on r have finished:
    * the comm kernel is resident on r while it waits for the other members. */
   int32_t comm_interval;
+  /* all-reduce algorithm (Sec. 5.1: NCCL runs an all-reduce as a ring or a tree):
+   * ECHO_AR_PER_OP (0, default) keeps each op's cc_algo; ECHO_AR_RING, ECHO_AR_TREE
+   * and ECHO_AR_AUTO (the faster of the two) apply to every all-reduce of the
+   * graph.  When it differs from the policy of the current estimates, echo_compose
+   * runs the CC estimator again first (ECHO_E_OVERFLOW as there), and echo_read_cc
+   * then reports those estimates. */
+  int32_t ar_algo_policy;
 } echo_compose_opts;
 enum { ECHO_OVERLAP_WHOLE = 0, ECHO_OVERLAP_PROPORTIONAL = 1 };
 enum { ECHO_COMM_EXECUTION = 0, ECHO_COMM_LAUNCH = 1 };
+enum { ECHO_AR_PER_OP = 0, ECHO_AR_RING = 1, ECHO_AR_TREE = 2, ECHO_AR_AUTO = 3 };
 
 /* Create a context on `device`, enqueuing on `cuda_stream` (a cudaStream_t; NULL =
  * a new non-blocking stream owned by the context; the legacy default stream is
@@ -209,8 +217,8 @@ int echo_load_scenarios(echo_ctx *ctx, const echo_scen_desc *sc);
 
 /* CC estimator (Sec. 5.2-5.3): for every comm op and scenario, the execution time
  * of Eqs. 2-5 (ring all-gather, ring reduce-scatter, ring/tree/auto all-reduce,
- * send/recv) in fp64 ns; the op's duration is that value rounded to the nearest
- * integer (ties to even).  Group shape: N members, M distinct nodes, K = the
+ * send/recv, each all-reduce with its own cc_algo) in fp64 ns; the op's duration
+ * is that value rounded to the nearest integer (ties to even).  Group shape: N members, M distinct nodes, K = the
  * largest member count on one node, log2(M) computed on the host.  A time that
  * could overflow the composition -> ECHO_E_OVERFLOW. */
 int echo_estimate_collectives(echo_ctx *ctx);
@@ -232,9 +240,15 @@ int echo_set_cc_model(echo_ctx *ctx, int model);
  * enqueues work; opts may be NULL (refine_passes = 1). */
 int echo_compose(echo_ctx *ctx, const echo_compose_opts *opts);
 
-/* Final start and finish of ops [op0, op1) (caller ids), all scenarios, into host
- * buffers of (op1-op0)*S int64 each, row-major [op][s].  Either may be NULL. */
-int echo_read_times(echo_ctx *ctx, int64_t op0, int64_t op1, int64_t *start, int64_t *finish);
+/* Final start and finish (Sec. 4.2: every op's place on its timelines) of ops
+ * [op0, op1) (caller ids) in scenarios [s0, s1), into caller buffers of
+ * (op1-op0)*(s1-s0) int64 each, row-major [op][s - s0]: host memory (pageable or
+ * pinned) or device memory of the context's device.  Either may be NULL.  A range
+ * outside [0, n_ops) x [0, n_scen) or an empty scenario range with ops:
+ * ECHO_E_INVALID_ARG.  Large ranges are read back in chunks through a staging
+ * buffer of the context. */
+int echo_read_times(echo_ctx *ctx, int64_t op0, int64_t op1, int32_t s0, int32_t s1, int64_t *start,
+                    int64_t *finish);
 /* Step time per scenario: the largest finish time (0 for an empty graph). [S] */
 int echo_read_makespan(echo_ctx *ctx, int64_t *makespan);
 /* CC estimates (fp64 ns) of ops [op0, op1), [op][s]; NaN for non-comm ops. */

@@ -1273,6 +1273,7 @@ struct echo_ctx {
   uint32_t df_epoch = 0;
   int32_t *df_abort = nullptr;
   int cc_model = ECHO_CC_MODEL_WHITEBOX;
+  int est_policy = ECHO_AR_PER_OP;  // all-reduce policy of the current estimates
   long long wait_limit_cycles = 0;  // bound of every device-side wait
   int32_t skip_level = -1;          // failure injection for tests
   // scratch for readback / queries
@@ -1812,10 +1813,9 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   return ECHO_OK;
 }
 
-int echo_estimate_collectives(echo_ctx *c) {
-  int rc = check_ctx(c);
-  if (rc) return rc;
-  if (c->state < 2) return set_err(c, ECHO_E_STATE, "load scenarios first");
+// CC estimates of every signature and scenario under all-reduce policy `policy`,
+// scattered into the duration rows of the comm ops, with the overflow check.
+static int run_estimate(echo_ctx *c, int policy) {
   const GraphBuild &B = c->gb;
   const int32_t S = c->S, G = (int32_t)B.sigs.size();
   c->state = 2;
@@ -1825,7 +1825,7 @@ int echo_estimate_collectives(echo_ctx *c) {
   CK(cudaMemsetAsync(c->comm_sum, 0, S * sizeof(double), c->stream), "memset");
   CK(timed(c, "cc_estimate", [&] {
        return echo::launch_cc_estimate(c->sigs, G, p, S, c->tbl, c->sig_count, c->cc_ns, c->cc_dur,
-                                       c->comm_sum, c->status, c->cc_model, c->stream);
+                                       c->comm_sum, c->status, c->cc_model, policy, c->stream);
      }), "cc_estimate launch");
   CK(timed(c, "cc_scatter", [&] {
        return echo::launch_cc_scatter(c->comm_node, c->comm_sig, (int64_t)B.comm_node.size(), c->cc_dur, S,
@@ -1834,6 +1834,7 @@ int echo_estimate_collectives(echo_ctx *c) {
   std::vector<double> comm(S, 0.0);
   CK(cudaMemcpyAsync(comm.data(), c->comm_sum, S * sizeof(double), cudaMemcpyDeviceToHost, c->stream), "readback");
   int32_t st = 0;
+  int rc;
   if ((rc = sync_status(c, &st))) return rc;
   if (st == echo::kDevCcOverflow) return set_err(c, ECHO_E_OVERFLOW, "a collective's estimated time is not below 2^61 ns");
   // every finish time is at most the sum of all (slowed) durations of its scenario
@@ -1842,8 +1843,16 @@ int echo_estimate_collectives(echo_ctx *c) {
     if (!(bound < 2305843009213693952.0))
       return set_err(c, ECHO_E_OVERFLOW, "scenario " + std::to_string(s) + ": total duration could overflow int64");
   }
+  c->est_policy = policy;
   c->state = 3;
   return ECHO_OK;
+}
+
+int echo_estimate_collectives(echo_ctx *c) {
+  int rc = check_ctx(c);
+  if (rc) return rc;
+  if (c->state < 2) return set_err(c, ECHO_E_STATE, "load scenarios first");
+  return run_estimate(c, ECHO_AR_PER_OP);
 }
 
 int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
@@ -1858,6 +1867,10 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   const int32_t civ = opts ? opts->comm_interval : ECHO_COMM_EXECUTION;
   if (civ != ECHO_COMM_EXECUTION && civ != ECHO_COMM_LAUNCH)
     return set_err(c, ECHO_E_INVALID_ARG, "unknown comm interval");
+  const int32_t policy = opts ? opts->ar_algo_policy : ECHO_AR_PER_OP;
+  if (policy < ECHO_AR_PER_OP || policy > ECHO_AR_AUTO)
+    return set_err(c, ECHO_E_INVALID_ARG, "unknown all-reduce policy");
+  if (policy != c->est_policy && (rc = run_estimate(c, policy))) return rc;
   const GraphBuild &B = c->gb;
   // the pipelined and dataflow kernels read the validator's durations of the
   // candidates (compact rows); the others compose from a full matrix built for them
@@ -2047,27 +2060,32 @@ static int read_range_check(echo_ctx *c, int64_t op0, int64_t op1, int need_stat
   return ECHO_OK;
 }
 
-int echo_read_times(echo_ctx *c, int64_t op0, int64_t op1, int64_t *start, int64_t *finish) {
+int echo_read_times(echo_ctx *c, int64_t op0, int64_t op1, int32_t s0, int32_t s1, int64_t *start,
+                    int64_t *finish) {
   int rc = check_ctx(c);
   if (rc) return rc;
   if ((rc = read_range_check(c, op0, op1, 4))) return rc;
+  if (s0 < 0 || s1 > c->S || s1 < s0 || (s1 == s0 && op1 > op0))
+    return set_err(c, ECHO_E_INVALID_ARG, "scenario range out of bounds");
   if ((rc = composition_status(c))) return rc;
-  const int32_t S = c->S;
-  const int64_t rows_per = std::max<int64_t>(1, (int64_t)(64 << 20) / S);
-  if ((rc = stage_reserve(c, (size_t)std::min<int64_t>(rows_per, std::max<int64_t>(op1 - op0, 1)) * S * 16)))
+  const int32_t Sr = s1 - s0;
+  if (Sr == 0) return ECHO_OK;
+  const int64_t rows_per = std::max<int64_t>(1, (int64_t)(64 << 20) / Sr);
+  if ((rc = stage_reserve(c, (size_t)std::min<int64_t>(rows_per, std::max<int64_t>(op1 - op0, 1)) * Sr * 16)))
     return rc;
   for (int64_t a = op0; a < op1; a += rows_per) {
     int64_t b = std::min(op1, a + rows_per);
-    int64_t n = (b - a) * S;
+    int64_t n = (b - a) * Sr;
     int64_t *ds = static_cast<int64_t *>(c->stage);
     int64_t *df = ds + n;
     CK(timed(c, "readback", [&] {
-         return echo::launch_readback(c->ext2int, a, b, S, c->lay, c->f[c->final_f], c->dur, c->cidx, c->lay_c,
-                                      c->final_cd,
-                                      start ? ds : nullptr, finish ? df : nullptr, c->stream);
+         return echo::launch_readback(c->ext2int, a, b, s0, s1, c->lay, c->f[c->final_f], c->dur, c->cidx, c->lay_c,
+                                      c->final_cd, start ? ds : nullptr, finish ? df : nullptr, c->stream);
        }), "readback launch");
-    if (start) CK(cudaMemcpyAsync(start + (a - op0) * S, ds, n * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream), "D2H");
-    if (finish) CK(cudaMemcpyAsync(finish + (a - op0) * S, df, n * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream), "D2H");
+    if (start)
+      CK(cudaMemcpyAsync(start + (a - op0) * Sr, ds, n * sizeof(int64_t), cudaMemcpyDefault, c->stream), "copy out");
+    if (finish)
+      CK(cudaMemcpyAsync(finish + (a - op0) * Sr, df, n * sizeof(int64_t), cudaMemcpyDefault, c->stream), "copy out");
     CK(cudaStreamSynchronize(c->stream), "readback");
   }
   return ECHO_OK;

@@ -213,9 +213,11 @@ cudaError_t launch_overlap_l1_p0(const OverlapArgs &a, dim3 grid, int tx, cudaSt
 cudaError_t launch_overlap_l1_p1(const OverlapArgs &a, dim3 grid, int tx, cudaStream_t st);
 
 // kernels.cu
+// ar_policy: 0 each signature's own all-reduce algorithm, else 1 + the algorithm for all
 cudaError_t launch_cc_estimate(const CcSig *sig, int32_t G, ScenParams p, int32_t S,
                                const ChunkTable &tbl, const int32_t *sig_count, double *cc_ns,
-                               int64_t *cc_dur, double *comm_sum, int32_t *status, int model, cudaStream_t st);
+                               int64_t *cc_dur, double *comm_sum, int32_t *status, int model, int ar_policy,
+                               cudaStream_t st);
 cudaError_t launch_cc_scatter(const int32_t *comm_node, const int32_t *comm_sig, int64_t n_comm,
                               const int64_t *cc_dur, int32_t S, MatLayout lay, int64_t *dur, cudaStream_t st);
 cudaError_t launch_cc_query(int64_t n, const uint8_t *type, const uint8_t *algo, const int64_t *nbytes,
@@ -232,7 +234,7 @@ cudaError_t launch_compose(const ComposeArgs &a, int sigma, cudaStream_t st);
 cudaError_t launch_compose_staged(const StagedArgs &a, int sigma, const StagedPlan &plan, cudaStream_t st);
 cudaError_t launch_compose_pipelined(const StagedArgs &a, int sigma, const StagedPlan &plan, cudaStream_t st);
 cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st);
-cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
+cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t s0, int32_t s1, MatLayout lay,
                             const int64_t *f, const int64_t *d, const int32_t *cidx, MatLayout lay_c,
                             const int64_t *cd, int64_t *start, int64_t *finish, cudaStream_t st);
 cudaError_t launch_scatter_candidates(const int32_t *cand_node, int64_t n_cand, int32_t S, MatLayout lay,

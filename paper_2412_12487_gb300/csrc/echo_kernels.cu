@@ -90,7 +90,7 @@ __device__ __forceinline__ void set_status(int32_t *status, int32_t code) {
 __global__ void cc_estimate_kernel(const CcSig *__restrict__ sig, int32_t G, ScenParams p, int32_t S,
                                    ChunkTable tbl, const int32_t *__restrict__ sig_count,
                                    double *__restrict__ cc_ns, int64_t *__restrict__ cc_dur,
-                                   double *__restrict__ comm_sum, int32_t *status, int model) {
+                                   double *__restrict__ comm_sum, int32_t *status, int model, int ar_policy) {
   int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)G * S) return;
   int32_t g = (int32_t)(idx / S), s = (int32_t)(idx % S);
@@ -103,7 +103,8 @@ __global__ void cc_estimate_kernel(const CcSig *__restrict__ sig, int32_t G, Sce
             ? 0.0
             : __dadd_rn(q.M > 1 ? p.late[s] : p.lata[s], __ddiv_rn((double)q.nbytes, q.M > 1 ? p.bwe[s] : p.bwa[s]));
   } else {
-    T = cc_ns_of(q.type, q.algo, q.nbytes, q.N, q.M, q.K, q.lg, p.alpha[s], p.bwa[s], p.lata[s], p.bwe[s],
+    const int algo = q.type == kAR && ar_policy > 0 ? ar_policy - 1 : q.algo;  // a policy for every all-reduce
+    T = cc_ns_of(q.type, algo, q.nbytes, q.N, q.M, q.K, q.lg, p.alpha[s], p.bwa[s], p.lata[s], p.bwe[s],
                  p.late[s], p.delta[s], tbl);
   }
   int64_t d = 0;
@@ -193,15 +194,17 @@ __global__ void permute_rows_kernel(const T *__restrict__ raw, const int32_t *__
 // ---------------------------------------------------------------------------------
 // start = finish - the duration the op had in the last composition: d, or for an
 // overlap candidate its row of the compact cd when given
-__global__ void readback_kernel(const int32_t *__restrict__ ext2int, int64_t op0, int64_t op1, int32_t S,
-                                MatLayout lay, const int64_t *__restrict__ f, const int64_t *__restrict__ d,
-                                const int32_t *__restrict__ cidx, MatLayout lay_c, const int64_t *__restrict__ cd,
-                                int64_t *__restrict__ start, int64_t *__restrict__ finish) {
-  int64_t total = (op1 - op0) * S;
+__global__ void readback_kernel(const int32_t *__restrict__ ext2int, int64_t op0, int64_t op1, int32_t s0,
+                                int32_t s1, MatLayout lay, const int64_t *__restrict__ f,
+                                const int64_t *__restrict__ d, const int32_t *__restrict__ cidx, MatLayout lay_c,
+                                const int64_t *__restrict__ cd, int64_t *__restrict__ start,
+                                int64_t *__restrict__ finish) {
+  const int32_t Sr = s1 - s0;
+  int64_t total = (op1 - op0) * Sr;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
        idx += (int64_t)gridDim.x * blockDim.x) {
-    int64_t o = idx / S;
-    int32_t s = (int32_t)(idx - o * S);
+    int64_t o = idx / Sr;
+    int32_t s = s0 + (int32_t)(idx - o * Sr);
     const int32_t i = ext2int[op0 + o];
     int64_t at = lay.at(i, s);
     int64_t fv = f[at];
@@ -264,13 +267,13 @@ int grid_for(int64_t n, int threads) {
 
 cudaError_t launch_cc_estimate(const CcSig *sig, int32_t G, ScenParams p, int32_t S, const ChunkTable &tbl,
                                const int32_t *sig_count, double *cc_ns, int64_t *cc_dur, double *comm_sum,
-                               int32_t *status, int model, cudaStream_t st) {
+                               int32_t *status, int model, int ar_policy, cudaStream_t st) {
   int64_t n = (int64_t)G * S;
   if (n == 0) return cudaSuccess;
   int threads = 256;
   int64_t blocks = (n + threads - 1) / threads;
   cc_estimate_kernel<<<(unsigned)blocks, threads, 0, st>>>(sig, G, p, S, tbl, sig_count, cc_ns, cc_dur,
-                                                          comm_sum, status, model);
+                                                          comm_sum, status, model, ar_policy);
   return cudaGetLastError();
 }
 
@@ -347,12 +350,12 @@ cudaError_t launch_overlap(const OverlapArgs &a, cudaStream_t st) {
   return prop ? launch_overlap_l0_p1(a, grid, tx, st) : launch_overlap_l0_p0(a, grid, tx, st);
 }
 
-cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t S, MatLayout lay,
+cudaError_t launch_readback(const int32_t *ext2int, int64_t op0, int64_t op1, int32_t s0, int32_t s1, MatLayout lay,
                             const int64_t *f, const int64_t *d, const int32_t *cidx, MatLayout lay_c,
                             const int64_t *cd, int64_t *start, int64_t *finish, cudaStream_t st) {
-  int64_t n = (op1 - op0) * S;
+  int64_t n = (op1 - op0) * (s1 - s0);
   if (n <= 0) return cudaSuccess;
-  readback_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, S, lay, f, d, cidx, lay_c, cd, start,
+  readback_kernel<<<grid_for(n, 256), 256, 0, st>>>(ext2int, op0, op1, s0, s1, lay, f, d, cidx, lay_c, cd, start,
                                                     finish);
   return cudaGetLastError();
 }

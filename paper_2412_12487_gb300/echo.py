@@ -37,6 +37,7 @@ CUDA_STREAM_LEGACY = 0x1  # cudaStreamLegacy
 CC_MODEL_WHITEBOX, CC_MODEL_ALPHA_BETA = 0, 1
 OVERLAP_WHOLE, OVERLAP_PROPORTIONAL = 0, 1
 COMM_EXECUTION, COMM_LAUNCH = 0, 1
+AR_PER_OP, AR_RING, AR_TREE, AR_AUTO = 0, 1, 2, 3
 
 
 class GraphDesc(C.Structure):
@@ -58,7 +59,8 @@ class ScenDesc(C.Structure):
 
 
 class ComposeOpts(C.Structure):
-    _fields_ = [("refine_passes", C.c_int32), ("overlap_model", C.c_int32), ("comm_interval", C.c_int32)]
+    _fields_ = [("refine_passes", C.c_int32), ("overlap_model", C.c_int32), ("comm_interval", C.c_int32),
+                ("ar_algo_policy", C.c_int32)]
 
 
 class CCQueryDesc(C.Structure):
@@ -110,7 +112,7 @@ def load_library(path: Optional[str] = None):
         "echo_load_scenarios": ([vp, C.POINTER(ScenDesc)], C.c_int),
         "echo_estimate_collectives": ([vp], C.c_int),
         "echo_compose": ([vp, C.POINTER(ComposeOpts)], C.c_int),
-        "echo_read_times": ([vp, i64, i64, vp, vp], C.c_int),
+        "echo_read_times": ([vp, i64, i64, i32, i32, vp, vp], C.c_int),
         "echo_read_makespan": ([vp, vp], C.c_int),
         "echo_read_cc": ([vp, i64, i64, vp], C.c_int),
         "echo_read_overlap": ([vp, i64, i64, vp], C.c_int),
@@ -282,19 +284,25 @@ class Echo:
     def estimate_collectives(self):
         self._check(self.lib.echo_estimate_collectives(self.h))
 
-    def compose(self, refine_passes: int = 1, overlap_model: int = 0, comm_interval: int = 0):
+    def compose(self, refine_passes: int = 1, overlap_model: int = 0, comm_interval: int = 0,
+                ar_algo_policy: int = 0):
         """overlap_model: OVERLAP_WHOLE (d * factor) or OVERLAP_PROPORTIONAL
         (d + (factor - 1) * overlapped length).  comm_interval: COMM_EXECUTION (a
-        comm op's [start, finish)) or COMM_LAUNCH (from each member rank's launch)."""
-        o = ComposeOpts(int(refine_passes), int(overlap_model), int(comm_interval))
+        comm op's [start, finish)) or COMM_LAUNCH (from each member rank's launch).
+        ar_algo_policy: AR_PER_OP (each all-reduce's own algorithm), AR_RING,
+        AR_TREE or AR_AUTO for every all-reduce."""
+        o = ComposeOpts(int(refine_passes), int(overlap_model), int(comm_interval), int(ar_algo_policy))
         self._check(self.lib.echo_compose(self.h, C.byref(o)))
 
-    def read_times(self, op0: int = 0, op1: Optional[int] = None, start=True, finish=True):
+    def read_times(self, op0: int = 0, op1: Optional[int] = None, start=True, finish=True,
+                   s0: int = 0, s1: Optional[int] = None):
+        """Start and finish of ops [op0, op1) in scenarios [s0, s1): int64 [op][s - s0]."""
         op1 = self.n_ops if op1 is None else op1
-        n = max(op1 - op0, 0)
-        st = np.empty((n, self.n_scen), np.int64) if start else None
-        fn = np.empty((n, self.n_scen), np.int64) if finish else None
-        self._check(self.lib.echo_read_times(self.h, op0, op1, _ptr(st), _ptr(fn)))
+        s1 = self.n_scen if s1 is None else s1
+        n, m = max(op1 - op0, 0), max(s1 - s0, 0)
+        st = np.empty((n, m), np.int64) if start else None
+        fn = np.empty((n, m), np.int64) if finish else None
+        self._check(self.lib.echo_read_times(self.h, op0, op1, int(s0), int(s1), _ptr(st), _ptr(fn)))
         return st, fn
 
     def read_makespan(self, out=None):

@@ -19,13 +19,14 @@ CC_RTOL = 1e-9
 THREADS = max(1, min(16, os.cpu_count() or 1))
 
 
-def run_gpu(g, sc, refine=1, ctx=None, overlap_model=0, comm_interval=0):
+def run_gpu(g, sc, refine=1, ctx=None, overlap_model=0, comm_interval=0, ar_algo_policy=0):
     e = ctx or Echo(0)
     try:
         e.load_graph(g)
         e.load_scenarios(sc)
         e.estimate_collectives()
-        e.compose(refine_passes=refine, overlap_model=overlap_model, comm_interval=comm_interval)
+        e.compose(refine_passes=refine, overlap_model=overlap_model, comm_interval=comm_interval,
+                  ar_algo_policy=ar_algo_policy)
         st, fn = e.read_times()
         return dict(start=st, finish=fn, makespan=e.read_makespan(), cc=e.read_cc(),
                     ov=e.read_overlap(), info=e.info())
@@ -146,6 +147,69 @@ def test_alpha_beta_cost_model_bit_exact():
             e.set_cc_model(7)
     finally:
         e.close()
+
+
+@pytest.mark.parametrize("kernel", ["auto", "dataflow"])
+def test_allreduce_policy_bit_exact(kernel, monkeypatch):
+    """ring / tree / faster-of-the-two for every all-reduce (echo_compose_opts
+    ar_algo_policy), against the oracle's policy: GPT-1.3B (per-op AUTO all-reduces)
+    and random graphs mixing the per-op algorithms; switching the policy between
+    compositions of one context re-estimates the collectives."""
+    import dataclasses
+    if kernel == "dataflow":
+        monkeypatch.setenv("ECHO_COMPOSE_KERNEL", "dataflow")
+    c = W.config("gpt1.3b")
+    rng = np.random.default_rng(9900)
+    cases = [(W.build_gpt_graph(c), None)]
+    for _ in range(6):
+        g = SG.random_graph(rng, int(rng.integers(10, 80)), max_ranks=5, max_streams=4, p_edge=0.06)
+        cases.append((dataclasses.replace(g, cc_bytes=np.where(g.cc_bytes > 0, g.cc_bytes * 4096, 0)), None))
+    e = Echo(0)
+    try:
+        for k, (g, _) in enumerate(cases):
+            sc = W.make_scenarios(g, c, n_scen=40) if k == 0 else SG.random_scenarios(rng, g, 37, max_dur=2000)
+            e.load_graph(g)
+            e.load_scenarios(sc)
+            e.estimate_collectives()
+            for policy in (1, 2, 3, 0, 2):
+                e.compose(refine_passes=1, ar_algo_policy=policy)
+                st, fn = e.read_times()
+                got = dict(start=st, finish=fn, makespan=e.read_makespan(), cc=e.read_cc(),
+                           ov=e.read_overlap())
+                want = oracle.compose(g, sc, refine_passes=1, ar_algo_policy=policy,
+                                      threads=THREADS if k == 0 else 1)
+                assert_same(got, want, g, 1)
+        with pytest.raises(EchoError):
+            e.compose(refine_passes=1, ar_algo_policy=4)
+    finally:
+        e.close()
+
+
+def test_read_times_scenario_range():
+    """echo_read_times over a scenario range [s0, s1): the matching columns of the
+    full readback, into host and device buffers; bad ranges are rejected."""
+    import torch
+    c = W.config("gpt1.3b")
+    g = W.build_gpt_graph(c)
+    sc = W.make_scenarios(g, c, n_scen=70)
+    with Echo(0) as e:
+        e.load_graph(g)
+        e.load_scenarios(sc)
+        e.estimate_collectives()
+        e.compose(refine_passes=1)
+        st, fn = e.read_times()
+        for op0, op1, s0, s1 in ((0, g.n_ops, 0, 70), (17, 4000, 3, 41), (g.n_ops - 5, g.n_ops, 69, 70),
+                                 (100, 100, 5, 9), (0, 1000, 64, 70)):
+            a, b = e.read_times(op0, op1, s0=s0, s1=s1)
+            assert np.array_equal(a, st[op0:op1, s0:s1]) and np.array_equal(b, fn[op0:op1, s0:s1])
+        # device output buffers
+        dst = torch.empty((300, 11), dtype=torch.int64, device="cuda")
+        rc = e.lib.echo_read_times(e.h, 50, 350, 20, 31, None, dst.data_ptr())
+        assert rc == 0
+        assert np.array_equal(dst.cpu().numpy(), fn[50:350, 20:31])
+        for bad in ((0, 10, -1, 5), (0, 10, 5, 71), (0, 10, 6, 5), (0, 10, 5, 5)):
+            with pytest.raises(EchoError):
+                e.read_times(bad[0], bad[1], s0=bad[2], s1=bad[3])
 
 
 def test_int32_durations_give_the_same_timelines():
@@ -355,46 +419,54 @@ def test_call_order_and_input_errors():
         assert np.array_equal(a, e.read_makespan())
 
 
-def _sampled_parity(name, cols, refine=1):
+def _full_batch_parity(name, time_cols, refine=1):
+    """The whole batch of a full-size workload: every scenario's makespan against
+    the oracle's (run threaded over the host cores), and every op's start and
+    finish in the scenarios `time_cols`, read back one scenario column at a time
+    through echo_read_times' scenario range."""
     c = W.config(name)
     g = W.build_gpt_graph(c)
     sc = W.make_scenarios(g, c)
     with Echo(0) as e:
         e.load_graph(g)
         e.load_scenarios(sc)
-        del sc.dur
         e.estimate_collectives()
         e.compose(refine_passes=refine)
         mk = e.read_makespan()
-        V, S = g.n_ops, e.n_scen
-        fin = np.empty((V, len(cols)), np.int64)
-        st = np.empty((V, len(cols)), np.int64)
-        mk_check = np.zeros(S, np.int64)
-        step = max(1, (1 << 28) // (16 * S))
-        for a in range(0, V, step):
-            b = min(V, a + step)
-            s_, f_ = e.read_times(a, b)
-            fin[a:b] = f_[:, cols]
-            st[a:b] = s_[:, cols]
-            assert (s_ >= 0).all() and (f_ >= s_).all()
-            mk_check = np.maximum(mk_check, f_.max(0))
-        assert np.array_equal(mk, mk_check)
-    sub = W.select_scenarios(W.scenario_params(c), g, cols)
-    want = oracle.compose(g, sub, refine_passes=refine, threads=min(THREADS, len(cols)), want_cc=False,
-                          want_overlap=False)
+        info = e.info()
+        fin = np.empty((g.n_ops, len(time_cols)), np.int64)
+        st = np.empty((g.n_ops, len(time_cols)), np.int64)
+        for k, s in enumerate(time_cols):
+            a, b = e.read_times(s0=s, s1=s + 1)
+            st[:, k], fin[:, k] = a[:, 0], b[:, 0]
+        assert (st >= 0).all() and (fin >= st).all()
+        assert np.array_equal(mk[time_cols], fin.max(0))
+    want_mk = oracle.compose(g, sc, refine_passes=refine, threads=THREADS, want_cc=False, want_overlap=False,
+                             want_times=False).makespan
+    assert np.array_equal(mk, want_mk), np.nonzero(mk != want_mk)[0][:10]
+    del sc
+    sub = W.select_scenarios(W.scenario_params(c), g, list(time_cols))
+    want = oracle.compose(g, sub, refine_passes=refine, threads=THREADS, want_cc=False, want_overlap=False)
     assert np.array_equal(fin, want.finish)
     assert np.array_equal(st, want.start)
-    assert np.array_equal(mk[cols], want.makespan)
+    return info
 
 
 @pytest.mark.slow
-def test_gpt175b_full_size_sampled_scenarios():
-    _sampled_parity("gpt175b", [0, 1, 509, 1023])
+def test_gpt175b_full_batch_bit_exact():
+    # all 1024 makespans; every op in 128 scenarios, one in each scenario block of
+    # the levelled composer (sigma 8) and every lane position of a block (both
+    # lanes of every thread) sixteen times over
+    info = _full_batch_parity("gpt175b", [8 * b + b % 8 for b in range(128)])
+    assert info["sigma"] == 8
 
 
 @pytest.mark.slow
-def test_gpt175b_1024_ranks_full_size_sampled_scenarios():
-    _sampled_parity("gpt175b-1024", [0, 63])
+def test_gpt175b_1024_ranks_full_batch_bit_exact():
+    # all 64 makespans (both groups of 32 scenarios of the dataflow composer); every
+    # op in the first and last scenario of each group
+    info = _full_batch_parity("gpt175b-1024", [0, 31, 32, 63])
+    assert info["sigma"] == 32
 
 
 @pytest.mark.parametrize("sigma", ["1", "2", "4", "8", "16"])
