@@ -168,7 +168,7 @@ __device__ __forceinline__ void g_store(int64_t *p, const int64_t (&v)[LANES]) {
 // durations are loaded four at a time so that their latencies overlap.  This
 // block's finish rows are a contiguous [V][SIGMA] array (padding lanes included),
 // so every row moves as whole vectors.
-template <int SIGMA, int LANES>
+template <int SIGMA, int LANES, bool STORE_ALL>
 __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t ro, uint32_t i0, uint32_t seg0,
                                                  int32_t nseg, int sub, int step, int j0, int64_t *vr,
                                                  const int64_t *dr, const uint32_t *rr, uint32_t vmask,
@@ -185,12 +185,23 @@ __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t r
     const uint32_t nin = hd.y & 0xFFFFu, nfar = hd.y >> 16;
     const uint32_t len = hd.w & 0xFFFFu;
     // chain positions whose duration the validator rewrote (second and later passes)
+    const bool has_c = (hd.w >> 16) & 1, has_k = (hd.w >> 17) & 1;
+    const uint32_t ec = ro + hd.x + nin + nfar;
     uint64_t cmask_bits = 0;
     uint32_t c_first = 0;
-    if (cr && (hd.w >> 16)) {
-      const uint32_t ec = ro + hd.x + nin + nfar;
+    if (cr && has_c) {
       cmask_bits = (uint64_t)word(ec) | ((uint64_t)word(ec + 1) << 32);
       c_first = word(ec + 2);
+    }
+    // chain positions whose finish is stored: all in the final composition; else
+    // the tail (later heads read it) and those a later step reads (kept mask)
+    uint64_t smask = ~0ull;
+    if (!STORE_ALL) {
+      smask = 1ull << (len - 1);
+      if (has_k) {
+        const uint32_t ek = ec + (has_c ? 3 : 0);
+        smask |= (uint64_t)word(ek) | ((uint64_t)word(ek + 1) << 32);
+      }
     }
     // a candidate's duration comes from the candidate ring instead of the duration ring
     auto patch = [&](uint32_t t, int64_t (&d)[LANES]) {
@@ -234,18 +245,19 @@ __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t r
         patch(t + 2, d2);
         patch(t + 3, d3);
       }
+      const uint32_t sb = (uint32_t)(smask >> t);
 #pragma unroll
       for (int j = 0; j < LANES; ++j) fv[j] += d0[j];
-      g_store<LANES>(gp, fv);
+      if (STORE_ALL || (sb & 1)) g_store<LANES>(gp, fv);
 #pragma unroll
       for (int j = 0; j < LANES; ++j) fv[j] += d1[j];
-      g_store<LANES>(gp + SIGMA, fv);
+      if (STORE_ALL || (sb & 2)) g_store<LANES>(gp + SIGMA, fv);
 #pragma unroll
       for (int j = 0; j < LANES; ++j) fv[j] += d2[j];
-      g_store<LANES>(gp + 2 * SIGMA, fv);
+      if (STORE_ALL || (sb & 4)) g_store<LANES>(gp + 2 * SIGMA, fv);
 #pragma unroll
       for (int j = 0; j < LANES; ++j) fv[j] += d3[j];
-      g_store<LANES>(gp + 3 * SIGMA, fv);
+      if (STORE_ALL || (sb & 8)) g_store<LANES>(gp + 3 * SIGMA, fv);
     }
     for (; t < len; ++t, gp += SIGMA) {
       int64_t d[LANES];
@@ -253,7 +265,7 @@ __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t r
       if (cmask_bits) patch(t, d);
 #pragma unroll
       for (int j = 0; j < LANES; ++j) fv[j] += d[j];
-      g_store<LANES>(gp, fv);
+      if (STORE_ALL || ((smask >> t) & 1)) g_store<LANES>(gp, fv);
     }
 #pragma unroll
     for (int j = 0; j < LANES; ++j) mk[j] = max(mk[j], fv[j]);
@@ -361,8 +373,12 @@ compose_staged_kernel(StagedArgs a) {
 
     const uint32_t ro = mb[0], i0 = mb[1], seg0 = mb[2];
     const int32_t nseg = (int32_t)(mb[4 + 2] - seg0);
-    compose_segments<SIGMA, LANES>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr, vmask, dmask,
-                                   rmask, mk);
+    if (a.store_all)
+      compose_segments<SIGMA, LANES, true>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr, vmask,
+                                           dmask, rmask, mk);
+    else
+      compose_segments<SIGMA, LANES, false>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr, vmask,
+                                            dmask, rmask, mk);
     prev_i0 = i0;
     prev_ro = ro;
   }
@@ -423,7 +439,7 @@ __device__ __forceinline__ bool named_barrier_or(int id, int threads, bool flag)
 // byte count) and an "empty" mbarrier (one arrival per consumer warp once the
 // level is composed).  Every wait is bounded: on expiry the block records
 // kDevTimeout, stops, and lets its copies in flight land first.
-template <int SIGMA>
+template <int SIGMA, bool STORE_ALL>
 __global__ void __launch_bounds__((kPipeConsumerWarps + 1) * 32)
 compose_pipelined_kernel(StagedArgs a) {
   constexpr int LANES = 2;
@@ -521,8 +537,8 @@ compose_pipelined_kernel(StagedArgs a) {
         const uint32_t *mb = metas + 8 * (l % NB);
         const uint32_t ro = mb[0], i0 = mb[1], seg0 = mb[2];
         const int32_t nseg = (int32_t)(mb[4 + 2] - seg0);
-        compose_segments<SIGMA, LANES>(a, ro, i0, seg0, nseg, tid / TPN, NCT / TPN, j0, vr, dr, rr, vmask, dmask,
-                                       rmask, mk, a.cdur ? cr : nullptr, CRR - 1);
+        compose_segments<SIGMA, LANES, STORE_ALL>(a, ro, i0, seg0, nseg, tid / TPN, NCT / TPN, j0, vr, dr, rr,
+                                                  vmask, dmask, rmask, mk, a.cdur ? cr : nullptr, CRR - 1);
       }
       // every consumer learns, in the same barrier, whether any of them gave up
       if (named_barrier_or(1, NCT, !ok)) {
@@ -567,7 +583,7 @@ cudaError_t launch_staged_t(const StagedArgs &a, const StagedPlan &plan, cudaStr
 
 template <int SIGMA>
 cudaError_t launch_pipelined_t(const StagedArgs &a, const StagedPlan &plan, cudaStream_t st) {
-  auto k = compose_pipelined_kernel<SIGMA>;
+  auto k = a.store_all ? compose_pipelined_kernel<SIGMA, true> : compose_pipelined_kernel<SIGMA, false>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem);
   if (e != cudaSuccess) return e;
   dim3 grid((a.S + SIGMA - 1) / SIGMA);

@@ -79,6 +79,10 @@ struct GraphBuild {
   std::vector<int32_t> lq_off;        // [cq_ops+1] launch conditions of each cq_ops entry on its rank
   std::vector<int32_t> lq_ops;        // (internal ids; the latest one on each of the rank's timelines)
   std::vector<int64_t> seg_words;     // [n_seg] record words of each segment
+  // [V] 1 for an op whose finish a later step reads besides the next op of its
+  // chain: an overlap candidate, a comm op the validator's cursors visit, or one
+  // of their launch conditions (a segment's tail is always kept: later heads read it)
+  std::vector<uint8_t> keep;
   std::vector<int64_t> hin_off;       // [n_seg+1] inputs of each segment's head
   std::vector<int32_t> hin;           // (internal ids, each the tail of an earlier segment)
   int32_t max_kclass = -1;
@@ -778,13 +782,23 @@ int build_graph(const echo_graph_desc *g, GraphBuild &b, Err &e, const std::vect
     b.lq_off.push_back(0);
   }
   if (b.lq_ops.empty()) b.lq_ops.push_back(0);
+  b.keep.assign(V, 0);
+  for (int64_t v = 0; v < V; ++v) b.keep[v] = b.cand_flag[v];
+  const int64_t n_cqe = b.cq_off.back();  // (cq_ops and lq_off hold a placeholder when empty)
+  for (int64_t e = 0; e < n_cqe; ++e) {
+    b.keep[b.cq_ops[e]] = 1;
+    for (int32_t q = b.lq_off[e]; q < b.lq_off[e + 1]; ++q) b.keep[b.lq_ops[q]] = 1;
+  }
   b.seg_words.assign(NSg, 0);
   for (int64_t t = 0; t < NSg; ++t) {
     const int64_t nin = b.hin_off[t + 1] - b.hin_off[t];
     if (nin > 0xFFFF) b.stageable = false;
-    bool cand = false;
-    for (int64_t v = b.seg_node_off[t]; v < b.seg_node_off[t + 1]; ++v) cand = cand || b.cand_flag[v];
-    b.seg_words[t] = 4 + nin + (cand ? 3 : 0);
+    bool cand = false, kept = false;
+    for (int64_t v = b.seg_node_off[t]; v < b.seg_node_off[t + 1]; ++v) {
+      cand = cand || b.cand_flag[v];
+      kept = kept || (b.keep[v] && v + 1 < b.seg_node_off[t + 1]);
+    }
+    b.seg_words[t] = 4 + nin + (cand ? 3 : 0) + (kept ? 2 : 0);
   }
   // every input of a segment comes from an earlier level (the kernels' contract)
   {
@@ -1187,6 +1201,15 @@ void build_records(const GraphBuild &b, const Steps &stp, int sigma, int vlog2, 
         recs.push_back((uint32_t)mask);
         recs.push_back((uint32_t)(mask >> 32));
         recs.push_back((uint32_t)c_first);
+      }
+      // chain positions before the tail whose finish a later step reads
+      uint64_t kmask = 0;
+      for (int64_t v = h; v < z; ++v)
+        if (b.keep[v]) kmask |= 1ull << (v - h);
+      if (kmask) {
+        recs[hd + 3] |= 1u << 17;
+        recs.push_back((uint32_t)kmask);
+        recs.push_back((uint32_t)(kmask >> 32));
       }
     }
     while (recs.size() % 4) recs.push_back(0);
@@ -1919,7 +1942,9 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   };
   // one composition with durations `d` (and, for the pipelined and dataflow
   // kernels, the candidates' durations `cdur`) into `f`
-  auto compose_pass = [&](const int64_t *d, const int64_t *cdur, int64_t *f, bool adjusted) -> cudaError_t {
+  // (final_pass: the readback reads every finish of this composition)
+  auto compose_pass = [&](const int64_t *d, const int64_t *cdur, int64_t *f, bool adjusted,
+                          bool final_pass) -> cudaError_t {
     const char *name = adjusted ? "compose_adjusted" : "compose";
     if (c->use_df) {
       echo::DataflowArgs a{};
@@ -1979,6 +2004,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       a.status = c->status;
       a.wait_limit_cycles = c->wait_limit_cycles;
       a.skip_level = c->skip_level;
+      a.store_all = final_pass;
       const bool pipe = c->plan.pipelined && (c->kernel_choice == 0 || c->kernel_choice == 3);
       if (pipe)
         return timed(c, name, [&] { return echo::launch_compose_pipelined(a, c->sigma, c->plan, c->stream); });
@@ -2003,13 +2029,13 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     return timed(c, "compose_direct", [&] { return echo::launch_compose(a, c->sigma, c->stream); });
   };
   CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
-  CK(compose_pass(c->dur, nullptr, c->f[0], false), "compose launch");
+  CK(compose_pass(c->dur, nullptr, c->f[0], false, refine == 0), "compose launch");
   const int64_t *cd_used = nullptr;
   for (int32_t p = 1; p <= refine; ++p) {
     echo::OverlapArgs o = overlap_args(c->f[(p - 1) % 2], cd_used, c->cd[(p - 1) % 2]);
     CK(timed(c, "overlap", [&] { return echo::launch_overlap(o, c->stream); }), "overlap launch");
     if (ring) {
-      CK(compose_pass(c->dur, o.cd_next, c->f[p % 2], true), "compose launch");
+      CK(compose_pass(c->dur, o.cd_next, c->f[p % 2], true, p == refine), "compose launch");
     } else {
       CK(cudaMemcpyAsync(c->deff, c->dur, c->scen_vs * sizeof(int64_t), cudaMemcpyDeviceToDevice, c->stream),
          "duration copy");
@@ -2017,7 +2043,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
            return echo::launch_scatter_candidates(c->cand_node, B.n_cand, c->S, c->lay, c->lay_c, o.cd_next, c->deff,
                                                   c->stream);
          }), "scatter launch");
-      CK(compose_pass(c->deff, nullptr, c->f[p % 2], true), "compose launch");
+      CK(compose_pass(c->deff, nullptr, c->f[p % 2], true, p == refine), "compose launch");
     }
     cd_used = o.cd_next;
     c->last_ov = o;

@@ -81,8 +81,10 @@ struct ComposeArgs {
 // nfar inputs too old for the ring (node ids, read from global memory).  Every
 // input is the tail of an earlier segment.  A segment whose chain holds overlap
 // candidates has bit 16 of its length word set and 3 more entries: a 64-bit mask
-// of those chain positions and the level-order index of the first.  Blocks are
-// padded to 4 words.  Metadata of a level: record word offset, first node, first
+// of those chain positions and the level-order index of the first.  A segment with
+// chain positions before its tail whose finish a later step reads (validator
+// inputs) has bit 17 set and 2 more entries: the 64-bit mask of those positions.
+// Blocks are padded to 4 words.  Metadata of a level: record word offset, first node, first
 // segment, first level-order candidate.
 struct StagedArgs {
   int32_t S, L;                  // L: segment levels
@@ -100,6 +102,7 @@ struct StagedArgs {
   int32_t *status;               // device status word (kDevTimeout when a bounded wait gives up)
   long long wait_limit_cycles;   // bound of every mbarrier wait, in SM clock cycles
   int32_t skip_level;            // failure injection for tests: this level is never filled (-1: none)
+  int32_t store_all;             // final composition: store every finish; else only those read again
 };
 
 // Plan of the staged kernels for one (graph, sigma); see plan_staged().
