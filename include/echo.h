@@ -51,7 +51,8 @@ typedef enum {
   ECHO_E_CUDA = 6,        /* a CUDA runtime call failed                                */
   ECHO_E_TIMEOUT = 7,     /* a bounded device-side wait gave up                        */
   ECHO_E_OVERFLOW = 8,    /* a finish time could exceed the int64 range                */
-  ECHO_E_UNSUPPORTED = 9  /* a size beyond what the library supports                   */
+  ECHO_E_UNSUPPORTED = 9, /* a size beyond what the library supports                   */
+  ECHO_E_BOUNDS = 10      /* a device-side index check failed (debug_bounds)           */
 } echo_status;
 
 /* op kinds (Sec. 4.2 timelines: computation, communication, memcpy) */
@@ -174,6 +175,13 @@ typedef struct {
    * runs the CC estimator again first (ECHO_E_OVERFLOW as there), and echo_read_cc
    * then reports those estimates. */
   int32_t ar_algo_policy;
+  /* nonzero: every index the composition and validator kernels gather through (from
+   * the graph's records, programs and candidate and comm lists) is checked on the
+   * device against the bounds of the buffer it indexes before the access; a failed
+   * check skips the access, stops the kernel's walk and makes the next echo_read_*
+   * return ECHO_E_BOUNDS.  Never traps.  For debugging; slower.  The environment
+   * variable ECHO_DEBUG_BOUNDS=1 turns it on for every composition. */
+  int32_t debug_bounds;
 } echo_compose_opts;
 enum { ECHO_OVERLAP_WHOLE = 0, ECHO_OVERLAP_PROPORTIONAL = 1 };
 enum { ECHO_COMM_EXECUTION = 0, ECHO_COMM_LAUNCH = 1 };

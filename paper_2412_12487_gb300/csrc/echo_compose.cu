@@ -51,14 +51,39 @@ compose_direct_kernel(ComposeArgs a) {
     if (active) {
       for (int64_t t = t0 + sub; t < t1; t += stride) {
         const int64_t h = a.seg_node_off[t], z = a.seg_node_off[t + 1] - 1;
+        if (a.dbg && !(range_ok(h, z + 1, a.V) && h <= z)) {  // debug bounds: skip a bad segment
+          atomicCAS(a.status, 0, (int32_t)kDevBounds);
+          continue;
+        }
         int64_t fv = 0;  // the head starts after its timelines and data predecessors
-        for (int64_t k = a.nq_off[h]; k < a.nq_off[h + 1]; ++k) fv = max(fv, fr[(int64_t)a.nq[k] * SIGMA + j]);
-        for (int64_t k = a.dp_off[h]; k < a.dp_off[h + 1]; ++k) fv = max(fv, f[a.lay.at(a.dp[k], s)]);
+        for (int64_t k = a.nq_off[h]; k < a.nq_off[h + 1]; ++k) {
+          const int64_t q = a.nq[k];
+          if (a.dbg && !in_range(q, a.n_queues)) {
+            atomicCAS(a.status, 0, (int32_t)kDevBounds);
+            continue;
+          }
+          fv = max(fv, fr[q * SIGMA + j]);
+        }
+        for (int64_t k = a.dp_off[h]; k < a.dp_off[h + 1]; ++k) {
+          const int64_t u = a.dp[k];
+          if (a.dbg && !in_range(u, a.V)) {
+            atomicCAS(a.status, 0, (int32_t)kDevBounds);
+            continue;
+          }
+          fv = max(fv, f[a.lay.at(u, s)]);
+        }
         for (int64_t i = h; i <= z; ++i) {  // along the chain every op starts when the previous ends
           fv += dur[a.lay.at(i, s)];
           f[a.lay.at(i, s)] = fv;
         }
-        for (int64_t k = a.nq_off[z]; k < a.nq_off[z + 1]; ++k) fr[(int64_t)a.nq[k] * SIGMA + j] = fv;
+        for (int64_t k = a.nq_off[z]; k < a.nq_off[z + 1]; ++k) {
+          const int64_t q = a.nq[k];
+          if (a.dbg && !in_range(q, a.n_queues)) {
+            atomicCAS(a.status, 0, (int32_t)kDevBounds);
+            continue;
+          }
+          fr[q * SIGMA + j] = fv;
+        }
         mk = max(mk, fv);
       }
     }
@@ -157,6 +182,22 @@ __device__ __forceinline__ void g_store(int64_t *p, const int64_t (&v)[LANES]) {
     *p = v[0];
 }
 
+// Debug bounds (out of line, off the hot path): the segment's chain rows, its
+// candidates' compact rows, every input's value-ring slot and far row.  A failed
+// check records kDevBounds.
+__device__ __noinline__ bool segment_ok(const StagedArgs &a, uint32_t first, uint32_t len, uint64_t cmask,
+                                        uint32_t c_first, uint32_t rr_a, uint32_t rmask, uint32_t e, uint32_t nin,
+                                        uint32_t nfar, uint32_t ring_bytes, uint32_t row_bytes) {
+  bool ok = len > 0 && range_ok(first, (int64_t)first + len, a.n_rows) && masked_row_ok(c_first, cmask, a.n_cand);
+  for (uint32_t x = 0; ok && x < nin + nfar; ++x) {
+    uint32_t w;
+    asm volatile("ld.shared.u32 %0, [%1];\n" : "=r"(w) : "r"(rr_a + ((e + x) & rmask) * 4));
+    ok = x < nin ? (w < ring_bytes && w % row_bytes == 0) : in_range(w, a.n_rows);
+  }
+  if (!ok) atomicCAS(a.status, 0, (int32_t)kDevBounds);
+  return ok;
+}
+
 // Compose the segments of one segment level (shared by the staged and the
 // pipelined kernels).  Segment k's header and entries are in the record ring at
 // word `ro`; its rows are i0 + header.z ... in the duration ring.  Thread `sub`
@@ -168,7 +209,7 @@ __device__ __forceinline__ void g_store(int64_t *p, const int64_t (&v)[LANES]) {
 // durations are loaded four at a time so that their latencies overlap.  This
 // block's finish rows are a contiguous [V][SIGMA] array (padding lanes included),
 // so every row moves as whole vectors.
-template <int SIGMA, int LANES, bool STORE_ALL>
+template <int SIGMA, int LANES, bool STORE_ALL, bool DBG>
 __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t ro, uint32_t i0, uint32_t seg0,
                                                  int32_t nseg, int sub, int step, int j0, int64_t *vr,
                                                  const int64_t *dr, const uint32_t *rr, uint32_t vmask,
@@ -210,6 +251,9 @@ __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t r
     };
     const uint32_t e = ro + hd.x;
     const uint32_t first = i0 + hd.z;
+    if (DBG && !segment_ok(a, first, len, cmask_bits, c_first, rr_a, rmask, e, nin, nfar, (vmask + 1) * kRowBytes,
+                             kRowBytes))
+      continue;  // debug bounds: a bad index skips the segment
     int64_t fv[LANES];
 #pragma unroll
     for (int j = 0; j < LANES; ++j) fv[j] = 0;
@@ -373,12 +417,15 @@ compose_staged_kernel(StagedArgs a) {
 
     const uint32_t ro = mb[0], i0 = mb[1], seg0 = mb[2];
     const int32_t nseg = (int32_t)(mb[4 + 2] - seg0);
-    if (a.store_all)
-      compose_segments<SIGMA, LANES, true>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr, vmask,
-                                           dmask, rmask, mk);
+    if (a.dbg)
+      compose_segments<SIGMA, LANES, true, true>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr,
+                                                 vmask, dmask, rmask, mk);
+    else if (a.store_all)
+      compose_segments<SIGMA, LANES, true, false>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr,
+                                                  vmask, dmask, rmask, mk);
     else
-      compose_segments<SIGMA, LANES, false>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr, vmask,
-                                            dmask, rmask, mk);
+      compose_segments<SIGMA, LANES, false, false>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr,
+                                                   vmask, dmask, rmask, mk);
     prev_i0 = i0;
     prev_ro = ro;
   }
@@ -439,7 +486,7 @@ __device__ __forceinline__ bool named_barrier_or(int id, int threads, bool flag)
 // byte count) and an "empty" mbarrier (one arrival per consumer warp once the
 // level is composed).  Every wait is bounded: on expiry the block records
 // kDevTimeout, stops, and lets its copies in flight land first.
-template <int SIGMA, bool STORE_ALL>
+template <int SIGMA, bool STORE_ALL, bool DBG>
 __global__ void __launch_bounds__((kPipeConsumerWarps + 1) * 32)
 compose_pipelined_kernel(StagedArgs a) {
   constexpr int LANES = 2;
@@ -488,8 +535,14 @@ compose_pipelined_kernel(StagedArgs a) {
         if (l == a.skip_level) break;  // failure injection: level l never arrives
         const uint4 m0 = *reinterpret_cast<const uint4 *>(a.meta + 4 * l);
         const uint4 m1 = *reinterpret_cast<const uint4 *>(a.meta + 4 * (l + 1));
-        const uint32_t ro = m0.x, i0 = m0.y, ro1 = m1.x, i1 = m1.y;
-        const uint32_t c0 = cdb ? m0.w : 0, c1 = cdb ? m1.w : 0;  // the level's candidate rows
+        uint32_t ro = m0.x, i0 = m0.y, ro1 = m1.x, i1 = m1.y;
+        uint32_t c0 = cdb ? m0.w : 0, c1 = cdb ? m1.w : 0;  // the level's candidate rows
+        if (DBG && !(range_ok(i0, i1, a.n_rows) && range_ok(ro, ro1, a.n_words) && range_ok(c0, c1, a.n_cand))) {
+          atomicCAS(a.status, 0, (int32_t)kDevBounds);  // debug bounds: copy nothing for this level
+          i1 = i0 = min(i0, a.n_rows);
+          ro1 = ro = min(ro, a.n_words);
+          c1 = c0 = min(c0, a.n_cand);
+        }
         // ring space: level l overwrites rows and words of levels below c_known only
         while (c_known < l && (l - c_known >= NB || i1 > hist[4 * (c_known % NB)] + RR ||
                                ro1 > hist[4 * (c_known % NB) + 1] + RB || c1 > hist[4 * (c_known % NB) + 2] + CRR)) {
@@ -537,8 +590,8 @@ compose_pipelined_kernel(StagedArgs a) {
         const uint32_t *mb = metas + 8 * (l % NB);
         const uint32_t ro = mb[0], i0 = mb[1], seg0 = mb[2];
         const int32_t nseg = (int32_t)(mb[4 + 2] - seg0);
-        compose_segments<SIGMA, LANES, STORE_ALL>(a, ro, i0, seg0, nseg, tid / TPN, NCT / TPN, j0, vr, dr, rr,
-                                                  vmask, dmask, rmask, mk, a.cdur ? cr : nullptr, CRR - 1);
+        compose_segments<SIGMA, LANES, STORE_ALL, DBG>(a, ro, i0, seg0, nseg, tid / TPN, NCT / TPN, j0, vr, dr,
+                                                       rr, vmask, dmask, rmask, mk, a.cdur ? cr : nullptr, CRR - 1);
       }
       // every consumer learns, in the same barrier, whether any of them gave up
       if (named_barrier_or(1, NCT, !ok)) {
@@ -583,7 +636,9 @@ cudaError_t launch_staged_t(const StagedArgs &a, const StagedPlan &plan, cudaStr
 
 template <int SIGMA>
 cudaError_t launch_pipelined_t(const StagedArgs &a, const StagedPlan &plan, cudaStream_t st) {
-  auto k = a.store_all ? compose_pipelined_kernel<SIGMA, true> : compose_pipelined_kernel<SIGMA, false>;
+  // debug bounds runs the checking variant, which stores every finish
+  auto k = a.dbg ? compose_pipelined_kernel<SIGMA, true, true>
+                 : a.store_all ? compose_pipelined_kernel<SIGMA, true, false> : compose_pipelined_kernel<SIGMA, false, false>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem);
   if (e != cudaSuccess) return e;
   dim3 grid((a.S + SIGMA - 1) / SIGMA);

@@ -27,6 +27,7 @@
 #include <cstdint>
 
 #include "echo_internal.h"
+#include "echo_bounds.h"
 
 namespace echo {
 namespace {
@@ -85,6 +86,36 @@ __device__ bool df_gather(const uint64_t *p, uint32_t n, uint32_t skip, uint64_t
   return true;
 }
 
+// Debug bounds: every index the batch of program entries [b, b + 8) will use (its
+// nodes, candidate rows, other-input words and their payloads, partial slots,
+// export ids, timelines) lies in its buffer (echo_bounds.h).  w holds the batch's
+// record words as loaded by the warp (lane l: words 2(l % 4), 2(l % 4) + 1 of
+// entry l / 4).  Uniform over the warp.
+__device__ __noinline__ bool df_batch_ok(uint2 w, int64_t b, int64_t e1, bool cand, const DataflowArgs &a) {
+  bool ok = true;
+  for (int j = 0; j < kDfBatch; ++j) {
+    const uint32_t v = __shfl_sync(0xffffffffu, w.x, 4 * j), ci = __shfl_sync(0xffffffffu, w.y, 4 * j);
+    const uint32_t hdr = __shfl_sync(0xffffffffu, w.x, 4 * j + 1), oo = __shfl_sync(0xffffffffu, w.y, 4 * j + 1);
+    const uint32_t slot = __shfl_sync(0xffffffffu, w.x, 4 * j + 2), nmme = __shfl_sync(0xffffffffu, w.y, 4 * j + 2);
+    const uint32_t xid = __shfl_sync(0xffffffffu, w.x, 4 * j + 3);
+    if (b + j >= e1) break;
+    ok &= in_range(v, a.V) && (!cand || ci == ~0u || in_range(ci, a.n_cand));
+    ok &= in_range(hdr & 15, a.n_streams) && ((hdr >> 16) >> a.n_streams) == 0;
+    const uint32_t n_extra = (hdr >> 8) & 0xFF;
+    ok &= range_ok(oo, (int64_t)oo + n_extra, a.n_opnd);
+    for (uint32_t i = 0; ok && i < n_extra; ++i) {
+      const uint32_t x = __ldg(&a.opnd[oo + i]), p = x & kDfPayload;
+      ok &= (x >> 30) == kDfInLocal ? in_range(p, a.V) : (x >> 30) == kDfInRemote && in_range(p, a.n_exports);
+    }
+    if (hdr & kDfComm) {
+      const uint32_t nm = nmme & 0xFFFF, me = nmme >> 16;
+      ok &= nm <= 1 || (me < nm && range_ok(slot, (int64_t)slot + nm, a.n_slots));
+    }
+    if (hdr & (kDfExport | kDfTwoHop)) ok &= in_range(xid, a.n_exports);
+  }
+  return ok;
+}
+
 __device__ __forceinline__ void cp_async_8(void *smem, const void *gmem) {
   const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
   asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(sa), "l"(gmem) : "memory");
@@ -131,12 +162,25 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
   };
   static_assert(kDfDepth == 3, "the record registers below hold kDfDepth + 1 batches");
   uint2 w0 = rec(e0), w1 = rec(e0 + kDfBatch), w2 = rec(e0 + 2 * kDfBatch), w3 = rec(e0 + 3 * kDfBatch);
+  // debug bounds: a batch is checked before its durations are copied; a bad index
+  // stops this warp (its copies land first) and, through the abort flag, the others
+  auto bad_batch = [&](int64_t bb, uint2 w) {
+    if (!a.dbg || df_batch_ok(w, bb, e1, CAND, a)) return false;
+    if (lane == 0) {
+      atomicCAS(a.status, (int32_t)kDevOk, (int32_t)kDevBounds);
+      atomicExch(a.abort_flag, 1);
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    return true;
+  };
+  if (bad_batch(e0, w0) || bad_batch(e0 + kDfBatch, w1) || bad_batch(e0 + 2 * kDfBatch, w2)) return;
   durs(e0, w0);
   durs(e0 + kDfBatch, w1);
   durs(e0 + 2 * kDfBatch, w2);
   int64_t cur = 0;  // finish of the previous op of the program
   for (int64_t b = e0; b < e1; b += kDfBatch) {
     const uint2 w4 = rec(b + 4 * kDfBatch);
+    if (bad_batch(b + 3 * kDfBatch, w3)) return;
     durs(b + 3 * kDfBatch, w3);
     asm volatile("cp.async.wait_group 3;" ::: "memory");  // this batch's group is complete
     const int64_t *d0 = dring + ((b - e0) / kDfBatch % (kDfDepth + 1)) * (kDfBatch * 32) + lane;

@@ -1509,6 +1509,7 @@ const char *echo_strerror(int s) {
     case ECHO_E_CUDA: return "CUDA error";
     case ECHO_E_TIMEOUT: return "device wait timed out";
     case ECHO_E_OVERFLOW: return "time overflow";
+    case ECHO_E_BOUNDS: return "a device-side index check failed";
     case ECHO_E_UNSUPPORTED: return "unsupported size";
     default: return "unknown status";
   }
@@ -1894,6 +1895,8 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
   if (policy < ECHO_AR_PER_OP || policy > ECHO_AR_AUTO)
     return set_err(c, ECHO_E_INVALID_ARG, "unknown all-reduce policy");
   if (policy != c->est_policy && (rc = run_estimate(c, policy))) return rc;
+  const char *dbg_env = std::getenv("ECHO_DEBUG_BOUNDS");
+  const int32_t dbg = (opts && opts->debug_bounds) || (dbg_env && std::atoi(dbg_env) != 0) ? 1 : 0;
   const GraphBuild &B = c->gb;
   // the pipelined and dataflow kernels read the validator's durations of the
   // candidates (compact rows); the others compose from a full matrix built for them
@@ -1938,6 +1941,9 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     o.model = model;
     o.cd_next = cd_next;
     o.ov = nullptr;  // the decisions are recomputed on demand by echo_read_overlap
+    o.n_kclass = c->C;
+    o.dbg = dbg;
+    o.status = c->status;
     return o;
   };
   // one composition with durations `d` (and, for the pipelined and dataflow
@@ -1979,6 +1985,8 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       a.status = c->status;
       a.wait_limit_cycles = c->wait_limit_cycles;
       a.skip_slot = c->skip_level;
+      a.n_opnd = (int64_t)B.df_opnd.size();
+      a.dbg = dbg;
       if ((err = cudaMemsetAsync(c->mk, 0, (size_t)c->S * sizeof(int64_t), c->stream)) != cudaSuccess ||
           (err = cudaMemsetAsync(c->df_abort, 0, sizeof(int32_t), c->stream)) != cudaSuccess)
         return err;
@@ -2005,6 +2013,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       a.wait_limit_cycles = c->wait_limit_cycles;
       a.skip_level = c->skip_level;
       a.store_all = final_pass;
+      a.dbg = dbg;
       const bool pipe = c->plan.pipelined && (c->kernel_choice == 0 || c->kernel_choice == 3);
       if (pipe)
         return timed(c, name, [&] { return echo::launch_compose_pipelined(a, c->sigma, c->plan, c->stream); });
@@ -2026,6 +2035,8 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     a.f = f;
     a.makespan = c->mk;
     a.gfrontier = c->gfrontier;
+    a.dbg = dbg;
+    a.status = c->status;
     return timed(c, "compose_direct", [&] { return echo::launch_compose(a, c->sigma, c->stream); });
   };
   CK(cudaMemsetAsync(c->status, 0, sizeof(int32_t), c->stream), "memset");
@@ -2077,6 +2088,7 @@ static int composition_status(echo_ctx *c) {
     }
     return set_err(c, ECHO_E_TIMEOUT, "a device-side wait of the composer gave up");
   }
+  if (st == echo::kDevBounds) return set_err(c, ECHO_E_BOUNDS, "a debug-bounds index check failed on the device");
   return ECHO_OK;
 }
 

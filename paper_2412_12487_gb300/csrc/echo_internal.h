@@ -5,6 +5,8 @@
 
 #include <cstdint>
 
+#include "echo_bounds.h"
+
 namespace echo {
 
 constexpr int kMaxStreams = 16;
@@ -22,7 +24,10 @@ constexpr int kPipeStages = 16;            // stages (mbarrier pairs) of the pip
 constexpr int kPipeConsumerWarps = 16;     // composing warps of the pipelined compose
 
 // device status word: first error wins
-enum DeviceStatus : int32_t { kDevOk = 0, kDevNegativeDuration = 1, kDevCcOverflow = 2, kDevTimeout = 3 };
+enum DeviceStatus : int32_t {
+  kDevOk = 0, kDevNegativeDuration = 1, kDevCcOverflow = 2, kDevTimeout = 3,
+  kDevBounds = 4  // a debug-bounds index check failed (echo_bounds.h)
+};
 
 // Device layout of every [op][scenario] matrix (durations, finish times, validator
 // outputs): scenario blocks of 2^slog2 scenarios, block b holding a contiguous
@@ -71,6 +76,8 @@ struct ComposeArgs {
   int64_t *f;                                 // finish times (MatLayout, out)
   int64_t *makespan;                          // [S] (out)
   int64_t *gfrontier;                         // [grid][n_queues][sigma] when not in smem
+  int32_t dbg;                                // debug bounds: check every index (echo_bounds.h)
+  int32_t *status;
 };
 
 // Staged and pipelined compose: per-segment-level records and duration rows are
@@ -103,6 +110,7 @@ struct StagedArgs {
   long long wait_limit_cycles;   // bound of every mbarrier wait, in SM clock cycles
   int32_t skip_level;            // failure injection for tests: this level is never filled (-1: none)
   int32_t store_all;             // final composition: store every finish; else only those read again
+  int32_t dbg;                   // debug bounds: check every index (echo_bounds.h)
 };
 
 // Plan of the staged kernels for one (graph, sigma); see plan_staged().
@@ -157,6 +165,9 @@ struct OverlapArgs {
   int32_t model;           // 0: d * factor; 1: d + (factor - 1) * overlapped length
   int64_t *cd_next;        // (out, compact; may be null) candidates' durations for the next pass
   uint8_t *ov;             // (out, [V][S] rows of the candidates; may be null)
+  int32_t n_kclass;        // rows of sf
+  int32_t dbg;             // debug bounds: check every index (echo_bounds.h)
+  int32_t *status;
 };
 
 // Dataflow composer (echo_dataflow.cu): one warp per (rank, group of 32
@@ -199,6 +210,8 @@ struct DataflowArgs {
   int32_t *status;
   long long wait_limit_cycles;
   int64_t skip_slot;           // failure injection for tests: this partial is never published (-1: none)
+  int64_t n_opnd;              // words of opnd
+  int32_t dbg;                 // debug bounds: check every index (echo_bounds.h)
 };
 cudaError_t launch_compose_dataflow(const DataflowArgs &a, cudaStream_t st);
 size_t dataflow_smem_bytes(int32_t n_streams);

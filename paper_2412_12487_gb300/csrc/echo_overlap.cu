@@ -7,6 +7,7 @@
 #include <cstdint>
 
 #include "echo_internal.h"
+#include "echo_bounds.h"
 #include "echo_slowdown.cuh"
 
 #if !defined(ECHO_OV_LAUNCH) || !defined(ECHO_OV_PROP)
@@ -29,6 +30,13 @@ __device__ __forceinline__ void cp_async8(void *dst, const void *src) {
 
 // When rank r launched the comm op of cq entry e: the latest finish among its
 // launch conditions on r (out of line: the cursor loads are unrolled many times).
+// debug bounds: the launch conditions of cq entry e are nodes of the graph
+__device__ __noinline__ bool lq_ok(const OverlapArgs &a, int32_t e) {
+  bool ok = true;
+  for (int32_t k = a.lq_off[e]; k < a.lq_off[e + 1]; ++k) ok &= in_range(a.lq_ops[k], a.lay.V);
+  return ok;
+}
+
 __device__ __noinline__ int64_t launch_time(const int32_t *__restrict__ lq_off, const int32_t *__restrict__ lq_ops,
                                             const int64_t *__restrict__ f, int sh, int32_t e) {
   int64_t t = 0;
@@ -94,6 +102,11 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
   auto load = [&](int j) {
     if (cur[j] < end[j]) {
       const int64_t w = a.cq_ops[cur[j]];
+      if (a.dbg && !(in_range(w, a.lay.V) && (!LAUNCH || lq_ok(a, cur[j])))) {  // debug bounds
+        atomicCAS(a.status, 0, (int32_t)kDevBounds);
+        sw[j] = fw[j] = INT64_MAX;
+        return;
+      }
       fw[j] = f[w << sh];
       if (LAUNCH) {  // from the rank's launch: its launch conditions' latest finish
         sw[j] = launch_time(a.lq_off, a.lq_ops, f, sh, cur[j]);
@@ -108,6 +121,10 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
     int64_t sv0 = 0;  // the piece's first candidate's start (only for a search)
     if (part > 0) {
       const int64_t v = a.cand_ops[c0], ci = a.cand_cidx[c0];
+      if (a.dbg && !(in_range(v, a.lay.V) && in_range(ci, a.lay_c.V))) {  // debug bounds
+        if (lane == 0) atomicCAS(a.status, 0, (int32_t)kDevBounds);
+        return;
+      }
       sv0 = f[v << sh] - (cu ? cu[ci << sh] : du[v << sh]);
     }
 #pragma unroll
@@ -120,6 +137,10 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
         if (part > 0) {
           while (lo < hi) {  // first comm op finishing after sv0 (finishes are sorted)
             const int32_t mid = (lo + hi) >> 1;
+            if (a.dbg && !in_range(a.cq_ops[mid], a.lay.V)) {  // debug bounds: stop searching
+              atomicCAS(a.status, 0, (int32_t)kDevBounds);
+              break;
+            }
             if (f[(int64_t)a.cq_ops[mid] << sh] > sv0)
               hi = mid;
             else
@@ -158,6 +179,12 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
     kc = in ? a.cand_kcl[i] : 0;
   };
   // the batch's finish times and durations (those of the pass that produced f)
+  // debug bounds: a batch's nodes, compact rows and kernel classes, before its copies
+  auto batch_ok = [&](int64_t i0, int32_t q, int32_t cx, int32_t kc) {
+    const int64_t i = i0 + (lane & (kOvBatch - 1));
+    const bool ok = i >= c1 || (in_range(q, a.lay.V) && in_range(cx, a.lay_c.V) && in_range(kc, a.n_kclass));
+    return __all_sync(0xffffffffu, ok);
+  };
   auto issue = [&](int64_t i0, int32_t q, int32_t cx) {
     int64_t *slot = ring + ((i0 - c0) / kOvBatch % kOvDepth) * (kOvBatch * 2 * 32);
 #pragma unroll
@@ -175,10 +202,19 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
   ids(c0, q0, x0, k0);
   ids(c0 + kOvBatch, q1, x1, k1);
   ids(c0 + 2 * kOvBatch, q2, x2, k2);
+  const bool dbg_bad = a.dbg && !(batch_ok(c0, q0, x0, k0) && batch_ok(c0 + kOvBatch, q1, x1, k1));
+  if (dbg_bad) {
+    if (lane == 0) atomicCAS(a.status, 0, (int32_t)kDevBounds);
+    return;
+  }
   issue(c0, q0, x0);
   issue(c0 + kOvBatch, q1, x1);
   for (int64_t i0 = c0; i0 < c1; i0 += kOvBatch) {
     ids(i0 + 3 * kOvBatch, q3, x3, k3);
+    if (a.dbg && !batch_ok(i0 + 2 * kOvBatch, q2, x2, k2)) {
+      if (lane == 0) atomicCAS(a.status, 0, (int32_t)kDevBounds);
+      break;  // (the copies in flight land below)
+    }
     issue(i0 + 2 * kOvBatch, q2, x2);
     asm volatile("cp.async.wait_group 2;\n" ::: "memory");  // this batch's copies landed
     int64_t *slot = ring + ((i0 - c0) / kOvBatch % kOvDepth) * (kOvBatch * 2 * 32);

@@ -17,7 +17,7 @@ from . import build as _build
 ECHO_OK = 0
 STATUS_NAMES = {0: "ECHO_OK", 1: "ECHO_E_INVALID_ARG", 2: "ECHO_E_BAD_GRAPH", 3: "ECHO_E_CYCLE",
                 4: "ECHO_E_STATE", 5: "ECHO_E_OOM", 6: "ECHO_E_CUDA", 7: "ECHO_E_TIMEOUT",
-                8: "ECHO_E_OVERFLOW", 9: "ECHO_E_UNSUPPORTED"}
+                8: "ECHO_E_OVERFLOW", 9: "ECHO_E_UNSUPPORTED", 10: "ECHO_E_BOUNDS"}
 
 # every function the header declares (checked by the tests)
 EXPORTS = ["echo_create", "echo_destroy", "echo_check_graph", "echo_check_replicas", "echo_overlap_candidates", "echo_load_graph", "echo_load_scenarios",
@@ -60,7 +60,7 @@ class ScenDesc(C.Structure):
 
 class ComposeOpts(C.Structure):
     _fields_ = [("refine_passes", C.c_int32), ("overlap_model", C.c_int32), ("comm_interval", C.c_int32),
-                ("ar_algo_policy", C.c_int32)]
+                ("ar_algo_policy", C.c_int32), ("debug_bounds", C.c_int32)]
 
 
 class CCQueryDesc(C.Structure):
@@ -285,13 +285,15 @@ class Echo:
         self._check(self.lib.echo_estimate_collectives(self.h))
 
     def compose(self, refine_passes: int = 1, overlap_model: int = 0, comm_interval: int = 0,
-                ar_algo_policy: int = 0):
+                ar_algo_policy: int = 0, debug_bounds: bool = False):
         """overlap_model: OVERLAP_WHOLE (d * factor) or OVERLAP_PROPORTIONAL
         (d + (factor - 1) * overlapped length).  comm_interval: COMM_EXECUTION (a
         comm op's [start, finish)) or COMM_LAUNCH (from each member rank's launch).
         ar_algo_policy: AR_PER_OP (each all-reduce's own algorithm), AR_RING,
-        AR_TREE or AR_AUTO for every all-reduce."""
-        o = ComposeOpts(int(refine_passes), int(overlap_model), int(comm_interval), int(ar_algo_policy))
+        AR_TREE or AR_AUTO for every all-reduce.  debug_bounds: device-side index
+        checks (ECHO_E_BOUNDS from the next read when one fails)."""
+        o = ComposeOpts(int(refine_passes), int(overlap_model), int(comm_interval), int(ar_algo_policy),
+                        1 if debug_bounds else 0)
         self._check(self.lib.echo_compose(self.h, C.byref(o)))
 
     def read_times(self, op0: int = 0, op1: Optional[int] = None, start=True, finish=True,

@@ -185,6 +185,43 @@ def test_allreduce_policy_bit_exact(kernel, monkeypatch):
         e.close()
 
 
+@pytest.mark.parametrize("kernel", ["direct", "staged", "pipelined", "dataflow"])
+def test_debug_bounds_checks_pass_and_change_nothing(kernel, monkeypatch):
+    """debug_bounds: every composer and the validator check each index they gather
+    through; on well-formed inputs no check fails and the timelines are the
+    oracle's, for GPT-1.3B and random graphs with all validator variants."""
+    monkeypatch.setenv("ECHO_COMPOSE_KERNEL", kernel)
+    if kernel != "dataflow":
+        monkeypatch.setenv("ECHO_SIGMA", "1" if kernel == "staged" else "4")
+    c = W.config("gpt1.3b")
+    g = W.build_gpt_graph(c)
+    rng = np.random.default_rng(3300)
+    e = Echo(0)
+    try:
+        sc = W.make_scenarios(g, c, n_scen=33)
+        e.load_graph(g)
+        e.load_scenarios(sc)
+        e.estimate_collectives()
+        e.compose(refine_passes=2, debug_bounds=True)
+        st, fn = e.read_times()
+        got = dict(start=st, finish=fn, makespan=e.read_makespan(), cc=e.read_cc(), ov=e.read_overlap())
+        assert_same(got, oracle.compose(g, sc, refine_passes=2, threads=THREADS), g, 2)
+        for case in range(8):
+            g = SG.random_graph(rng, int(rng.integers(20, 300)), max_ranks=5, max_streams=8, p_edge=0.03)
+            sc = SG.random_scenarios(rng, g, 35, max_dur=60)
+            model, civ = case % 2, (case // 2) % 2
+            e.load_graph(g)
+            e.load_scenarios(sc)
+            e.estimate_collectives()
+            e.compose(refine_passes=1 + case % 3, overlap_model=model, comm_interval=civ, debug_bounds=True)
+            st, fn = e.read_times()
+            got = dict(start=st, finish=fn, makespan=e.read_makespan(), cc=e.read_cc(), ov=e.read_overlap())
+            want = oracle.compose(g, sc, refine_passes=1 + case % 3, overlap_model=model, comm_interval=civ)
+            assert_same(got, want, g, 1 + case % 3)
+    finally:
+        e.close()
+
+
 def test_read_times_scenario_range():
     """echo_read_times over a scenario range [s0, s1): the matching columns of the
     full readback, into host and device buffers; bad ranges are rejected."""
