@@ -20,7 +20,6 @@ import argparse
 import hashlib
 import json
 import os
-import re
 import statistics
 import subprocess
 import sys
@@ -35,7 +34,9 @@ sys.path.insert(0, ROOT)
 METRIC = "node×scenario timeline updates/sec and achieved HBM GB/s vs GB300 peak"
 UNIT = "updates/s"
 WORKLOAD = "gpt175b"
-PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "compose_gpt175b.md")
+# DRAM bytes per node-scenario of the composition kernels from the committed ncu
+# capture (a data file beside its summary), valid for the kernel source it names
+PROFILE_DATA = os.path.join(ROOT, "profiles", "compose_gpt175b.json")
 
 
 def log(*a):
@@ -109,25 +110,26 @@ def measured_peaks():
         return 6800.0, "fallback"
 
 
-def kernel_source_hash():
+def source_hash(name):
+    """sha256[:16] of a kernel source file of the library."""
     h = hashlib.sha256()
-    with open(os.path.join(ROOT, "paper_2412_12487_gb300", "csrc", "echo_compose.cu"), "rb") as f:
+    with open(os.path.join(ROOT, "paper_2412_12487_gb300", "csrc", name), "rb") as f:
         h.update(f.read())
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(launch_units):
-    """DRAM bytes per compose launch from the committed ncu summary, scaled to
-    ``launch_units`` node-scenarios, if it was taken on the current kernel source."""
+def profiled_traffic(kernel, launch_units):
+    """DRAM bytes per launch of `kernel` from the committed ncu data (per node-
+    scenario, scaled to ``launch_units`` node-scenarios), if it was taken on the
+    kernel's current source."""
     try:
-        text = open(PROFILE_SUMMARY).read()
-    except OSError:
+        with open(PROFILE_DATA) as f:
+            d = json.load(f)["kernels"][kernel]
+        if d["source_sha256_16"] != source_hash(d["source"]):
+            return None
+        return float(d["dram_bytes_per_node_scenario"]) * launch_units
+    except (OSError, ValueError, KeyError, TypeError):
         return None
-    m_hash = re.search(r"kernel source sha256\[:16\]:\s*([0-9a-f]{16})", text)
-    m_bytes = re.search(r"dram bytes per node-scenario \(compose\):\s*([0-9.]+)", text)
-    if not m_hash or not m_bytes or m_hash.group(1) != kernel_source_hash():
-        return None
-    return float(m_bytes.group(1)) * launch_units
 
 
 _HOST_BUFFERS = []
@@ -174,12 +176,43 @@ def build_inputs(rank, world, n_scen=None, pinned=True, workload=WORKLOAD):
     return c, g, sc, dur_t
 
 
-def algorithmic_bytes_per_pass(g, info, S):
+def algorithmic_bytes(g, info, S):
+    """Bytes each kernel of one step must move (reuse of values written in the same
+    pass is not counted):
+      compose           first composition: every compute/memcpy duration read, the
+                        finishes that a later step reads written (all of them for the
+                        dataflow composer), the graph arrays, the CC table;
+      compose_adjusted  final composition: durations read and every finish written,
+                        plus the validator's rows of the candidates;
+      overlap           validator: each candidate's finish and duration read, its
+                        next duration written, the comm rows its cursors visit."""
     from paper_2412_12487_gb300 import workloads as W
     v_cd = int(((g.kind == W.KIND_COMPUTE) | (g.kind == W.KIND_MEMCPY)).sum())
     v_comm = g.n_ops - v_cd
     graph = 8 * (g.n_ops + 1) + 4 * g.n_edges + 4 * g.n_ops
-    return S * (16 * v_cd + 8 * v_comm) + graph + 16 * info["n_signatures"] * S
+    cc = 16 * info["n_signatures"] * S
+    n_cand, n_kept, n_ce = info["n_overlap_candidates"], info["n_kept_finishes"], info["n_validator_comm_entries"]
+    return {"compose": S * (8 * v_cd + 8 * n_kept) + graph + cc,
+            "compose_adjusted": S * (16 * v_cd + 8 * v_comm + 8 * n_cand) + graph + cc,
+            "overlap": S * (24 * n_cand + 16 * n_ce)}
+
+
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:  # pragma: no cover
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu part")):
+                return line.split(":", 1)[1].strip()
+    except OSError:  # pragma: no cover
+        pass
+    return "unknown"
 
 
 def run_echo(args):
@@ -281,15 +314,27 @@ def run_echo(args):
     value = units * world / (ms / 1e3)
     e2e_value = units * world / (e2e_ms / 1e3)
 
-    comp_launches, comp_ms = prof.get("compose", (0, 0.0))
     launches = sum(n for k, (n, _) in prof.items() if k != "dur_copy")  # kernels only
     peak, peak_kind = measured_peaks()
-    b_pass = algorithmic_bytes_per_pass(g, info, S)
-    per_launch_ms = comp_ms / max(comp_launches, 1)
-    achieved = b_pass / (per_launch_ms / 1e3) / 1e9 if comp_launches else None
+    alg = algorithmic_bytes(g, info, S)
     composer = "dataflow" if info["sigma"] == 32 else "levelled"
-    # the committed capture is of the levelled composer on this workload
-    traffic = profiled_traffic(V * S) if args.workload == WORKLOAD and composer == "levelled" else None
+    kernels = {}
+    for k, (n, t_) in prof.items():
+        ent = {"launches": n, "ms_per_launch": t_ / max(n, 1)}
+        if k in alg and n:
+            ach = alg[k] / (t_ / n / 1e3) / 1e9
+            ent.update({"alg_bytes_per_launch": alg[k], "achieved_gbs": ach, "frac": ach / peak})
+        kernels[k] = ent
+    # the dominant kernel of the step (largest total time) carries the roofline
+    dom = max((k for k in alg if k in prof), key=lambda k: prof[k][1], default=None)
+    traffic = None
+    if dom and args.workload == WORKLOAD:
+        traffic = profiled_traffic(dom, V * S)
+    roof = {"kernel": dom, "bound": "hbm", "achieved": kernels[dom]["achieved_gbs"] if dom else None,
+            "peak": peak, "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+            "unit": "GB/s", "frac": kernels[dom]["frac"] if dom else None, "traffic": traffic,
+            "alg_bytes_per_launch": alg.get(dom)}
+    step_bytes = sum(alg[k] * prof[k][0] for k in alg if k in prof) / max(args.steps, 1)
     out = None
     if rank == 0:
         cpu = cpu_baseline(g, c, args) if world == 1 and args.cpu_sample > 0 else None
@@ -310,11 +355,9 @@ def run_echo(args):
                                   "other's compute)",
                     "inputs": "durations as int32 (every value fits), composed in int64"},
             "gpu_launches": launches,
-            "kernels": {k: {"launches": n, "ms_per_launch": t_ / max(n, 1)} for k, (n, t_) in prof.items()},
-            "roofline": {"kernel": "compose", "bound": "hbm", "achieved": achieved, "peak": peak,
-                         "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
-                         "unit": "GB/s", "frac": (achieved / peak) if achieved else None,
-                         "traffic": traffic, "alg_bytes_per_launch": b_pass},
+            "kernels": kernels,
+            "roofline": roof,
+            "step_alg_gbs": step_bytes / (ms / 1e3) / 1e9,
             "clocks": clk,
             "cpu_baseline": cpu,
         }
@@ -325,32 +368,70 @@ def run_echo(args):
     return out
 
 
-def cpu_baseline(g, c, args, n_sample=None):
-    """The CPU oracle as it stands, single-threaded, on a bounded sample of the
-    same workload (the first scenarios of the batch)."""
+def cpu_baseline(g, c, args):
+    """The CPU oracle as it stands on the host cores, on bounded samples of the same
+    workload (the batch's first scenarios): scenario-parallel on every core (the
+    reported value), and single-threaded beside it.  One sample step = CC estimate,
+    two compositions and the overlap test, as on the GPU."""
     import oracle
     from paper_2412_12487_gb300 import workloads as W
-    n_sample = min(n_sample or args.cpu_sample, c.n_scen)
-    sub = W.select_scenarios(W.scenario_params(c), g, list(range(n_sample)))
+    cores = os.cpu_count() or 1
+    base = W.scenario_params(c)
+    n1 = min(max(1, args.cpu_sample), c.n_scen)
+    sub = W.select_scenarios(base, g, list(range(n1)))
     t0 = time.time()
-    oracle.compose(g, sub, refine_passes=1, threads=1, want_cc=False, want_overlap=False)
-    dt = time.time() - t0
-    return {"value": 2 * g.n_ops * n_sample / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{n_sample} of the {c.n_scen} scenarios of {c.name} ({g.n_ops} ops), "
-                      f"CC estimate + 2 compositions + overlap, {dt:.1f} s single-threaded",
-            "seconds": dt, "host_cores_available": os.cpu_count()}
+    oracle.compose(g, sub, refine_passes=1, threads=1, want_cc=False, want_overlap=False, want_times=False)
+    dt1 = time.time() - t0
+    nm = min(cores * max(1, args.cpu_sample // 2), c.n_scen)
+    sub = W.select_scenarios(base, g, list(range(nm)))
+    t0 = time.time()
+    oracle.compose(g, sub, refine_passes=1, threads=cores, want_cc=False, want_overlap=False, want_times=False)
+    dtm = time.time() - t0
+    model = cpu_model()
+    return {"value": 2 * g.n_ops * nm / dtm, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{nm} of the {c.n_scen} scenarios of {c.name} ({g.n_ops} ops), one scenario per "
+                      f"thread on {cores} threads: CC estimate + 2 compositions + overlap test, {dtm:.1f} s",
+            "seconds": dtm, "cpu_model": model,
+            "single_core": {"value": 2 * g.n_ops * n1 / dt1, "unit": UNIT, "cores": 1,
+                            "sample": f"{n1} scenarios, single-threaded, {dt1:.1f} s"}}
 
 
 CCQ_WORKLOAD = "cc-queries"
 
 
+def cc_query_fp64_ops(q):
+    """fp64 adds, multiplies and divides of each query's estimate, branch by branch
+    as the closed forms of Sec. 5.3 evaluate them (ring: per-step size and time,
+    steps times step, setup, reduction; tree: chunk size, beta, gamma, the four
+    terms of Eq. 5; AUTO: both; send/recv: one chunk transfer times eta)."""
+    from paper_2412_12487_gb300 import workloads as W
+    n = q.cc_type.shape[0]
+    add, mul, div = np.zeros(n), np.zeros(n), np.zeros(n)
+    live = (q.n_ranks > 1) & (q.nbytes > 0)
+    t, a, inter = q.cc_type, q.cc_algo, q.n_nodes > 1
+    ring_ar = live & (t == W.CC_ALLREDUCE) & (a != W.ALGO_TREE)
+    tree_ar = live & (t == W.CC_ALLREDUCE) & (a != W.ALGO_RING)
+    for m, (ad, mu, dv) in ((live & (t == W.CC_SENDRECV), (2, 1, 2)), (live & (t == W.CC_ALLGATHER), (2, 2, 2)),
+                            (live & (t == W.CC_REDUCESCATTER), (3, 3, 2)), (ring_ar, (3, 3, 2))):
+        add[m] += ad
+        mul[m] += mu
+        div[m] += dv
+    add[tree_ar] += 5 + inter[tree_ar]
+    mul[tree_ar] += 6
+    div[tree_ar] += 2 + inter[tree_ar]
+    return float(add.sum()), float(mul.sum()), float(div.sum())
+
+
 def run_cc_queries(args):
     """The standalone CC-estimator sweep (1M queries of Sec. 5.3's closed forms):
     queries/s of the estimator kernel (device time) and through the C ABI call
-    (host arrays in, host results out), with the oracle's rate on a sample."""
+    (host arrays in, host results out), with the oracle's rate on a sample.  Its
+    roofline is the fp64 rate of this device for the sweep's mix of adds,
+    multiplies and divides (measured in the same run), beside the HBM bound of its
+    82 bytes per query."""
     import torch
     import oracle
-    from paper_2412_12487_gb300 import Echo
+    from paper_2412_12487_gb300 import Echo, echo as E
     from paper_2412_12487_gb300 import workloads as W
     n = args.scenarios or 1_000_000
     q = W.make_cc_queries(n)
@@ -370,6 +451,12 @@ def run_cc_queries(args):
         prof = e.read_profile()
     k_n, k_ms = prof.get("cc_query", (0, 0.0))
     kern_ms = k_ms / max(k_n, 1)
+    rates = E.measure_fp64(0)
+    n_add, n_mul, n_div = cc_query_fp64_ops(q)
+    bound_s = n_add / rates["dadd"] + n_mul / rates["dmul"] + n_div / rates["ddiv"]
+    ops = n_add + n_mul + n_div
+    peak_hbm, peak_kind = measured_peaks()
+    bytes_q = 1 + 1 + 8 + 4 + 4 + 6 * 8 + 8 + 8  # type, algo, size, N, M, parameters, log2 M in; estimate out
     oracle.build()
     m = min(n, 20000)
     t0 = time.perf_counter()
@@ -386,14 +473,26 @@ def run_cc_queries(args):
             "data": "synthetic", "config": {"workload": f"{n} CC-estimator queries (Sec. 5.3)"},
             "e2e": {"value": n / (call_ms / 1e3), "unit": "queries/s", "ms_per_step": call_ms,
                     "h2d_bytes_per_step": n * (1 + 1 + 8 + 4 + 4 + 6 * 8), "d2h_bytes_per_step": n * 8},
+            "gpu_launches": k_n,
+            "roofline": {"kernel": "cc_query", "bound": "alu", "unit": "Gop/s",
+                         "achieved": ops / (kern_ms / 1e3) / 1e9, "peak": ops / bound_s / 1e9,
+                         "frac": bound_s / (kern_ms / 1e3), "traffic": None,
+                         "peak_source": "fp64 add/mul/div rates measured in this run (echo_measure_fp64), "
+                                        "weighted by the sweep's operation mix",
+                         "fp64_ops_per_query": ops / n, "fp64_rates_per_s": rates},
+            "roofline_hbm": {"bound": "hbm", "unit": "GB/s", "achieved": n * bytes_q / (kern_ms / 1e3) / 1e9,
+                             "peak": peak_hbm, "frac": n * bytes_q / (kern_ms / 1e3) / 1e9 / peak_hbm,
+                             "peak_source": f"{peak_kind} copy bandwidth", "bytes_per_query": bytes_q},
             "max_rel_diff_vs_oracle_sample": rel,
             "cpu_baseline": {"value": m / cpu_s, "unit": "queries/s", "cores": 1, "kind": "oracle",
+                             "cpu_model": cpu_model(),
                              "sample": f"first {m} queries, one at a time through the oracle's C function"}}
 
 
 def run_reference(args):
     """Reference arm: the CPU oracle (a plain event-driven simulator written from
-    the paper) timed on the host cores on the same workload, one scenario per step."""
+    the paper) timed on the host cores on the same workload, each step one scenario
+    per core composed in parallel (a bounded sample of the batch)."""
     rank, world, _ = dist_env()
     if rank != 0:
         return None
@@ -402,26 +501,26 @@ def run_reference(args):
     c = W.config(args.workload)
     g = W.build_gpt_graph(c)
     base = W.scenario_params(c)
+    cores = os.cpu_count() or 1
     oracle.build()
 
     def step(i):
-        sub = W.select_scenarios(base, g, [i % base.n_scen])
-        oracle.compose(g, sub, refine_passes=1, threads=1, want_cc=False, want_overlap=False)
+        sub = W.select_scenarios(base, g, [(i * cores + k) % base.n_scen for k in range(cores)])
+        t0 = time.time()
+        oracle.compose(g, sub, refine_passes=1, threads=cores, want_cc=False, want_overlap=False, want_times=False)
+        return time.time() - t0
 
     for i in range(args.warmup):
         step(i)
-    t0 = time.time()
-    for i in range(args.steps):
-        step(args.warmup + i)
-    dt = (time.time() - t0) / args.steps
-    v = 2 * g.n_ops / dt
+    dt = sum(step(args.warmup + i) for i in range(args.steps)) / args.steps
+    v = 2 * g.n_ops * cores / dt
     return {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-            "config": {"workload": f"{c.name} x 1 scenario per step (bounded sample of the "
-                                   f"{c.n_scen}-scenario batch)", "ops": g.n_ops},
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": "one scenario per step, single-threaded"},
+            "config": {"workload": f"{c.name} x {cores} scenarios per step, one per core (bounded sample of "
+                                   f"the {c.n_scen}-scenario batch)", "ops": g.n_ops},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "cpu_model": cpu_model(),
+                             "sample": f"{cores} scenarios per step, one per thread"},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 

@@ -316,6 +316,9 @@ typedef struct {
   int32_t replicas_folded;
   int64_t n_validator_comm_entries; /* (comm op, member rank) pairs the validator's cursors
                                        visit: those that can overlap a compute op of the rank */
+  int64_t n_kept_finishes;  /* ops whose finish a composition before the last stores (the
+                               others are read by no later step); n_ops_composed for the
+                               dataflow composer, which stores every finish */
 } echo_graph_info;
 int echo_graph_info_get(echo_ctx *ctx, echo_graph_info *info);
 
@@ -330,6 +333,14 @@ typedef struct {
 } echo_kernel_stat;
 int echo_set_profiling(echo_ctx *ctx, int enable);
 int echo_read_profile(echo_ctx *ctx, echo_kernel_stat *out, int cap, int *n);
+
+/* Measurement support (the paper has no counterpart): the fp64 rates of `device`,
+ * in operations per second, of round-to-nearest add, multiply and divide
+ * (rates[0..2]), from CUDA-event timing of independent chains of each.  The
+ * roofline of the CC estimator's fp64 arithmetic uses them.  Changes no clock or
+ * setting of the device; the calling thread's current device is restored.
+ * Allocates and frees 8 bytes. */
+int echo_measure_fp64(int device, double *rates);
 
 const char *echo_strerror(int status);
 /* Copies the context's last error message (NUL-terminated) into buf. */

@@ -2269,6 +2269,14 @@ int echo_graph_info_get(echo_ctx *c, echo_graph_info *info) {
   info->n_segment_levels = B.Ls;
   info->n_overlap_candidates = B.cand_off.empty() ? 0 : B.cand_off.back();
   info->n_validator_comm_entries = B.cq_off.empty() ? 0 : B.cq_off.back();
+  info->n_kept_finishes = B.V;
+  if (!c->use_df) {  // segment tails and the ops whose finish the validator reads
+    int64_t n = 0;
+    for (int64_t t = 0; t < B.n_seg; ++t)
+      for (int64_t v = B.seg_node_off[t]; v < B.seg_node_off[t + 1]; ++v)
+        n += (v + 1 == B.seg_node_off[t + 1]) || B.keep[v];
+    info->n_kept_finishes = n;
+  }
   info->n_ranks = B.R;
   info->n_streams = B.NS;
   info->sigma = c->sigma;

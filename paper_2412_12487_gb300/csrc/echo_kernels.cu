@@ -383,7 +383,79 @@ cudaError_t launch_read_ov(const int32_t *ext2int, int64_t op0, int64_t op1, int
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------------
+// fp64 rates of this device (measurement support): each thread keeps 8 independent
+// chains of one operation (add, multiply or divide with round-to-nearest, as the
+// CC estimator uses them), so the pipe, not the dependence latency, sets the rate.
+// The result feeds a kernel in the sink so nothing is optimized away.
+// ---------------------------------------------------------------------------------
+constexpr int kFp64Chains = 8;
+template <int OP>
+__global__ void fp64_rate_kernel(int iters, double y, double *sink) {
+  double x[kFp64Chains];
+#pragma unroll
+  for (int k = 0; k < kFp64Chains; ++k) x[k] = 1.0 + (threadIdx.x + k) * 1e-9;
+  for (int i = 0; i < iters; ++i) {
+#pragma unroll
+    for (int k = 0; k < kFp64Chains; ++k)
+      x[k] = OP == 0 ? __dadd_rn(x[k], y) : OP == 1 ? __dmul_rn(x[k], y) : __ddiv_rn(x[k], y);
+  }
+  double t = 0.0;
+#pragma unroll
+  for (int k = 0; k < kFp64Chains; ++k) t = __dadd_rn(t, x[k]);
+  if (t == 12345.0) sink[0] = t;  // never true for these inputs
+}
+
 }  // namespace echo
+
+extern "C" int echo_measure_fp64(int device, double *rates) {
+  using namespace echo;
+  if (!rates) return ECHO_E_INVALID_ARG;
+  int prev = 0;
+  if (cudaGetDevice(&prev) != cudaSuccess || cudaSetDevice(device) != cudaSuccess) return ECHO_E_CUDA;
+  struct Restore {
+    int dev;
+    ~Restore() { cudaSetDevice(dev); }
+  } restore{prev};
+  int sms = 0;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+  double *sink = nullptr;
+  if (cudaMalloc(&sink, sizeof(double)) != cudaSuccess) return ECHO_E_OOM;
+  cudaEvent_t a, b;
+  cudaEventCreate(&a);
+  cudaEventCreate(&b);
+  const int threads = 256, blocks = sms * 8;
+  int rc = ECHO_OK;
+  for (int op = 0; op < 3 && rc == ECHO_OK; ++op) {
+    const int iters = op == 2 ? 256 : 4096;
+    const double y = op == 1 ? 1.0000000001 : op == 2 ? 0.9999999999 : 1e-12;
+    auto launch = [&]() {
+      if (op == 0) fp64_rate_kernel<0><<<blocks, threads>>>(iters, y, sink);
+      else if (op == 1) fp64_rate_kernel<1><<<blocks, threads>>>(iters, y, sink);
+      else fp64_rate_kernel<2><<<blocks, threads>>>(iters, y, sink);
+    };
+    launch();  // warm-up
+    float best = 0.f;
+    for (int rep = 0; rep < 5; ++rep) {
+      cudaEventRecord(a);
+      launch();
+      cudaEventRecord(b);
+      if (cudaEventSynchronize(b) != cudaSuccess) {
+        rc = ECHO_E_CUDA;
+        break;
+      }
+      float ms = 0.f;
+      cudaEventElapsedTime(&ms, a, b);
+      if (rep == 0 || ms < best) best = ms;
+    }
+    rates[op] = (double)blocks * threads * iters * kFp64Chains / (best * 1e-3);
+  }
+  if (cudaGetLastError() != cudaSuccess && rc == ECHO_OK) rc = ECHO_E_CUDA;
+  cudaEventDestroy(a);
+  cudaEventDestroy(b);
+  cudaFree(sink);
+  return rc;
+}
 
 // ---------------------------------------------------------------------------------
 // Allocation-free CC queries.

@@ -24,7 +24,7 @@ EXPORTS = ["echo_create", "echo_destroy", "echo_check_graph", "echo_check_replic
            "echo_estimate_collectives", "echo_compose", "echo_read_times", "echo_read_makespan",
            "echo_read_cc", "echo_read_overlap", "echo_cc_query", "echo_cc_query_noalloc",
            "echo_graph_info_get", "echo_set_cc_model",
-           "echo_set_profiling", "echo_read_profile", "echo_strerror", "echo_last_error"]
+           "echo_set_profiling", "echo_read_profile", "echo_measure_fp64", "echo_strerror", "echo_last_error"]
 
 
 class EchoError(RuntimeError):
@@ -77,7 +77,8 @@ class GraphInfo(C.Structure):
                 ("n_signatures", C.c_int64), ("n_segments", C.c_int64), ("n_segment_levels", C.c_int64),
                 ("n_overlap_candidates", C.c_int64), ("n_ops_composed", C.c_int64),
                 ("n_ranks", C.c_int32), ("n_streams", C.c_int32), ("sigma", C.c_int32),
-                ("replicas_folded", C.c_int32), ("n_validator_comm_entries", C.c_int64)]
+                ("replicas_folded", C.c_int32), ("n_validator_comm_entries", C.c_int64),
+                ("n_kept_finishes", C.c_int64)]
 
 
 class KernelStat(C.Structure):
@@ -122,6 +123,7 @@ def load_library(path: Optional[str] = None):
         "echo_set_cc_model": ([vp, C.c_int], C.c_int),
         "echo_set_profiling": ([vp, C.c_int], C.c_int),
         "echo_read_profile": ([vp, C.POINTER(KernelStat), C.c_int, C.POINTER(C.c_int)], C.c_int),
+        "echo_measure_fp64": ([C.c_int, vp], C.c_int),
         "echo_strerror": ([C.c_int], C.c_char_p),
         "echo_last_error": ([vp, C.c_char_p, C.c_size_t], C.c_int),
     }
@@ -201,6 +203,16 @@ def overlap_candidates(g) -> np.ndarray:
         raise EchoError(rc, lib.echo_strerror(rc).decode())
     assert int(out.sum()) == int(n.value)
     return out
+
+
+def measure_fp64(device: int = 0) -> Dict[str, float]:
+    """fp64 add / multiply / divide rates of the device (operations per second)."""
+    lib = load_library()
+    r = np.zeros(3, np.float64)
+    rc = lib.echo_measure_fp64(int(device), _ptr(r))
+    if rc:
+        raise EchoError(rc, lib.echo_strerror(rc).decode())
+    return {"dadd": float(r[0]), "dmul": float(r[1]), "ddiv": float(r[2])}
 
 
 class Echo:
