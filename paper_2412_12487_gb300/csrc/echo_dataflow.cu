@@ -109,11 +109,57 @@ __device__ __noinline__ bool df_batch_ok(uint2 w, int64_t b, int64_t e1, bool ca
     }
     if (hdr & kDfComm) {
       const uint32_t nm = nmme & 0xFFFF, me = nmme >> 16;
-      ok &= nm <= 1 || (me < nm && range_ok(slot, (int64_t)slot + nm, a.n_slots));
+      if (slot & kDfBlockJoin)  // a block join: its members are this block's warps
+        ok &= nm == (uint32_t)a.wpb && me < nm;
+      else
+        ok &= nm <= 1 || (me < nm && range_ok(slot, (int64_t)slot + nm, a.n_slots));
     }
     if (hdr & (kDfExport | kDfTwoHop)) ok &= in_range(xid, a.n_exports);
   }
   return ok;
+}
+
+// Join of a comm op whose nm members are the warps of this block (member me is this
+// warp): each member stores its partial launch time, tagged with the join's
+// sequence number, into slot seq % 2, and waits until every member's word of that
+// slot carries the tag.  Members reach the block's joins in the same (internal)
+// order and a member can only start join n + 2 once every member has finished
+// reading join n, so two slots suffice; the tag ((seq / 2) mod 7) + 1 tells join n
+// from n - 2.  Bounded like df_gather; false when this wait or another warp's
+// gave up.
+__device__ bool block_join(uint64_t *bjoin, uint32_t seq, uint32_t me, uint32_t nm, int64_t &t,
+                           const DataflowArgs &a) {
+  uint64_t *row = bjoin + (size_t)(seq & 1) * nm * 32 + (threadIdx.x & 31);
+  const uint64_t tag = (uint64_t)((seq >> 1) % 7 + 1) << 61;
+  asm volatile("st.volatile.shared.u64 [%0], %1;" ::"r"((uint32_t)__cvta_generic_to_shared(row + me * 32)),
+               "l"(tag | (uint64_t)t)
+               : "memory");
+  const long long t0 = clock64();
+  for (uint32_t round = 0;; ++round) {
+    bool ok = true;
+    int64_t m = t;
+    for (uint32_t k = 0; k < nm; ++k) {
+      uint64_t x;
+      asm volatile("ld.volatile.shared.u64 %0, [%1];" : "=l"(x) : "r"((uint32_t)__cvta_generic_to_shared(row + k * 32))
+                   : "memory");
+      ok &= (x & ~kValueMask) == tag;
+      m = max(m, (int64_t)(x & kValueMask));
+    }
+    if (__all_sync(kFull, ok)) {
+      t = m;
+      return true;
+    }
+    const bool give_up = ((round & 15) == 15 && ld_relaxed_s32(a.abort_flag) != 0) ||
+                         clock64() - t0 > a.wait_limit_cycles;
+    if (__any_sync(kFull, give_up)) {
+      if ((threadIdx.x & 31) == 0) {
+        atomicExch(a.abort_flag, 1);
+        atomicCAS(a.status, (int32_t)kDevOk, (int32_t)kDevTimeout);
+      }
+      return false;
+    }
+    if (round >= 64) __nanosleep(64);
+  }
 }
 
 __device__ __forceinline__ void cp_async_8(void *smem, const void *gmem) {
@@ -122,14 +168,19 @@ __device__ __forceinline__ void cp_async_8(void *smem, const void *gmem) {
 }
 
 template <bool CAND>
-__global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_kernel(DataflowArgs a) {
-  // per warp: the duration ring [kDfDepth + 1][kDfBatch][32], then [n_streams][32]
-  // latest finishes of the rank's timelines
+__global__ void __launch_bounds__(kDfMaxWarpsPerBlock * 32, 2) compose_dataflow_kernel(DataflowArgs a) {
+  // block: [2][wpb][32] tagged partial launch times of the block joins; then per
+  // warp the duration ring [kDfDepth + 1][kDfBatch][32] and [n_streams][32] latest
+  // finishes of the rank's timelines
   extern __shared__ int64_t df_smem[];
-  int64_t *dring = df_smem + (int64_t)(threadIdx.x >> 5) * ((kDfDepth + 1) * kDfBatch * 32 + a.n_streams * 32);
+  uint64_t *bjoin = reinterpret_cast<uint64_t *>(df_smem);
+  int64_t *dring = df_smem + 2 * a.wpb * 32 +
+                   (int64_t)(threadIdx.x >> 5) * ((kDfDepth + 1) * kDfBatch * 32 + a.n_streams * 32);
   int64_t *df_last = dring + (kDfDepth + 1) * kDfBatch * 32;
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
-  const int64_t wid = (int64_t)blockIdx.x * (kDfThreads / 32) + wib;
+  for (int k = threadIdx.x; k < 2 * a.wpb * 32; k += blockDim.x) bjoin[k] = 0;  // tag 0: never written
+  __syncthreads();
+  const int64_t wid = (int64_t)blockIdx.x * a.wpb + wib;
   if (wid >= (int64_t)a.R * a.G) return;  // uniform over the warp
   const int32_t r = (int32_t)(wid % a.R), g = (int32_t)(wid / a.R);
   const int32_t s = g * 32 + lane;
@@ -230,7 +281,13 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
       if (hdr & kDfComm) {
         const uint32_t slot = __shfl_sync(kFull, w0.x, 4 * j + 2), nmme = __shfl_sync(kFull, w0.y, 4 * j + 2);
         const uint32_t nm = nmme & 0xFFFF, me = nmme >> 16;
-        if (nm > 1) {
+        if (slot & kDfBlockJoin) {  // the members are this block's warps: join in shared memory
+          if (!block_join(bjoin, slot & ~kDfBlockJoin, me, nm, t, a)) {
+            asm volatile("cp.async.wait_all;" ::: "memory");
+            return;
+          }
+          fv = t + d0[j * 32];
+        } else if (nm > 1) {
           if (a.skip_slot != (int64_t)slot + me) st_relaxed_u64(part + ((int64_t)(slot + me) << 5), tag | (uint64_t)t);
           if (!(hdr & kDfTwoHop) || me == 0) {
             for (uint32_t m0 = 0; m0 < nm; m0 += 8)  // the other members, 8 at a time
@@ -268,33 +325,38 @@ __global__ void __launch_bounds__(kDfThreads, kDfMinBlocks) compose_dataflow_ker
 
 }  // namespace
 
-size_t dataflow_smem_bytes(int32_t n_streams) {
-  return (size_t)(kDfThreads / 32) * ((kDfDepth + 1) * kDfBatch * 32 + n_streams * 32) * sizeof(int64_t);
+size_t dataflow_smem_bytes(int32_t n_streams, int32_t wpb) {
+  return ((size_t)2 * wpb * 32 + (size_t)wpb * ((kDfDepth + 1) * kDfBatch * 32 + n_streams * 32)) * sizeof(int64_t);
 }
 
-bool dataflow_fits(int64_t n_warps, int32_t n_streams, int device) {
+bool dataflow_fits(int64_t n_warps, int32_t n_streams, int32_t wpb, int device) {
   int sms = 0, coop = 0, per_sm0 = 0, per_sm1 = 0;
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
   cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, device);
-  const size_t smem = dataflow_smem_bytes(n_streams);
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm0, compose_dataflow_kernel<false>, kDfThreads, smem) !=
+  const size_t smem = dataflow_smem_bytes(n_streams, wpb);
+  if (cudaFuncSetAttribute(compose_dataflow_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
           cudaSuccess ||
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm1, compose_dataflow_kernel<true>, kDfThreads, smem) !=
+      cudaFuncSetAttribute(compose_dataflow_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+          cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm0, compose_dataflow_kernel<false>, 32 * wpb, smem) !=
+          cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm1, compose_dataflow_kernel<true>, 32 * wpb, smem) !=
           cudaSuccess) {
     cudaGetLastError();
     return false;
   }
-  const int64_t blocks = (n_warps + kDfThreads / 32 - 1) / (kDfThreads / 32);
+  const int64_t blocks = (n_warps + wpb - 1) / wpb;
   return coop && blocks <= (int64_t)std::min(per_sm0, per_sm1) * sms;
 }
 
 cudaError_t launch_compose_dataflow(const DataflowArgs &a, cudaStream_t st) {
   const int64_t warps = (int64_t)a.R * a.G;
   if (warps == 0) return cudaSuccess;
-  const dim3 grid((unsigned)((warps + kDfThreads / 32 - 1) / (kDfThreads / 32))), block(kDfThreads);
+  if (a.wpb < 1 || a.wpb > kDfMaxWarpsPerBlock || a.R % a.wpb) return cudaErrorInvalidValue;
+  const dim3 grid((unsigned)((warps + a.wpb - 1) / a.wpb)), block(32 * a.wpb);
   DataflowArgs args = a;
   void *params[] = {&args};
-  const size_t smem = dataflow_smem_bytes(a.n_streams);
+  const size_t smem = dataflow_smem_bytes(a.n_streams, a.wpb);
   if (a.cdur)
     return cudaLaunchCooperativeKernel((const void *)compose_dataflow_kernel<true>, grid, block, params, smem, st);
   return cudaLaunchCooperativeKernel((const void *)compose_dataflow_kernel<false>, grid, block, params, smem, st);

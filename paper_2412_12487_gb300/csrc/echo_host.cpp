@@ -91,6 +91,7 @@ struct GraphBuild {
   std::vector<int64_t> df_off;
   std::vector<uint32_t> df_rec, df_opnd;
   int64_t df_slots = 0, df_exports = 0;
+  int32_t df_wpb = 1;  // warps per block: a block holds df_wpb consecutive ranks (for block joins)
   bool stageable = true;              // every head has < 2^16 inputs
 };
 
@@ -245,13 +246,38 @@ void build_dataflow(GraphBuild &b) {
     return std::binary_search(ro.data() + ro_off[u], ro.data() + ro_off[u + 1], r);
   };
   auto members = [&](int32_t v) { return ro_off[v + 1] - ro_off[v]; };
-  // partial slots, and the producers of each comm op that run on none of its members
+  // Block joins: a comm op whose members are exactly the ranks of one block of
+  // df_wpb consecutive ranks (aligned) joins through shared memory.  The width is the
+  // one (dividing R, at most 8) whose blocks hold the most comm ops.
+  auto aligned_group = [&](int64_t v, int32_t w) {
+    if (members((int32_t)v) != w) return false;
+    const int32_t r0 = ro[ro_off[v]];
+    return r0 % w == 0 && ro[ro_off[v] + w - 1] == r0 + w - 1;
+  };
+  b.df_wpb = 1;
+  {
+    int64_t best = 0;
+    for (int32_t w = 2; w <= 8; w *= 2) {
+      if (R % w) continue;
+      int64_t n = 0;
+      for (int64_t v = 0; v < V; ++v) n += b.is_comm[v] && aligned_group(v, w);
+      if (n > best) {
+        best = n;
+        b.df_wpb = w;
+      }
+    }
+  }
+  // partial slots (block joins take a per-block sequence number instead), and the
+  // producers of each comm op that run on none of its members
   std::vector<int64_t> slot(V, 0);
   std::vector<uint8_t> uncovered(std::max<int64_t>(b.dp_off[V], 1), 0);
+  std::vector<uint32_t> bseq(R / b.df_wpb, 0);
   b.df_slots = 0;
   for (int64_t v = 0; v < V; ++v) {
     if (!b.is_comm[v]) continue;
-    if (members((int32_t)v) > 1) {
+    if (b.df_wpb > 1 && aligned_group(v, b.df_wpb)) {
+      slot[v] = echo::kDfBlockJoin | bseq[ro[ro_off[v]] / b.df_wpb]++;
+    } else if (members((int32_t)v) > 1) {
       slot[v] = b.df_slots;
       b.df_slots += members((int32_t)v);
     }
@@ -328,7 +354,7 @@ void build_dataflow(GraphBuild &b) {
       w[1] = b.cidx[v] >= 0 ? (uint32_t)b.cidx[v] : ~0u;
       w[2] = hdr;
       w[3] = (uint32_t)b.df_opnd.size();
-      w[4] = comm ? (uint32_t)slot[v] : 0u;
+      w[4] = comm ? (uint32_t)slot[v] : 0u;  // (kDfBlockJoin | sequence number for a block join)
       w[5] = comm ? (uint32_t)nm | ((uint32_t)me << 16) : 0u;
       w[6] = publish || two_hop ? (uint32_t)exp_id[v] : 0u;
       w[7] = 0u;
@@ -338,7 +364,9 @@ void build_dataflow(GraphBuild &b) {
       prev_tl[r] = (int8_t)k;
     }
   }
-  if (b.df_slots >= (int64_t)UINT32_MAX) return;
+  if (b.df_slots >= (int64_t)echo::kDfBlockJoin) return;
+  for (uint32_t n : bseq)
+    if (n >= echo::kDfBlockJoin) return;
   if (b.df_rec.empty()) b.df_rec.assign(8, 0);
   if (b.df_opnd.empty()) b.df_opnd.push_back(0);
   b.df_ok = true;
@@ -1719,7 +1747,7 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   const int32_t n_groups = (S + 31) / 32;
   bool use_df = false;
   if (B.df_ok && (c->kernel_choice == 0 || c->kernel_choice == 4) &&
-      echo::dataflow_fits((int64_t)B.R * n_groups, B.NS, c->device)) {
+      echo::dataflow_fits((int64_t)B.R * n_groups, B.NS, B.df_wpb, c->device)) {
     int64_t longest = 0;
     for (int32_t r = 0; r < B.R; ++r) longest = std::max(longest, B.df_off[r + 1] - B.df_off[r]);
     use_df = c->kernel_choice == 4 || 2 * longest < 5 * make_steps(B, kStepNodes).L;
@@ -1986,6 +2014,7 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       a.wait_limit_cycles = c->wait_limit_cycles;
       a.skip_slot = c->skip_level;
       a.n_opnd = (int64_t)B.df_opnd.size();
+      a.wpb = B.df_wpb;
       a.dbg = dbg;
       if ((err = cudaMemsetAsync(c->mk, 0, (size_t)c->S * sizeof(int64_t), c->stream)) != cudaSuccess ||
           (err = cudaMemsetAsync(c->df_abort, 0, sizeof(int32_t), c->stream)) != cudaSuccess)

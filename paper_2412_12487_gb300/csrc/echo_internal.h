@@ -182,8 +182,6 @@ struct OverlapArgs {
 // kind, an earlier op of the rank (node id) or another warp's op (export id).
 // Published values are times (below 2^61) tagged with the launch's epoch (1-7)
 // in the top 3 bits.
-constexpr int kDfThreads = 32;     // one warp per block
-constexpr int kDfMinBlocks = 21;  // warps per SM to keep resident (80 registers a thread)
 constexpr int kDfBatch = 8;
 constexpr int kDfDepth = 3;       // batches of durations in flight ahead of the one in use
 constexpr uint32_t kDfPayload = 0x3FFFFFFFu;
@@ -192,6 +190,10 @@ enum : uint32_t { kDfComm = 1u << 4, kDfPrev = 1u << 5, kDfExport = 1u << 6, kDf
 // anything beyond "the previous op of the program is the only input"
 constexpr uint32_t kDfSlowMask = 0xFFFFFF00u | kDfComm | kDfExport | kDfTwoHop;
 constexpr uint32_t kDfDirectMembers = 8;  // larger groups gather at their first member
+// a comm op whose members are the ranks of one block: its slot word holds this
+// flag and the op's sequence number among the block's joins (shared-memory join)
+constexpr uint32_t kDfBlockJoin = 0x80000000u;
+constexpr int kDfMaxWarpsPerBlock = 8;
 
 struct DataflowArgs {
   int32_t S, G, R, n_streams;  // scenarios, groups of 32 scenarios, ranks, timelines per rank
@@ -212,11 +214,12 @@ struct DataflowArgs {
   int64_t skip_slot;           // failure injection for tests: this partial is never published (-1: none)
   int64_t n_opnd;              // words of opnd
   int32_t dbg;                 // debug bounds: check every index (echo_bounds.h)
+  int32_t wpb;                 // warps per block (consecutive ranks of one scenario group)
 };
 cudaError_t launch_compose_dataflow(const DataflowArgs &a, cudaStream_t st);
-size_t dataflow_smem_bytes(int32_t n_streams);
+size_t dataflow_smem_bytes(int32_t n_streams, int32_t wpb);
 // whether every warp of R * G warps can be resident at once (cooperative launch)
-bool dataflow_fits(int64_t n_warps, int32_t n_streams, int device);
+bool dataflow_fits(int64_t n_warps, int32_t n_streams, int32_t wpb, int device);
 
 // shared memory of an overlap-test block: each warp's ring of candidate rows
 inline size_t overlap_smem_bytes() { return (size_t)kOvWarps * kOvDepth * kOvBatch * 2 * 32 * sizeof(int64_t); }
