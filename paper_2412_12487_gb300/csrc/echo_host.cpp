@@ -1740,17 +1740,22 @@ int echo_load_scenarios(echo_ctx *c, const echo_scen_desc *sc) {
   }
   const int64_t V = B.V;
   // The dataflow composer (rows of 32 scenarios, a warp per rank) is serial in
-  // the length of the longest rank program, the levelled ones in their number
-  // of steps; measured on GB300 a program entry costs about 0.25-0.55 us and a
-  // step about 1.2-1.8 us, so it is chosen when the longest program is shorter
-  // than 2.5 steps per entry (and every warp can be resident).
+  // the length of the longest rank program, the levelled ones in their number of
+  // steps.  Measured on GB300: a program entry costs about 0.22 us while at most
+  // 8 warps share an SM, and proportionally more beyond (0.24 us on GPT-1.3B x 256,
+  // 0.37 us at 13.5 warps per SM on the 1024-rank workload, 0.52 us at 20 on
+  // GPT-175B x 1024); a levelled step costs about 1.1 us.  The cheaper estimate
+  // wins (when every warp can be resident).
   const int32_t n_groups = (S + 31) / 32;
   bool use_df = false;
   if (B.df_ok && (c->kernel_choice == 0 || c->kernel_choice == 4) &&
       echo::dataflow_fits((int64_t)B.R * n_groups, B.NS, B.df_wpb, c->device)) {
     int64_t longest = 0;
     for (int32_t r = 0; r < B.R; ++r) longest = std::max(longest, B.df_off[r + 1] - B.df_off[r]);
-    use_df = c->kernel_choice == 4 || 2 * longest < 5 * make_steps(B, kStepNodes).L;
+    const double warps_per_sm = (double)B.R * n_groups / std::max(c->sms, 1);
+    const double df_us = (double)longest * 0.22 * std::max(1.0, warps_per_sm / 8.0);
+    const double lev_us = (double)make_steps(B, kStepNodes).L * 1.1;
+    use_df = c->kernel_choice == 4 || df_us < lev_us;
   }
   const int sigma = use_df ? 32 : pick_sigma(S, c->sms);
   int slog2 = 0;

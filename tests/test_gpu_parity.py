@@ -388,7 +388,12 @@ def test_high_fan_in_collective_and_global_frontier():
         assert_same(got, oracle.compose(g, sc), g)
 
 
-def test_many_scenarios_several_waves():
+@pytest.mark.parametrize("kernel", ["pipelined", "auto"])
+def test_many_scenarios_several_waves(kernel, monkeypatch):
+    # 3001 scenarios: the levelled composer at its widest blocks (sigma 16, 188
+    # blocks: more than one wave), and whichever composer the cost model picks
+    if kernel != "auto":
+        monkeypatch.setenv("ECHO_COMPOSE_KERNEL", kernel)
     c = W.config("tiny")
     g = W.build_gpt_graph(c)
     cr = W.GPTConfig(**{**c.__dict__, "fixed_scenario": False})
@@ -396,7 +401,8 @@ def test_many_scenarios_several_waves():
     got = run_gpu(g, sc)
     want = oracle.compose(g, sc, threads=THREADS)
     assert_same(got, want, g)
-    assert got["info"]["sigma"] == 16
+    if kernel != "auto":
+        assert got["info"]["sigma"] == 16
 
 
 def test_cc_queries_match_oracle():

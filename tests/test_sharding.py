@@ -86,3 +86,48 @@ def test_two_gloo_ranks_compose_their_slices_and_gather(tmp_path):
     assert np.array_equal(got["ov"], want.overlapped)
     # max over ranks: [1, 10, 4] from ranks holding 4 and 3 scenarios
     assert got["t"].tolist() == [1.0, 10.0, 4.0]
+
+
+def _gpu_worker(rank, world, port, out_path):
+    # the same rank logic with each rank composing its slice through the library on
+    # cuda:0 (independent compositions, one context per process)
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    import torch.distributed as dist
+    from paper_2412_12487_gb300 import Echo
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        g, full = _batch()
+        s0, s1 = SH.shard_bounds(N_TOTAL, world, rank)
+        with Echo(0) as e:
+            e.load_graph(g)
+            e.load_scenarios(SH.slice_scenarios(full, s0, s1))
+            e.estimate_collectives()
+            e.compose(refine_passes=1)
+            st, fn = e.read_times()
+            mk = e.read_makespan()
+            ov = e.read_overlap()
+        mk = SH.gather_scenarios(mk, N_TOTAL)
+        fin = SH.gather_scenarios(fn, N_TOTAL)
+        sta = SH.gather_scenarios(st, N_TOTAL)
+        ov = SH.gather_scenarios(ov, N_TOTAL)
+        if rank == 0:
+            np.savez(out_path, mk=mk, fin=fin, st=sta, ov=ov)
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.gpu
+def test_two_gloo_ranks_compose_their_slices_through_the_library(tmp_path):
+    import torch.multiprocessing as mp
+    import oracle
+    oracle.build()
+    out = str(tmp_path / "rank0.npz")
+    mp.start_processes(_gpu_worker, args=(2, _free_port(), out), nprocs=2, join=True, start_method="spawn")
+    got = np.load(out)
+    g, full = _batch()
+    want = oracle.compose(g, full, refine_passes=1)
+    assert np.array_equal(got["mk"], want.makespan)
+    assert np.array_equal(got["fin"], want.finish)
+    assert np.array_equal(got["st"], want.start)
+    assert np.array_equal(got["ov"], want.overlapped)
