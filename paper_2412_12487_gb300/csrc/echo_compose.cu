@@ -200,7 +200,10 @@ __device__ __noinline__ bool segment_ok(const StagedArgs &a, uint32_t first, uin
 
 // Compose the segments of one segment level (shared by the staged and the
 // pipelined kernels).  Segment k's header and entries are in the record ring at
-// word `ro`; its rows are i0 + header.z ... in the duration ring.  Thread `sub`
+// word `ro`; its rows are i0 + header.z ... (global rows), held in the duration
+// ring of RR rows from ring row dpos0 + header.z on (wrapping).  Candidate rows of
+// the level start at level-order index c0, in ring row cpos0 of the CRR-row
+// candidate ring.  Thread `sub`
 // handles segments sub, sub + step, ... for scenario lanes j0 .. j0+LANES-1; the
 // segments of a level come heaviest first, so a warp's lanes hold segments of
 // similar weight.  Every input of a head is the tail of an earlier segment: the
@@ -213,8 +216,9 @@ template <int SIGMA, int LANES, bool STORE_ALL, bool DBG>
 __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t ro, uint32_t i0, uint32_t seg0,
                                                  int32_t nseg, int sub, int step, int j0, int64_t *vr,
                                                  const int64_t *dr, const uint32_t *rr, uint32_t vmask,
-                                                 uint32_t dmask, uint32_t rmask, int64_t (&mk)[LANES],
-                                                 const int64_t *cr = nullptr, uint32_t cmask = 0) {
+                                                 uint32_t dpos0, uint32_t RR, uint32_t rmask, int64_t (&mk)[LANES],
+                                                 const int64_t *cr = nullptr, uint32_t cpos0 = 0, uint32_t c0 = 0,
+                                                 uint32_t CRR = 0) {
   int64_t *fb = a.f + ((int64_t)blockIdx.x * a.n_rows) * SIGMA;
   const uint32_t vr_a = saddr(vr) + j0 * 8, dr_a = saddr(dr) + j0 * 8;
   const uint32_t rr_a = saddr(rr);
@@ -245,9 +249,13 @@ __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t r
       }
     }
     // a candidate's duration comes from the candidate ring instead of the duration ring
+    // (the level's candidates span at most CRR rows, so one wrap suffices)
     auto patch = [&](uint32_t t, int64_t (&d)[LANES]) {
-      if ((cmask_bits >> t) & 1)
-        s_load<LANES>(cr_a + ((c_first + (uint32_t)__popcll(cmask_bits & ((1ull << t) - 1))) & cmask) * kRowBytes, d);
+      if ((cmask_bits >> t) & 1) {
+        uint32_t x = cpos0 + (c_first - c0) + (uint32_t)__popcll(cmask_bits & ((1ull << t) - 1));
+        if (x >= CRR) x -= CRR;
+        s_load<LANES>(cr_a + x * kRowBytes, d);
+      }
     };
     const uint32_t e = ro + hd.x;
     const uint32_t first = i0 + hd.z;
@@ -274,15 +282,21 @@ __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t r
       g_max<LANES>(fv, fb + (int64_t)u0 * SIGMA + j0);
       g_max<LANES>(fv, fb + (int64_t)u1 * SIGMA + j0);
     }
-    // along the chain every op starts when the previous one ends
+    // along the chain every op starts when the previous one ends; p is the ring
+    // row of chain position t (a level's rows span at most RR rows)
     int64_t *gp = fb + (int64_t)first * SIGMA + j0;
+    uint32_t p = dpos0 + hd.z;
+    if (p >= RR) p -= RR;
+    auto next = [&](uint32_t x) { return x + 1 == RR ? 0u : x + 1; };
     uint32_t t = 0;
     for (; t + 4 <= len; t += 4, gp += 4 * SIGMA) {
       int64_t d0[LANES], d1[LANES], d2[LANES], d3[LANES];
-      s_load<LANES>(dr_a + ((first + t) & dmask) * kRowBytes, d0);
-      s_load<LANES>(dr_a + ((first + t + 1) & dmask) * kRowBytes, d1);
-      s_load<LANES>(dr_a + ((first + t + 2) & dmask) * kRowBytes, d2);
-      s_load<LANES>(dr_a + ((first + t + 3) & dmask) * kRowBytes, d3);
+      const uint32_t p1 = next(p), p2 = next(p1), p3 = next(p2);
+      s_load<LANES>(dr_a + p * kRowBytes, d0);
+      s_load<LANES>(dr_a + p1 * kRowBytes, d1);
+      s_load<LANES>(dr_a + p2 * kRowBytes, d2);
+      s_load<LANES>(dr_a + p3 * kRowBytes, d3);
+      p = next(p3);
       if (cmask_bits) {
         patch(t, d0);
         patch(t + 1, d1);
@@ -303,9 +317,9 @@ __device__ __forceinline__ void compose_segments(const StagedArgs &a, uint32_t r
       for (int j = 0; j < LANES; ++j) fv[j] += d3[j];
       if (STORE_ALL || (sb & 8)) g_store<LANES>(gp + 3 * SIGMA, fv);
     }
-    for (; t < len; ++t, gp += SIGMA) {
+    for (; t < len; ++t, gp += SIGMA, p = next(p)) {
       int64_t d[LANES];
-      s_load<LANES>(dr_a + ((first + t) & dmask) * kRowBytes, d);
+      s_load<LANES>(dr_a + p * kRowBytes, d);
       if (cmask_bits) patch(t, d);
 #pragma unroll
       for (int j = 0; j < LANES; ++j) fv[j] += d[j];
@@ -336,9 +350,9 @@ compose_staged_kernel(StagedArgs a) {
   const int32_t S = a.S;
   const int32_t s0 = blockIdx.x * SIGMA;
   const int tid = threadIdx.x;
-  const StagedLayout lay = staged_layout(SIGMA, a.vlog2, a.dlog2, a.rlog2, a.clog2);
   const uint32_t vmask = (1u << a.vlog2) - 1, dmask = (1u << a.dlog2) - 1, rmask = (1u << a.rlog2) - 1;
   const uint32_t RR = dmask + 1, RB = rmask + 1;
+  const StagedLayout lay = staged_layout(SIGMA, a.vlog2, RR, a.rlog2, (size_t)1 << a.clog2);
   int64_t *mk_s = reinterpret_cast<int64_t *>(sbuf);                  // [SIGMA]
   uint2 *hist = reinterpret_cast<uint2 *>(sbuf + lay.hist);           // [16] (rows, words) copied by group
   uint32_t *meta_s = reinterpret_cast<uint32_t *>(sbuf + lay.meta);   // [2][kMetaCap][4]
@@ -419,13 +433,13 @@ compose_staged_kernel(StagedArgs a) {
     const int32_t nseg = (int32_t)(mb[4 + 2] - seg0);
     if (a.dbg)
       compose_segments<SIGMA, LANES, true, true>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr,
-                                                 vmask, dmask, rmask, mk);
+                                                 vmask, i0 & dmask, RR, rmask, mk);
     else if (a.store_all)
       compose_segments<SIGMA, LANES, true, false>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr,
-                                                  vmask, dmask, rmask, mk);
+                                                  vmask, i0 & dmask, RR, rmask, mk);
     else
       compose_segments<SIGMA, LANES, false, false>(a, ro, i0, seg0, nseg, tid / TPN, THREADS / TPN, j0, vr, dr, rr,
-                                                   vmask, dmask, rmask, mk);
+                                                   vmask, i0 & dmask, RR, rmask, mk);
     prev_i0 = i0;
     prev_ro = ro;
   }
@@ -482,14 +496,17 @@ __device__ __forceinline__ bool named_barrier_or(int id, int threads, bool flag)
 // segment level's duration rows, record block and metadata into the rings with the
 // TMA engine (at most five 1-D bulk copies per level: this block's rows of a level
 // are contiguous), as far ahead as the rings allow; kPipeConsumerWarps warps
-// compose.  Stage l % kPipeStages has a "full" mbarrier (armed with the level's
+// compose, one scenario per thread up to SIGMA 8 (a segment's SIGMA threads
+// share its walk), two above.  The duration and candidate rings hold any number
+// of rows (a.d_rows, a.c_rows: all the shared memory the rest leaves), so the
+// producer writes each level's first ring rows beside its metadata.  Stage l % kPipeStages has a "full" mbarrier (armed with the level's
 // byte count) and an "empty" mbarrier (one arrival per consumer warp once the
 // level is composed).  Every wait is bounded: on expiry the block records
 // kDevTimeout, stops, and lets its copies in flight land first.
 template <int SIGMA, bool STORE_ALL, bool DBG>
 __global__ void __launch_bounds__((kPipeConsumerWarps + 1) * 32)
 compose_pipelined_kernel(StagedArgs a) {
-  constexpr int LANES = 2;
+  constexpr int LANES = SIGMA <= 8 ? 1 : 2;
   constexpr int TPN = SIGMA / LANES;  // threads per segment
   constexpr int NB = kPipeStages;
   constexpr int NCT = kPipeConsumerWarps * 32;
@@ -497,14 +514,15 @@ compose_pipelined_kernel(StagedArgs a) {
   const int32_t S = a.S;
   const int32_t s0 = blockIdx.x * SIGMA;
   const int tid = threadIdx.x;
-  const StagedLayout lay = staged_layout(SIGMA, a.vlog2, a.dlog2, a.rlog2, a.clog2);
-  const uint32_t vmask = (1u << a.vlog2) - 1, dmask = (1u << a.dlog2) - 1, rmask = (1u << a.rlog2) - 1;
-  const uint32_t RR = dmask + 1, RB = rmask + 1, CRR = 1u << a.clog2;
+  const StagedLayout lay = staged_layout(SIGMA, a.vlog2, a.d_rows, a.rlog2, a.c_rows);
+  const uint32_t vmask = (1u << a.vlog2) - 1, rmask = (1u << a.rlog2) - 1;
+  const uint32_t RR = a.d_rows, RB = rmask + 1, CRR = a.c_rows;
   int64_t *mk_s = reinterpret_cast<int64_t *>(sbuf);                       // [SIGMA]
   uint64_t *full = reinterpret_cast<uint64_t *>(sbuf + lay.meta);          // [NB]
   uint64_t *empty = full + NB;                                              // [NB]
   uint32_t *hist = reinterpret_cast<uint32_t *>(sbuf + lay.meta + 256);    // [NB][4] producer only
   uint32_t *metas = reinterpret_cast<uint32_t *>(sbuf + lay.meta + 512);   // [NB][8]
+  uint32_t *pos = reinterpret_cast<uint32_t *>(sbuf + lay.meta + 1024);    // [NB][2] first ring rows
   int64_t *vr = reinterpret_cast<int64_t *>(sbuf + lay.vr);
   int64_t *dr = reinterpret_cast<int64_t *>(sbuf + lay.dr);
   uint32_t *rr = reinterpret_cast<uint32_t *>(sbuf + lay.rr);
@@ -527,14 +545,18 @@ compose_pipelined_kernel(StagedArgs a) {
     if (lane == 0) {
       const int64_t *durb = a.dur + ((int64_t)blockIdx.x * a.n_rows) * SIGMA;
       const int64_t *cdb = a.cdur ? a.cdur + ((int64_t)blockIdx.x * a.n_cand) * SIGMA : nullptr;
-      const uint32_t emask = RR * SIGMA - 1, cemask = CRR * SIGMA - 1;
       int32_t c_known = 0;  // every level < c_known has been composed
       int32_t issued = 0;   // levels [0, issued) have been armed
       bool fail = false;
+      // metadata of levels l and l+1, and l+2 in flight (its load latency overlaps a level)
+      uint4 m_cur = *reinterpret_cast<const uint4 *>(a.meta);
+      uint4 m_nxt = *reinterpret_cast<const uint4 *>(a.meta + 4 * min(1, a.L));
       for (int32_t l = 0; l < a.L; ++l) {
         if (l == a.skip_level) break;  // failure injection: level l never arrives
-        const uint4 m0 = *reinterpret_cast<const uint4 *>(a.meta + 4 * l);
-        const uint4 m1 = *reinterpret_cast<const uint4 *>(a.meta + 4 * (l + 1));
+        const uint4 m_fut = *reinterpret_cast<const uint4 *>(a.meta + 4 * min(l + 2, a.L));
+        const uint4 m0 = m_cur, m1 = m_nxt;
+        m_cur = m_nxt;
+        m_nxt = m_fut;
         uint32_t ro = m0.x, i0 = m0.y, ro1 = m1.x, i1 = m1.y;
         uint32_t c0 = cdb ? m0.w : 0, c1 = cdb ? m1.w : 0;  // the level's candidate rows
         if (DBG && !(range_ok(i0, i1, a.n_rows) && range_ok(ro, ro1, a.n_words) && range_ok(c0, c1, a.n_cand))) {
@@ -556,17 +578,22 @@ compose_pipelined_kernel(StagedArgs a) {
         hist[4 * (l % NB)] = i0;
         hist[4 * (l % NB) + 1] = ro;
         hist[4 * (l % NB) + 2] = c0;
+        // ring rows of the level's first row and first candidate (read by the
+        // consumers after the level's full barrier, which this arrival releases)
+        const uint32_t dp = i0 % RR, cp = CRR ? c0 % CRR : 0;
+        pos[2 * (l % NB)] = dp;
+        pos[2 * (l % NB) + 1] = cp;
         uint64_t *bar = &full[l % NB];
         const uint32_t e0 = i0 * SIGMA, ne = (i1 - i0) * SIGMA, w0 = ro & rmask, nw = ro1 - ro;
         const uint32_t ce0 = c0 * SIGMA, nce = (c1 - c0) * SIGMA;
         mbar_arrive_expect_tx(bar, ne * 8 + nw * 4 + 32 + nce * 8);
         if (nce) {
-          const uint32_t nce1 = min(nce, cemask + 1 - (ce0 & cemask));
-          bulk_g2s(cr + (ce0 & cemask), cdb + ce0, nce1 * 8, bar);
+          const uint32_t nce1 = min(nce, (CRR - cp) * SIGMA);
+          bulk_g2s(cr + cp * SIGMA, cdb + ce0, nce1 * 8, bar);
           if (nce1 < nce) bulk_g2s(cr, cdb + ce0 + nce1, (nce - nce1) * 8, bar);
         }
-        const uint32_t ne1 = min(ne, emask + 1 - (e0 & emask));
-        bulk_g2s(dr + (e0 & emask), durb + e0, ne1 * 8, bar);
+        const uint32_t ne1 = min(ne, (RR - dp) * SIGMA);
+        bulk_g2s(dr + dp * SIGMA, durb + e0, ne1 * 8, bar);
         if (ne1 < ne) bulk_g2s(dr, durb + e0 + ne1, (ne - ne1) * 8, bar);
         const uint32_t nw1 = min(nw, RB - w0);
         bulk_g2s(rr + w0, a.recs + ro, nw1 * 4, bar);
@@ -583,15 +610,19 @@ compose_pipelined_kernel(StagedArgs a) {
   } else {
     // ---------------- consumer warps ----------------
     const int j0 = (tid % TPN) * LANES;
-    int64_t mk[LANES] = {0, 0};
+    int64_t mk[LANES];
+#pragma unroll
+    for (int j = 0; j < LANES; ++j) mk[j] = 0;
     for (int32_t l = 0; l < a.L; ++l) {
       const bool ok = mbar_wait(&full[l % NB], (l / NB) & 1, a.wait_limit_cycles);
       if (ok) {
         const uint32_t *mb = metas + 8 * (l % NB);
-        const uint32_t ro = mb[0], i0 = mb[1], seg0 = mb[2];
+        const uint32_t ro = mb[0], i0 = mb[1], seg0 = mb[2], c0 = mb[3];
         const int32_t nseg = (int32_t)(mb[4 + 2] - seg0);
+        const uint32_t dp = pos[2 * (l % NB)], cp = pos[2 * (l % NB) + 1];
         compose_segments<SIGMA, LANES, STORE_ALL, DBG>(a, ro, i0, seg0, nseg, tid / TPN, NCT / TPN, j0, vr, dr,
-                                                       rr, vmask, dmask, rmask, mk, a.cdur ? cr : nullptr, CRR - 1);
+                                                       rr, vmask, dp, RR, rmask, mk, a.cdur ? cr : nullptr, cp,
+                                                       c0, CRR);
       }
       // every consumer learns, in the same barrier, whether any of them gave up
       if (named_barrier_or(1, NCT, !ok)) {
@@ -639,10 +670,12 @@ cudaError_t launch_pipelined_t(const StagedArgs &a, const StagedPlan &plan, cuda
   // debug bounds runs the checking variant, which stores every finish
   auto k = a.dbg ? compose_pipelined_kernel<SIGMA, true, true>
                  : a.store_all ? compose_pipelined_kernel<SIGMA, true, false> : compose_pipelined_kernel<SIGMA, false, false>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem);
+  (void)plan;
+  const size_t smem = staged_layout(SIGMA, a.vlog2, a.d_rows, a.rlog2, a.c_rows).total;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid((a.S + SIGMA - 1) / SIGMA);
-  k<<<grid, (kPipeConsumerWarps + 1) * 32, plan.smem, st>>>(a);
+  k<<<grid, (kPipeConsumerWarps + 1) * 32, smem, st>>>(a);
   return cudaGetLastError();
 }
 

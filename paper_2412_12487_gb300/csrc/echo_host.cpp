@@ -1160,7 +1160,7 @@ echo::StagedPlan plan_staged(const GraphBuild &b, const Steps &st, int sigma, si
   for (int d = dmin + 2; d >= dmin; --d)
     for (int v = vwant; v >= 6; --v)
       for (int r = rmin + 1; r >= rmin; --r) {
-        const size_t need = echo::staged_layout(sigma, v, d, r, cring).total;
+        const size_t need = echo::staged_layout(sigma, v, (size_t)1 << d, r, (size_t)1 << cring).total;
         if (need <= smem_cap && d < 31 && r < 31 && cring < 31) {
           best.ok = true;
           best.dring_log2 = d;
@@ -1168,6 +1168,13 @@ echo::StagedPlan plan_staged(const GraphBuild &b, const Steps &st, int sigma, si
           best.rring_log2 = r;
           best.cring_log2 = cring;
           best.smem = need;
+          // the pipelined kernel's duration ring takes every row the rest leaves:
+          // more levels in flight hide more of each level's copy latency
+          const int64_t row = (int64_t)sigma * 8, fixed = (int64_t)echo::staged_layout(sigma, v, 0, r, 0).total;
+          const int64_t crows = std::max<int64_t>(crows2, 2), room = (int64_t)smem_cap - fixed;
+          best.pipe_crows = (uint32_t)crows;
+          best.pipe_drows = (uint32_t)std::max<int64_t>(room / row, (int64_t)1 << d);
+          best.pipe_drows_c = (uint32_t)std::max<int64_t>((room - crows * row) / row, (int64_t)1 << d);
           return best;
         }
       }
@@ -2036,6 +2043,8 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       a.dlog2 = c->plan.dring_log2;
       a.rlog2 = c->plan.rring_log2;
       a.clog2 = c->plan.cring_log2;
+      a.d_rows = (uint32_t)1 << c->plan.dring_log2;
+      a.c_rows = (uint32_t)1 << c->plan.cring_log2;
       a.meta = c->d_meta;
       a.recs = c->d_recs;
       a.dur = d;
@@ -2049,6 +2058,10 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
       a.store_all = final_pass;
       a.dbg = dbg;
       const bool pipe = c->plan.pipelined && (c->kernel_choice == 0 || c->kernel_choice == 3);
+      if (pipe) {
+        a.d_rows = cdur ? c->plan.pipe_drows_c : c->plan.pipe_drows;
+        a.c_rows = cdur ? c->plan.pipe_crows : 0;
+      }
       if (pipe)
         return timed(c, name, [&] { return echo::launch_compose_pipelined(a, c->sigma, c->plan, c->stream); });
       return timed(c, name, [&] { return echo::launch_compose_staged(a, c->sigma, c->plan, c->stream); });

@@ -97,6 +97,7 @@ struct StagedArgs {
   int32_t S, L;                  // L: segment levels
   uint32_t n_rows, n_words;      // nodes; words of all record blocks
   int32_t vlog2, dlog2, rlog2;   // log2 sizes: value ring (segments), duration ring (rows), record ring (words)
+  uint32_t d_rows, c_rows;       // ring sizes in rows (any size): duration and candidate rings
   const uint32_t *meta;          // [4*(L+1)]: record word offset, first node, first segment, first candidate
   const uint32_t *recs;          // record blocks
   const int64_t *dur;            // durations (MatLayout)
@@ -105,7 +106,7 @@ struct StagedArgs {
   // pipelined kernel only
   const int64_t *cdur;           // validator durations of the candidates ([n_cand] rows per block), or null
   uint32_t n_cand;               // overlap candidates
-  int32_t clog2;                 // log2 rows of the candidate ring
+  int32_t clog2;                 // log2 rows of the candidate ring (staged kernel)
   int32_t *status;               // device status word (kDevTimeout when a bounded wait gives up)
   long long wait_limit_cycles;   // bound of every mbarrier wait, in SM clock cycles
   int32_t skip_level;            // failure injection for tests: this level is never filled (-1: none)
@@ -121,6 +122,10 @@ struct StagedPlan {
   int vring_log2 = 0, dring_log2 = 0, rring_log2 = 0;  // sizes (segments, rows, words)
   int cring_log2 = 0;  // candidate ring (rows of the validator's durations, pipelined kernel)
   size_t smem = 0;
+  // the pipelined kernel's rings take rows of any count, so they fill the shared
+  // memory left: without a candidate ring (a composition with the original
+  // durations) and with one (a composition that reads the validator's)
+  uint32_t pipe_drows = 0, pipe_drows_c = 0, pipe_crows = 0;
 };
 
 // Shared-memory layout of the staged kernels (byte offsets).  Every region starts
@@ -129,15 +134,16 @@ struct StagedLayout {
   size_t hist, meta, vr, dr, rr, cr, total;
 };
 __host__ __device__ inline size_t round16(size_t x) { return (x + 15) & ~(size_t)15; }
-__host__ __device__ inline StagedLayout staged_layout(int sigma, int vlog2, int dlog2, int rlog2, int clog2) {
+// d_rows, c_rows: rows of the duration and candidate rings.
+__host__ __device__ inline StagedLayout staged_layout(int sigma, int vlog2, size_t d_rows, int rlog2, size_t c_rows) {
   StagedLayout L;
   L.hist = 128;                        // [0, 128): per-scenario makespans
   L.meta = L.hist + 16 * 8;            // 16 copy-group extents
   L.vr = L.meta + round16((size_t)2 * kMetaCap * 16);
   L.dr = L.vr + round16(((size_t)1 << vlog2) * sigma * 8);
-  L.rr = L.dr + round16(((size_t)1 << dlog2) * sigma * 8);
+  L.rr = L.dr + round16(d_rows * sigma * 8);
   L.cr = L.rr + round16(((size_t)1 << rlog2) * 4);
-  L.total = L.cr + round16(((size_t)1 << clog2) * sigma * 8);
+  L.total = L.cr + round16(c_rows * sigma * 8);
   return L;
 }
 
