@@ -498,8 +498,8 @@ def _full_batch_parity(name, time_cols, refine=1):
 @pytest.mark.slow
 def test_gpt175b_full_batch_bit_exact():
     # all 1024 makespans; every op in 128 scenarios, one in each scenario block of
-    # the levelled composer (sigma 8) and every lane position of a block (both
-    # lanes of every thread) sixteen times over
+    # the levelled composer (sigma 8) and every scenario position of a block
+    # sixteen times over
     info = _full_batch_parity("gpt175b", [8 * b + b % 8 for b in range(128)])
     assert info["sigma"] == 8
 
