@@ -236,28 +236,38 @@ __global__ void __launch_bounds__(kDfMaxWarpsPerBlock * 32, 2) compose_dataflow_
     asm volatile("cp.async.wait_group 3;" ::: "memory");  // this batch's group is complete
     const int64_t *d0 = dring + ((b - e0) / kDfBatch % (kDfDepth + 1)) * (kDfBatch * 32) + lane;
     const int n_here = e1 - b < kDfBatch ? (int)(e1 - b) : kDfBatch;
+    // the batch's node ids, headers and durations in registers: their shuffles and
+    // loads issue together, before any of the batch's stores (entries past the
+    // program's end read zero words and an unused ring slot)
+    uint32_t ev[kDfBatch], eh[kDfBatch];
+    int64_t ed[kDfBatch];
+#pragma unroll
+    for (int j = 0; j < kDfBatch; ++j) {
+      ev[j] = __shfl_sync(kFull, w0.x, 4 * j);
+      eh[j] = __shfl_sync(kFull, w0.x, 4 * j + 1);
+      ed[j] = d0[j * 32];
+    }
     // a full batch of common ops (inputs: the previous op at most) runs branch-free
     bool plain = n_here == kDfBatch;
 #pragma unroll
-    for (int j = 0; j < kDfBatch; ++j) plain &= (__shfl_sync(kFull, w0.x, 4 * j + 1) & kDfSlowMask) == 0;
+    for (int j = 0; j < kDfBatch; ++j) plain &= (eh[j] & kDfSlowMask) == 0;
     if (plain) {
 #pragma unroll
       for (int j = 0; j < kDfBatch; ++j) {
-        const uint32_t v = __shfl_sync(kFull, w0.x, 4 * j), hdr = __shfl_sync(kFull, w0.x, 4 * j + 1);
-        cur = ((hdr & kDfPrev) ? cur : 0) + d0[j * 32];
-        f[(int64_t)v << 5] = cur;
-        last[(hdr & 15) * 32] = cur;
+        cur = ((eh[j] & kDfPrev) ? cur : 0) + ed[j];
+        f[(int64_t)ev[j] << 5] = cur;
+        last[(eh[j] & 15) * 32] = cur;
         mx = max(mx, cur);
       }
     } else {
 #pragma unroll
     for (int j = 0; j < kDfBatch; ++j) {
       if (j >= n_here) break;
-      const uint32_t v = __shfl_sync(kFull, w0.x, 4 * j);
-      const uint32_t hdr = __shfl_sync(kFull, w0.x, 4 * j + 1);
+      const uint32_t v = ev[j];
+      const uint32_t hdr = eh[j];
       int64_t t = (hdr & kDfPrev) ? cur : 0;
       if ((hdr & kDfSlowMask) == 0) {  // the common op: its inputs are the previous op at most
-        cur = t + d0[j * 32];
+        cur = t + ed[j];
         f[(int64_t)v << 5] = cur;
         last[(hdr & 15) * 32] = cur;
         mx = max(mx, cur);
@@ -277,7 +287,7 @@ __global__ void __launch_bounds__(kDfMaxWarpsPerBlock * 32, 2) compose_dataflow_
           return;
         }
       }
-      int64_t fv = t + d0[j * 32];
+      int64_t fv = t + ed[j];
       if (hdr & kDfComm) {
         const uint32_t slot = __shfl_sync(kFull, w0.x, 4 * j + 2), nmme = __shfl_sync(kFull, w0.y, 4 * j + 2);
         const uint32_t nm = nmme & 0xFFFF, me = nmme >> 16;
@@ -286,7 +296,7 @@ __global__ void __launch_bounds__(kDfMaxWarpsPerBlock * 32, 2) compose_dataflow_
             asm volatile("cp.async.wait_all;" ::: "memory");
             return;
           }
-          fv = t + d0[j * 32];
+          fv = t + ed[j];
         } else if (nm > 1) {
           if (a.skip_slot != (int64_t)slot + me) st_relaxed_u64(part + ((int64_t)(slot + me) << 5), tag | (uint64_t)t);
           if (!(hdr & kDfTwoHop) || me == 0) {
@@ -295,7 +305,7 @@ __global__ void __launch_bounds__(kDfMaxWarpsPerBlock * 32, 2) compose_dataflow_
                 asm volatile("cp.async.wait_all;" ::: "memory");
                 return;
               }
-            fv = t + d0[j * 32];
+            fv = t + ed[j];
           } else {  // the first member gathers and publishes the finish
             int64_t u = 0;
             if (!df_gather(xval + ((int64_t)__shfl_sync(kFull, w0.x, 4 * j + 3) << 5), 1, ~0u, tag, u, a)) {
