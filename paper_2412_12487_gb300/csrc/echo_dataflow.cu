@@ -162,9 +162,9 @@ __device__ bool block_join(uint64_t *bjoin, uint32_t seq, uint32_t me, uint32_t 
   }
 }
 
-__device__ __forceinline__ void cp_async_8(void *smem, const void *gmem) {
+__device__ __forceinline__ void cp_async_16(void *smem, const void *gmem) {
   const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(sa), "l"(gmem) : "memory");
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sa), "l"(gmem) : "memory");
 }
 
 template <bool CAND>
@@ -187,8 +187,8 @@ __global__ void __launch_bounds__(kDfMaxWarpsPerBlock * 32, 2) compose_dataflow_
   int64_t *last = df_last + lane;
   for (int k = 0; k < a.n_streams; ++k) last[k * 32] = 0;
   // rows of 32 scenarios: element (i, s) of an [n][S] matrix at ((g * n + i) << 5) + lane
-  const int64_t *dur = a.dur + (((int64_t)g * a.V) << 5) + lane;
-  const int64_t *cdu = CAND ? a.cdur + (((int64_t)g * a.n_cand) << 5) + lane : nullptr;
+  const int64_t *dur = a.dur + (((int64_t)g * a.V) << 5);
+  const int64_t *cdu = CAND ? a.cdur + (((int64_t)g * a.n_cand) << 5) : nullptr;
   int64_t *f = a.f + (((int64_t)g * a.V) << 5) + lane;
   uint64_t *part = a.part + (((int64_t)g * a.n_slots) << 5) + lane;
   uint64_t *xval = a.xval + (((int64_t)g * a.n_exports) << 5) + lane;
@@ -196,18 +196,25 @@ __global__ void __launch_bounds__(kDfMaxWarpsPerBlock * 32, 2) compose_dataflow_
   const int64_t e0 = a.off[r], e1 = a.off[r + 1];
   int64_t mx = 0;
   // batches of 8 entries of 8 words: lane l holds words 2(l % 4) and 2(l % 4) + 1
-  // of entry l / 4.  Records are loaded kDfDepth + 1 batches ahead of their use;
-  // each lane copies its own duration elements kDfDepth batches ahead into the
-  // ring (cp.async, one commit group per batch), and reads only its own.
+  // of entry l / 4.  Records are loaded kDfDepth + 1 batches ahead of their use,
+  // durations kDfDepth batches ahead into the ring (cp.async, one commit group per
+  // batch): lane l copies 16 bytes, the scenarios 2(l % 16) and 2(l % 16) + 1, of
+  // entries 2k + l / 16.  A lane reads elements other lanes copied, so the warp
+  // synchronizes after its wait for a batch's group, and before it overwrites the
+  // slot the previous batch was read from.
   auto rec = [&](int64_t b) -> uint2 {
     return b + lane / 4 < e1 ? __ldg(reinterpret_cast<const uint2 *>(a.rec) + 4 * b + lane) : make_uint2(0, 0);
   };
   auto durs = [&](int64_t b, uint2 w) {  // copies batch b's durations into its ring slot
-    int64_t *slot = dring + ((b - e0) / kDfBatch % (kDfDepth + 1)) * (kDfBatch * 32) + lane;
+    int64_t *slot = dring + ((b - e0) / kDfBatch % (kDfDepth + 1)) * (kDfBatch * 32) + (lane & 15) * 2;
+    __syncwarp();
 #pragma unroll
-    for (int j = 0; j < kDfBatch; ++j) {
-      const uint32_t v = __shfl_sync(kFull, w.x, 4 * j), ci = __shfl_sync(kFull, w.y, 4 * j);
-      if (b + j < e1) cp_async_8(slot + j * 32, (CAND && ci != ~0u) ? cdu + ((int64_t)ci << 5) : dur + ((int64_t)v << 5));
+    for (int k = 0; k < kDfBatch / 2; ++k) {
+      const int j = 2 * k + (lane >> 4);
+      const uint32_t v = __shfl_sync(kFull, w.x, 4 * j), ci = CAND ? __shfl_sync(kFull, w.y, 4 * j) : ~0u;
+      if (b + j < e1)
+        cp_async_16(slot + j * 32, ((CAND && ci != ~0u) ? cdu + ((int64_t)ci << 5) : dur + ((int64_t)v << 5)) +
+                                       (lane & 15) * 2);
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
   };
@@ -233,7 +240,8 @@ __global__ void __launch_bounds__(kDfMaxWarpsPerBlock * 32, 2) compose_dataflow_
     const uint2 w4 = rec(b + 4 * kDfBatch);
     if (bad_batch(b + 3 * kDfBatch, w3)) return;
     durs(b + 3 * kDfBatch, w3);
-    asm volatile("cp.async.wait_group 3;" ::: "memory");  // this batch's group is complete
+    asm volatile("cp.async.wait_group 3;" ::: "memory");  // this lane's copies of the batch are complete
+    __syncwarp();                                          // and so are the other lanes'
     const int64_t *d0 = dring + ((b - e0) / kDfBatch % (kDfDepth + 1)) * (kDfBatch * 32) + lane;
     const int n_here = e1 - b < kDfBatch ? (int)(e1 - b) : kDfBatch;
     // the batch's node ids, headers and durations in registers: their shuffles and
