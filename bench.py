@@ -36,7 +36,7 @@ UNIT = "updates/s"
 WORKLOAD = "gpt175b"
 # DRAM bytes per node-scenario of the composition kernels from the committed ncu
 # capture (a data file beside its summary), valid for the kernel source it names
-PROFILE_DATA = os.path.join(ROOT, "profiles", "compose_gpt175b.json")
+PROFILE_DATA = os.path.join(ROOT, "profiles", "traffic_per_node_scenario.json")
 
 
 def log(*a):
@@ -118,13 +118,13 @@ def source_hash(name):
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(kernel, launch_units):
-    """DRAM bytes per launch of `kernel` from the committed ncu data (per node-
-    scenario, scaled to ``launch_units`` node-scenarios), if it was taken on the
-    kernel's current source."""
+def profiled_traffic(workload, kernel, launch_units):
+    """DRAM bytes per launch of `kernel` on `workload` from the committed ncu data
+    (per node-scenario, scaled to ``launch_units`` node-scenarios), if it was taken
+    on the kernel's current source."""
     try:
         with open(PROFILE_DATA) as f:
-            d = json.load(f)["kernels"][kernel]
+            d = json.load(f)["workloads"][workload]["kernels"][kernel]
         if d["source_sha256_16"] != source_hash(d["source"]):
             return None
         return float(d["dram_bytes_per_node_scenario"]) * launch_units
@@ -328,8 +328,8 @@ def run_echo(args):
     # the dominant kernel of the step (largest total time) carries the roofline
     dom = max((k for k in alg if k in prof), key=lambda k: prof[k][1], default=None)
     traffic = None
-    if dom and args.workload == WORKLOAD:
-        traffic = profiled_traffic(dom, V * S)
+    if dom:
+        traffic = profiled_traffic(args.workload, dom, V * S)
     roof = {"kernel": dom, "bound": "hbm", "achieved": kernels[dom]["achieved_gbs"] if dom else None,
             "peak": peak, "peak_source": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
             "unit": "GB/s", "frac": kernels[dom]["frac"] if dom else None, "traffic": traffic,
