@@ -1958,9 +1958,11 @@ int echo_compose(echo_ctx *c, const echo_compose_opts *opts) {
     o.S = c->S;
     o.n_streams = B.NS;
     o.n_ranks = B.R;
-    {  // pieces of each rank's list: enough warps for about four waves (16 warps per
-       // SM), each piece at least 64 candidates long
-      const int64_t base = (int64_t)B.R * ((c->S + 31) / 32), want = 4 * 16 * (int64_t)c->sms;
+    {  // pieces of each rank's list: enough warps for about sixteen waves (16 warps
+       // per SM; shorter pieces even out the last wave: 9.27 -> 8.79 ms on the
+       // 1024-rank workload, 1.24 -> 1.09 ms on GPT-175B against four waves), each
+       // piece at least 64 candidates long
+      const int64_t base = (int64_t)B.R * ((c->S + 31) / 32), want = 16 * 16 * (int64_t)c->sms;
       const int64_t per_rank = B.n_cand / std::max<int32_t>(B.R, 1);
       o.parts = (int32_t)std::max<int64_t>(1, std::min((want + base - 1) / base, per_rank / 64));
     }
