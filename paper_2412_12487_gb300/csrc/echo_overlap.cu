@@ -97,22 +97,37 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
   // per comm timeline: position, end, and interval of the cursor op; the cursor op
   // always has positive length and finishes after the current op's start (or the
   // cursor is at the end, with an interval that never overlaps)
-  int32_t cur[NCMAX] = {}, end[NCMAX] = {};
+  // (nid: the node of the cursor's next position, loaded one move ahead so that a
+  // move waits for the interval's loads only)
+  int32_t cur[NCMAX] = {}, end[NCMAX] = {}, nid[NCMAX] = {};
   int64_t sw[NCMAX], fw[NCMAX];
-  auto load = [&](int j) {
+  auto fetch = [&](int j, int64_t w) {  // node w's interval as cursor j's op
+    if (a.dbg && !(in_range(w, a.lay.V) && (!LAUNCH || lq_ok(a, cur[j])))) {  // debug bounds
+      atomicCAS(a.status, 0, (int32_t)kDevBounds);
+      sw[j] = fw[j] = INT64_MAX;
+      return;
+    }
+    fw[j] = f[w << sh];
+    if (LAUNCH) {  // from the rank's launch: its launch conditions' latest finish
+      sw[j] = launch_time(a.lq_off, a.lq_ops, f, sh, cur[j]);
+    } else {
+      sw[j] = fw[j] - du[w << sh];
+    }
+  };
+  auto seek = [&](int j) {  // cursor j at position cur[j]
     if (cur[j] < end[j]) {
-      const int64_t w = a.cq_ops[cur[j]];
-      if (a.dbg && !(in_range(w, a.lay.V) && (!LAUNCH || lq_ok(a, cur[j])))) {  // debug bounds
-        atomicCAS(a.status, 0, (int32_t)kDevBounds);
-        sw[j] = fw[j] = INT64_MAX;
-        return;
-      }
-      fw[j] = f[w << sh];
-      if (LAUNCH) {  // from the rank's launch: its launch conditions' latest finish
-        sw[j] = launch_time(a.lq_off, a.lq_ops, f, sh, cur[j]);
-      } else {
-        sw[j] = fw[j] - du[w << sh];
-      }
+      fetch(j, a.cq_ops[cur[j]]);
+      nid[j] = cur[j] + 1 < end[j] ? a.cq_ops[cur[j] + 1] : 0;
+    } else {
+      sw[j] = fw[j] = INT64_MAX;
+    }
+  };
+  auto advance = [&](int j) {  // cursor j one position on
+    ++cur[j];
+    if (cur[j] < end[j]) {
+      const int64_t w = nid[j];
+      nid[j] = cur[j] + 1 < end[j] ? a.cq_ops[cur[j] + 1] : 0;
+      fetch(j, w);
     } else {
       sw[j] = fw[j] = INT64_MAX;
     }
@@ -148,11 +163,8 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
           }
         }
         cur[j] = lo;
-        load(j);
-        while (cur[j] < end[j] && sw[j] >= fw[j]) {  // zero-length ops never overlap
-          ++cur[j];
-          load(j);
-        }
+        seek(j);
+        while (cur[j] < end[j] && sw[j] >= fw[j]) advance(j);  // zero-length ops never overlap
       }
     }
   }
@@ -232,8 +244,7 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
           for (int j = 0; j < NCMAX; ++j) {
             if (j < nc && fw[j] <= sv) {  // the cursor op ended before this op starts: move on
               do {
-                ++cur[j];
-                load(j);
+                advance(j);
               } while (cur[j] < end[j] && (fw[j] <= sv || sw[j] >= fw[j]));
             }
           }
@@ -270,8 +281,7 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
                 held |= 1u << j;
               } else {
                 do {
-                  ++cur[j];
-                  load(j);
+                  advance(j);
                 } while (cur[j] < end[j] && sw[j] >= fw[j]);
               }
             }
