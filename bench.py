@@ -111,11 +111,15 @@ def measured_peaks():
 
 
 def source_hash(name):
-    """sha256[:16] of a kernel source file of the library."""
-    h = hashlib.sha256()
-    with open(os.path.join(ROOT, "paper_2412_12487_gb300", "csrc", name), "rb") as f:
-        h.update(f.read())
-    return h.hexdigest()[:16]
+    """sha256[:16] of a kernel source file of the library, comments and whitespace
+    left out (so that a change to the comments alone keeps a capture current)."""
+    import re
+    with open(os.path.join(ROOT, "paper_2412_12487_gb300", "csrc", name), encoding="utf-8") as f:
+        src = f.read()
+    src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", " ", src)
+    src = " ".join(src.split())
+    return hashlib.sha256(src.encode()).hexdigest()[:16]
 
 
 def profiled_traffic(workload, kernel, launch_units):

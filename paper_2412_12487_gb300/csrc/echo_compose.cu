@@ -203,10 +203,9 @@ __device__ __noinline__ bool segment_ok(const StagedArgs &a, uint32_t first, uin
 // word `ro`; its rows are i0 + header.z ... (global rows), held in the duration
 // ring of RR rows from ring row dpos0 + header.z on (wrapping).  Candidate rows of
 // the level start at level-order index c0, in ring row cpos0 of the CRR-row
-// candidate ring.  Thread `sub`
-// handles segments sub, sub + step, ... for scenario lanes j0 .. j0+LANES-1; the
-// segments of a level come heaviest first, so a warp's lanes hold segments of
-// similar weight.  Every input of a head is the tail of an earlier segment: the
+// candidate ring.  Thread `sub` handles segments sub, sub + step, ... for scenario
+// lanes j0 .. j0+LANES-1; the segments of a level come heaviest first, so a warp's
+// lanes hold segments of similar weight.  Every input of a head is the tail of an earlier segment: the
 // recent ones are read from the value ring (entries are byte offsets of their
 // slots), older ones from global memory (entries are node ids).  Inputs and
 // durations are loaded four at a time so that their latencies overlap.  This
@@ -499,9 +498,9 @@ __device__ __forceinline__ bool named_barrier_or(int id, int threads, bool flag)
 // compose, one scenario per thread up to SIGMA 8 (a segment's SIGMA threads
 // share its walk), two above.  The duration and candidate rings hold any number
 // of rows (a.d_rows, a.c_rows: all the shared memory the rest leaves), so the
-// producer writes each level's first ring rows beside its metadata.  Stage l % kPipeStages has a "full" mbarrier (armed with the level's
-// byte count) and an "empty" mbarrier (one arrival per consumer warp once the
-// level is composed).  Every wait is bounded: on expiry the block records
+// producer writes each level's first ring rows beside its metadata.  Stage
+// l % kPipeStages has a "full" mbarrier (armed with the level's byte count) and
+// an "empty" mbarrier (one arrival per consumer warp once the level is composed).  Every wait is bounded: on expiry the block records
 // kDevTimeout, stops, and lets its copies in flight land first.
 template <int SIGMA, bool STORE_ALL, bool DBG>
 __global__ void __launch_bounds__((kPipeConsumerWarps + 1) * 32)
