@@ -235,9 +235,15 @@ __global__ void __launch_bounds__(kOvWarps * 32, overlap_min_blocks(NCMAX)) over
     //    (and, proportional model, its covered length in place of its finish)
     uint32_t hits = 0;
     if (act) {
+      // (the next candidate's finish and duration load while this one is tested)
+      int64_t fn = slot[0], dn = slot[32];
 #pragma unroll 1
       for (int u = 0; u < n_here; ++u) {
-        const int64_t fv = slot[(2 * u) * 32], dv = slot[(2 * u + 1) * 32];
+        const int64_t fv = fn, dv = dn;
+        if (u + 1 < n_here) {
+          fn = slot[(2 * u + 2) * 32];
+          dn = slot[(2 * u + 3) * 32];
+        }
         const int64_t sv = fv - dv;
         if (fmin <= sv) {
 #pragma unroll
